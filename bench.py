@@ -1,0 +1,384 @@
+"""Throughput of HW-Router batched route scoring on GB300.
+
+One step = one hwr_route_batch call over one batch of synthetic queries: the
+whole hot path (feature assembly, latency predictor, cost, quality, SLO mask,
+argmax) for every (query, deployment) pair of the batch.
+
+Default workload: the large bf16 configuration -- Q = 65,536 queries,
+D = 64 deployments (16 models x 4 GPU types), 48 features, predictor
+48 -> 256 -> 256 -> 2, 1024-wide bf16 embeddings, lambda = 0.3, SLO = 10 s.
+
+Printed (one JSON line, rank 0):
+  value     routed queries/s with inputs resident in HBM (device pointers),
+            timed with CUDA events over K steps after W warm-up steps;
+  e2e       the same through the C ABI with pinned host buffers: the
+            host->device copy of the batch and the device->host copy of the
+            results are inside every timed step;
+  roofline  the dominant kernel's algorithmic FLOP (or bytes) per launch over
+            its CUDA-event duration, against the measured GB300 peak;
+  q1_latency_us  p50 / p99 single-query route latency through the C ABI with
+            host buffers, at D = 32 (the batch-sweep shape);
+  cpu_baseline   the CPU oracle on a bounded sample of the same workload.
+--impl reference times the CPU oracle (the reference arm for this build).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import workload as W  # noqa: E402
+
+L2_BYTES = 129 * 1024 * 1024
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0,
+                  "bf16_tflops_sustained": 1700.0, "sm_max_mhz": 2070.0}
+# fp32 SIMT peak: 152 SMs x 128 FP32 lanes x 2 flop (FMA) x max SM clock.
+SMS, FP32_LANES = 152, 128
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return d, "measured"
+    except (OSError, ValueError):
+        return dict(FALLBACK_PEAKS), "fallback"
+
+
+def workload_name(p):
+    return (f"{p['name']}: Q={p['Q']} D={p['D']} ({p['M']} models x {p['G']} GPU types) "
+            f"F={p['F']} MLP {p['F']}->{p['H1']}->{p['H2']}->2 E={p['E']} {p['dtype']} "
+            f"lambda={p['lam']} SLO={p['slo']}s")
+
+
+def flops_per_pair(p):
+    # layer 2 (2 H1 H2) + the two heads (2 * 2 H2) + the layer-1 query suffix
+    # (2 features x H1 x 2); the deployment prefix of layer 1 is per snapshot.
+    return 2 * p["H1"] * p["H2"] + 4 * p["H2"] + 4 * p["H1"]
+
+
+def bytes_per_query(p):
+    es = 2 if p["dtype"] == "bf16" else 4
+    return p["E"] * es + 8 + 12
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons, sampled during the timed region."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.file = None
+
+    def start(self):
+        try:
+            self.file = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=self.file, stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if not self.proc:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.file.flush()
+        self.file.seek(0)
+        rows = [l.split(",") for l in self.file.read().splitlines() if l.strip()]
+        os.unlink(self.file.name)
+        sm, mx, reasons = [], [], set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for r in rows:
+            if len(r) < 9:
+                continue
+            try:
+                sm.append(float(r[1]))
+                mx.append(float(r[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, r[5:9]):
+                if v.strip().lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx),
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def cpu_oracle_rate(p, seconds, nthreads):
+    """Queries/s of the oracle (fp64 mode) on a sample sized to ~`seconds`."""
+    import oracle as O
+    orc = O.Problem(p)
+    n = 32
+    t = time.perf_counter()
+    orc.route(p["in_len"][:n], p["out_len"][:n], p["emb"][:n], nthreads=nthreads)
+    per_q = (time.perf_counter() - t) / n
+    n = int(min(p["Q"], max(64, seconds / max(per_q, 1e-9))))
+    t = time.perf_counter()
+    orc.route(p["in_len"][:n], p["out_len"][:n], p["emb"][:n], nthreads=nthreads)
+    dt = time.perf_counter() - t
+    return n / dt, n, dt
+
+
+def run_reference(args, p):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return
+    cores = len(os.sched_getaffinity(0))
+    import oracle as O
+    orc = O.Problem(p)
+    # per-step sample sized to about 1.5 s of CPU work
+    t = time.perf_counter()
+    orc.route(p["in_len"][:32], p["out_len"][:32], p["emb"][:32], nthreads=cores)
+    per_q = (time.perf_counter() - t) / 32
+    S = int(min(p["Q"], max(32, 1.5 / max(per_q, 1e-9))))
+    for k in range(args.warmup):
+        lo = (k * S) % max(1, p["Q"] - S + 1)
+        orc.route(p["in_len"][lo:lo + S], p["out_len"][lo:lo + S], p["emb"][lo:lo + S],
+                  nthreads=cores)
+    t = time.perf_counter()
+    for k in range(args.steps):
+        lo = (k * S) % max(1, p["Q"] - S + 1)
+        orc.route(p["in_len"][lo:lo + S], p["out_len"][lo:lo + S], p["emb"][lo:lo + S],
+                  nthreads=cores)
+    dt = time.perf_counter() - t
+    v = S * args.steps / dt
+    line = {
+        "impl": "reference", "metric": "routed_queries_per_s", "value": v,
+        "unit": "queries/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": dt / args.steps * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": workload_name(p), "sample_queries_per_step": S},
+        "cpu_baseline": {"value": v, "unit": "queries/s", "cores": cores, "kind": "oracle",
+                         "sample": f"{S} queries of the workload per step, fp64 oracle, "
+                                   f"{cores} OpenMP threads"},
+        "e2e": {"value": v, "unit": "queries/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def q1_latency(H, iters=2000):
+    """p50/p99 of one-query routes through the C ABI with pinned host buffers."""
+    import torch
+    p = W.make_config(4, Q=1024)
+    r = H.Router(p)
+    il = torch.from_numpy(p["in_len"]).pin_memory()
+    ol = torch.from_numpy(p["out_len"]).pin_memory()
+    em = torch.from_numpy(p["emb"].view(np.int16)).pin_memory()
+    ch = torch.empty(1, dtype=torch.int32).pin_memory()
+    lat = torch.empty(1, dtype=torch.float32).pin_memory()
+    ut = torch.empty(1, dtype=torch.float32).pin_memory()
+    es = em.element_size() * p["E"]
+    times = []
+    for k in range(iters + 200):
+        i = k % p["Q"]
+        t = time.perf_counter()
+        r.route_host_ptrs(1, il.data_ptr() + 4 * i, ol.data_ptr() + 4 * i,
+                          em.data_ptr() + es * i, ch.data_ptr(), lat.data_ptr(),
+                          ut.data_ptr(), slo=p["slo"], lam=p["lam"])
+        if k >= 200:
+            times.append(time.perf_counter() - t)
+    r.close()
+    a = np.array(times) * 1e6
+    return {"p50": float(np.percentile(a, 50)), "p99": float(np.percentile(a, 99)),
+            "calls": iters, "config": "D=32 (8 models x 4 GPU types), MLP 48->256->256->2, "
+                                      "E=1024 bf16, host buffers, end to end",
+            "paper_routing_overhead_us": 200.0}
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="hwr", choices=["hwr", "reference"])
+    ap.add_argument("--config", type=int, default=3)
+    ap.add_argument("--q", type=int, default=None, help="override the query count")
+    ap.add_argument("--path", default="auto", choices=["auto", "simt", "tensor"])
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--no-q1", action="store_true")
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3)
+    rank, world, local = dist_env()
+
+    if args.impl == "reference":
+        if rank == 0:
+            p = W.make_config(args.config, Q=args.q, seed_offset=0)
+            run_reference(args, p)
+        return
+
+    import torch
+    import paper_2608_14575_gb300 as H
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    H.build()
+
+    p = W.make_config(args.config, Q=args.q, seed_offset=rank)
+    Q = p["Q"]
+    dev = torch.device("cuda", local)
+    stream = torch.cuda.current_stream()
+    r = H.Router(p, stream=stream.cuda_stream)
+    flags = {"auto": 0, "simt": H.HWR_PATH_SIMT, "tensor": H.HWR_PATH_TENSOR}[args.path]
+
+    emb_np = p["emb"].view(np.int16) if p["dtype"] == "bf16" else p["emb"]
+    in_bytes = Q * bytes_per_query(p)
+    nbuf = max(1, min(4, -(-3 * L2_BYTES // max(in_bytes, 1))))
+    bufs = []
+    for _ in range(nbuf):
+        bufs.append((torch.from_numpy(p["in_len"]).to(dev), torch.from_numpy(p["out_len"]).to(dev),
+                     torch.from_numpy(emb_np).to(dev)))
+    ch = torch.empty(Q, dtype=torch.int32, device=dev)
+    lat = torch.empty(Q, dtype=torch.float32, device=dev)
+    ut = torch.empty(Q, dtype=torch.float32, device=dev)
+
+    def step(k, extra=0):
+        il, ol, em = bufs[k % nbuf]
+        r.route_device(il, ol, em, ch, lat, ut, slo=p["slo"], lam=p["lam"],
+                       flags=flags | extra)
+
+    for k in range(args.warmup):
+        step(k)
+    torch.cuda.synchronize()
+    r.stats(reset=True)
+    before = r.stats()["kernel_launches"]
+    clocks = ClockSampler(local)
+    clocks.start()
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for k in range(args.steps):
+        step(k, H.HWR_PROFILE)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    clk = clocks.stop()
+    ms = e0.elapsed_time(e1) / args.steps
+    if dist:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    st = r.stats(reset=True)
+    launches = st["kernel_launches"] - before
+    value = world * Q / (ms * 1e-3)
+
+    # dominant kernel and its roofline
+    pk, src = peaks()
+    kms = {k: st["profiled_ms"][k] / max(1, st["profiled_launches"][k])
+           for k in H.KERNELS if st["profiled_launches"][k]}
+    top = max(kms, key=kms.get)
+    pairs = Q * p["D"]
+    if top == "mlp_tc":
+        flop = pairs * flops_per_pair(p)
+        ach = flop / (kms[top] * 1e-3) / 1e12
+        roof = {"bound": "tensor", "achieved": ach, "peak": pk["bf16_tflops"],
+                "unit": "TFLOP/s", "frac": ach / pk["bf16_tflops"], "traffic": None,
+                "kernel": top, "ms_per_launch": kms[top],
+                "peak_source": f"{src} bf16 burst (cuBLAS), frac vs sustained "
+                               f"{ach / pk.get('bf16_tflops_sustained', pk['bf16_tflops']):.3f}"}
+    elif top == "qual_tc":
+        byt = Q * bytes_per_query(p)
+        ach = byt / (kms[top] * 1e-3) / 1e9
+        roof = {"bound": "hbm", "achieved": ach, "peak": pk["hbm_gbs"], "unit": "GB/s",
+                "frac": ach / pk["hbm_gbs"], "traffic": None, "kernel": top,
+                "ms_per_launch": kms[top], "peak_source": f"{src} copy bandwidth"}
+    else:
+        flop = pairs * flops_per_pair(p)
+        peak = SMS * FP32_LANES * 2 * pk.get("sm_max_mhz", 2070.0) * 1e6 / 1e12
+        ach = flop / (kms[top] * 1e-3) / 1e12
+        roof = {"bound": "alu", "achieved": ach, "peak": peak, "unit": "TFLOP/s",
+                "frac": ach / peak, "traffic": None, "kernel": top, "ms_per_launch": kms[top],
+                "peak_source": "fp32 FMA: 152 SMs x 128 lanes x 2 x max SM clock"}
+
+    line = {
+        "metric": "routed_queries_per_s", "value": value, "unit": "queries/s",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": p["dtype"], "data": "synthetic (seeded; shapes and distributions of the "
+                                     "paper's workload stand-ins)",
+        "config": {"workload": workload_name(p), "queries_per_gpu": Q,
+                   "path": args.path,
+                   "l2": f"{nbuf} input buffers of {in_bytes / 2**20:.0f} MiB rotated per step "
+                         f"({'inputs > L2' if in_bytes > L2_BYTES else 'rotation > L2'})",
+                   "parallelism": f"replicas x{world} (queries sharded, no collective)"},
+        "kernel_ms": kms, "gpu_launches": launches, "roofline": roof, "clocks": clk,
+    }
+
+    if not args.no_e2e:
+        pin = (torch.from_numpy(p["in_len"]).pin_memory(), torch.from_numpy(p["out_len"]).pin_memory(),
+               torch.from_numpy(emb_np).pin_memory())
+        och = torch.empty(Q, dtype=torch.int32).pin_memory()
+        olat = torch.empty(Q, dtype=torch.float32).pin_memory()
+        out_ = torch.empty(Q, dtype=torch.float32).pin_memory()
+
+        def host_step():
+            r.route_host_ptrs(Q, pin[0].data_ptr(), pin[1].data_ptr(), pin[2].data_ptr(),
+                              och.data_ptr(), olat.data_ptr(), out_.data_ptr(),
+                              slo=p["slo"], lam=p["lam"], flags=flags)
+        for _ in range(args.warmup):
+            host_step()
+        if dist:
+            dist.barrier()
+        t = time.perf_counter()
+        for _ in range(args.steps):
+            host_step()
+        dt = (time.perf_counter() - t) / args.steps
+        if dist:
+            tt = torch.tensor([dt], device=dev)
+            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+            dt = float(tt.item())
+        line["e2e"] = {"value": world * Q / dt, "unit": "queries/s",
+                       "h2d_bytes_per_step": Q * (bytes_per_query(p) - 12),
+                       "d2h_bytes_per_step": Q * 12, "ms_per_step": dt * 1e3}
+    if rank == 0 and not args.no_q1:
+        line["q1_latency_us"] = q1_latency(H)
+    if rank == 0 and not args.no_cpu:
+        cores = len(os.sched_getaffinity(0))
+        v, n, dt = cpu_oracle_rate(p, 10.0, cores)
+        line["cpu_baseline"] = {"value": v, "unit": "queries/s", "cores": cores,
+                                "kind": "oracle",
+                                "sample": f"first {n} queries of the workload, fp64 oracle, "
+                                          f"{cores} OpenMP threads, {dt:.1f} s"}
+    r.close()
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if dist:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,725 @@
+// C-ABI host code of the route-scoring library (declarations in include/hwr.h).
+//
+// Owns the context: device copies of the deployment table, the predictor
+// (fp32 copies for the SIMT kernels, bf16 shared-memory images for the
+// tcgen05 kernels), the model embeddings and the hardware snapshot; grow-only
+// scratch and I/O staging; and the dispatch of each call onto the kernels of
+// k_simt.cu and k_tc.cu on the context stream.
+#include <math.h>
+#include <stdarg.h>
+#include <stdio.h>
+#include <stdlib.h>
+#include <string.h>
+
+#include <string>
+#include <vector>
+
+#include "hwr_internal.cuh"
+
+using namespace hwr;
+
+namespace {
+
+thread_local std::string g_create_error;
+
+// Host-side fault hook for tests: HWR_TEST_FAIL_ALLOC=n makes the n-th
+// allocation of a context (counting from 1) report failure.
+struct AllocHook {
+    long fail_at = 0, count = 0;
+};
+
+constexpr int TC_MIN_Q = 512;  // below this the fused SIMT kernel is faster
+
+}  // namespace
+
+struct hwr_ctx {
+    int M = 0, G = 0, D = 0, F = 0, H1 = 0, H2 = 0, E = 0, P = 0;
+    int Mpad = 0, Epad = 0;
+    hwr_dtype dtype = HWR_F32;
+    bool tc_ok = false;
+    cudaStream_t stream = nullptr;
+    bool own_stream = false;
+    bool broken = false;
+    bool have_snapshot = false;
+    std::string err;
+    AllocHook hook;
+    std::vector<void *> allocs;  // device buffers (cudaMalloc)
+
+    // device state
+    int32_t *dep_model = nullptr, *dep_gpu = nullptr;
+    float *log10p = nullptr;
+    float *W1 = nullptr, *b1 = nullptr, *W2 = nullptr, *b2 = nullptr;
+    float *W3 = nullptr, *b3 = nullptr, *mu = nullptr, *sd = nullptr;
+    uint8_t *xform = nullptr;
+    float *memb = nullptr;
+    float *W1q = nullptr;            // [2][H1]
+    uint16_t *W2img = nullptr, *membimg = nullptr;
+    int32_t *running = nullptr, *waiting = nullptr;
+    float *kv = nullptr, *gpu_util = nullptr, *ttft = nullptr, *tpot = nullptr;
+    float *X = nullptr, *Spre = nullptr, *A = nullptr;
+    // host feature constants for the tensor path
+    float mu_in = 0, sd_in = 1, mu_out = 0, sd_out = 1;
+    uint8_t xf_in = 0, xf_out = 0;
+
+    // mapped pinned status word written by kernels with bounded waits
+    int32_t *status_h = nullptr, *status_d = nullptr;
+
+    // snapshot staging (pinned) and its copy-done event
+    void *snap_h = nullptr;
+    void *snap_d = nullptr;
+    cudaEvent_t snap_ev = nullptr;
+
+    // grow-only scratch
+    float *qual = nullptr;   size_t qual_cap = 0;     // [Q][Mpad]
+    float *ctab = nullptr;   size_t ctab_cap = 0;
+    float *qseq = nullptr;   size_t qseq_cap = 0;
+    int seq_qs = 0;
+
+    // I/O staging for host pointers: device [emb | in | out] and [chosen | lat | util]
+    char *io_d = nullptr;    size_t io_cap = 0;
+    char *out_d = nullptr;   size_t out_cap = 0;
+    char *pin_h = nullptr;   size_t pin_cap = 0;       // pinned host staging
+    cudaEvent_t pin_ev = nullptr;
+
+    // profiling
+    struct Pending { int k; cudaEvent_t a, b; };
+    std::vector<Pending> pending;
+    std::vector<cudaEvent_t> ev_pool;
+    hwr_stats stats;
+};
+
+// ---------------------------------------------------------------------------
+// helpers
+
+static hwr_status fail(hwr_ctx *c, hwr_status s, const char *fmt, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    if (c) {
+        c->err = buf;
+        if (s == HWR_ERR_CUDA || s == HWR_ERR_TIMEOUT) c->broken = true;
+    } else {
+        g_create_error = buf;
+    }
+    return s;
+}
+
+static hwr_status cuda_fail(hwr_ctx *c, cudaError_t e, const char *what) {
+    return fail(c, e == cudaErrorMemoryAllocation ? HWR_ERR_OOM : HWR_ERR_CUDA,
+                "%s: %s", what, cudaGetErrorString(e));
+}
+
+#define CK(ctx, call, what)                                   \
+    do {                                                      \
+        cudaError_t e_ = (call);                              \
+        if (e_ != cudaSuccess) return cuda_fail(ctx, e_, what); \
+    } while (0)
+
+static bool hook_fires(hwr_ctx *c) {
+    return c->hook.fail_at > 0 && ++c->hook.count == c->hook.fail_at;
+}
+
+template <class T>
+static hwr_status dev_alloc(hwr_ctx *c, T **p, size_t n) {
+    *p = nullptr;
+    if (n == 0) n = 1;
+    if (hook_fires(c)) return fail(c, HWR_ERR_OOM, "allocation %ld failed (test hook)", c->hook.count);
+    void *q = nullptr;
+    cudaError_t e = cudaMalloc(&q, n * sizeof(T));
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        return fail(c, HWR_ERR_OOM, "cudaMalloc(%zu): %s", n * sizeof(T), cudaGetErrorString(e));
+    }
+    c->allocs.push_back(q);
+    *p = (T *)q;
+    return HWR_OK;
+}
+
+static void dev_free(hwr_ctx *c, void *p) {
+    if (!p) return;
+    for (size_t i = 0; i < c->allocs.size(); ++i)
+        if (c->allocs[i] == p) {
+            c->allocs.erase(c->allocs.begin() + i);
+            break;
+        }
+    cudaFree(p);
+}
+
+// Grow a scratch buffer to hold n elements (contents not preserved).
+template <class T>
+static hwr_status grow(hwr_ctx *c, T **p, size_t *cap, size_t n) {
+    if (n <= *cap && *p) return HWR_OK;
+    size_t want = n + n / 4 + 64;
+    if (*p) {
+        cudaError_t e = cudaStreamSynchronize(c->stream);
+        if (e != cudaSuccess) return cuda_fail(c, e, "synchronize before regrow");
+        dev_free(c, *p);
+        *p = nullptr;
+        *cap = 0;
+    }
+    hwr_status s = dev_alloc(c, p, want);
+    if (s == HWR_OK) *cap = want;
+    return s;
+}
+
+static hwr_status pin_grow(hwr_ctx *c, size_t bytes) {
+    if (bytes <= c->pin_cap && c->pin_h) return HWR_OK;
+    if (c->pin_h) {
+        cudaStreamSynchronize(c->stream);
+        cudaFreeHost(c->pin_h);
+        c->pin_h = nullptr;
+        c->pin_cap = 0;
+    }
+    size_t want = bytes + bytes / 4 + 4096;
+    if (hook_fires(c)) return fail(c, HWR_ERR_OOM, "allocation %ld failed (test hook)", c->hook.count);
+    cudaError_t e = cudaHostAlloc((void **)&c->pin_h, want, cudaHostAllocDefault);
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        c->pin_h = nullptr;
+        return fail(c, HWR_ERR_OOM, "cudaHostAlloc(%zu): %s", want, cudaGetErrorString(e));
+    }
+    c->pin_cap = want;
+    return HWR_OK;
+}
+
+static float bf16_bits_to_f32(uint16_t b) {
+    uint32_t u = (uint32_t)b << 16;
+    float f;
+    memcpy(&f, &u, 4);
+    return f;
+}
+
+static Model model_view(const hwr_ctx *c) {
+    Model m;
+    m.M = c->M; m.G = c->G; m.D = c->D; m.F = c->F; m.H1 = c->H1; m.H2 = c->H2;
+    m.E = c->E; m.P = c->P;
+    m.dep_model = c->dep_model; m.dep_gpu = c->dep_gpu; m.log10p = c->log10p;
+    m.W1 = c->W1; m.b1 = c->b1; m.W2 = c->W2; m.b2 = c->b2; m.W3 = c->W3; m.b3 = c->b3;
+    m.mu = c->mu; m.sd = c->sd; m.xform = c->xform; m.memb = c->memb;
+    m.running = c->running; m.waiting = c->waiting; m.kv = c->kv;
+    m.gpu_util = c->gpu_util; m.ttft = c->ttft; m.tpot = c->tpot;
+    m.X = c->X; m.Spre = c->Spre; m.A = c->A;
+    return m;
+}
+
+static TcModel tc_view(const hwr_ctx *c) {
+    TcModel t;
+    t.M = c->M; t.Mpad = c->Mpad; t.D = c->D; t.H1 = c->H1; t.H2 = c->H2;
+    t.E = c->E; t.Epad = c->Epad;
+    t.W2img = c->W2img; t.membimg = c->membimg; t.A = c->A; t.W1q = c->W1q;
+    t.b2 = c->b2; t.W3 = c->W3; t.b3 = c->b3; t.dep_model = c->dep_model;
+    t.mu_in = c->mu_in; t.sd_in = c->sd_in; t.mu_out = c->mu_out; t.sd_out = c->sd_out;
+    t.xf_in = c->xf_in; t.xf_out = c->xf_out;
+    return t;
+}
+
+// Profiling: bracket a launch with events when asked.
+static cudaEvent_t take_event(hwr_ctx *c) {
+    if (!c->ev_pool.empty()) {
+        cudaEvent_t e = c->ev_pool.back();
+        c->ev_pool.pop_back();
+        return e;
+    }
+    cudaEvent_t e = nullptr;
+    if (cudaEventCreate(&e) != cudaSuccess) {
+        cudaGetLastError();
+        return nullptr;
+    }
+    return e;
+}
+
+struct LaunchScope {
+    hwr_ctx *c;
+    int k;
+    bool prof;
+    cudaEvent_t a = nullptr;
+    LaunchScope(hwr_ctx *c_, int k_, bool prof_) : c(c_), k(k_), prof(prof_) {
+        if (prof && (a = take_event(c))) cudaEventRecord(a, c->stream);
+    }
+    void done() {
+        c->stats.kernel_launches++;
+        c->stats.launches[k]++;
+        if (prof && a) {
+            cudaEvent_t b = take_event(c);
+            if (b) {
+                cudaEventRecord(b, c->stream);
+                c->pending.push_back({k, a, b});
+            } else {
+                c->ev_pool.push_back(a);
+            }
+        }
+    }
+};
+
+static hwr_status collect_profile(hwr_ctx *c) {
+    if (c->pending.empty()) return HWR_OK;
+    CK(c, cudaStreamSynchronize(c->stream), "synchronize for profile");
+    for (auto &p : c->pending) {
+        float ms = 0.f;
+        if (cudaEventElapsedTime(&ms, p.a, p.b) == cudaSuccess) {
+            c->stats.profiled_ms[p.k] += ms;
+            c->stats.profiled_launches[p.k]++;
+        } else {
+            cudaGetLastError();
+        }
+        c->ev_pool.push_back(p.a);
+        c->ev_pool.push_back(p.b);
+    }
+    c->pending.clear();
+    return HWR_OK;
+}
+
+static hwr_status check_status_word(hwr_ctx *c) {
+    int32_t st = *(volatile int32_t *)c->status_h;
+    if (st == ST_TIMEOUT)
+        return fail(c, HWR_ERR_TIMEOUT, "a device-side wait exceeded its bound (kernel gave up)");
+    if (st != ST_OK) return fail(c, HWR_ERR_CUDA, "kernel reported status %d", st);
+    return HWR_OK;
+}
+
+// ---------------------------------------------------------------------------
+// create / destroy
+
+static hwr_status validate_create(const hwr_deployment_table *t, const hwr_predictor *p,
+                                  const void *memb, int32_t E, hwr_dtype edt) {
+    if (!t || !p || !memb) return fail(nullptr, HWR_ERR_INVALID_ARG, "NULL table, predictor or model_emb");
+    if (!t->dep_model || !t->dep_gpu || !t->model_log10_params)
+        return fail(nullptr, HWR_ERR_INVALID_ARG, "NULL array in deployment table");
+    if (!p->W1 || !p->W2 || !p->W3 || !p->b1 || !p->b2 || !p->b3 || !p->feat_mean ||
+        !p->feat_std || !p->feat_xform)
+        return fail(nullptr, HWR_ERR_INVALID_ARG, "NULL array in predictor");
+    const int M = t->n_models, G = t->n_gpu_types, D = t->n_deployments;
+    if (M < 1 || G < 1 || D < 1) return fail(nullptr, HWR_ERR_INVALID_ARG, "M, G and D must be >= 1");
+    if (p->dtype != HWR_F32 && p->dtype != HWR_BF16)
+        return fail(nullptr, HWR_ERR_INVALID_ARG, "unknown predictor dtype %d", (int)p->dtype);
+    if (edt != p->dtype)
+        return fail(nullptr, HWR_ERR_DTYPE, "embedding dtype %d differs from predictor dtype %d",
+                    (int)edt, (int)p->dtype);
+    if (p->F < M + G + 9) return fail(nullptr, HWR_ERR_INVALID_ARG, "F=%d < M+G+9=%d", p->F, M + G + 9);
+    if (E < 8 || E % 8) return fail(nullptr, HWR_ERR_INVALID_ARG, "E=%d must be a multiple of 8, >= 8", E);
+    if (p->H1 < 1 || p->H2 < 1) return fail(nullptr, HWR_ERR_INVALID_ARG, "H1, H2 must be >= 1");
+    if (D > MAX_D) return fail(nullptr, HWR_ERR_UNSUPPORTED, "D=%d > %d", D, MAX_D);
+    if (p->H1 > MAX_H || p->H2 > MAX_H) return fail(nullptr, HWR_ERR_UNSUPPORTED, "H1/H2 > %d", MAX_H);
+    if (p->F > 256) return fail(nullptr, HWR_ERR_UNSUPPORTED, "F=%d > 256", p->F);
+    if (E > 8192) return fail(nullptr, HWR_ERR_UNSUPPORTED, "E=%d > 8192", E);
+    if (M > 64) return fail(nullptr, HWR_ERR_UNSUPPORTED, "M=%d > 64", M);
+    for (int d = 0; d < D; ++d) {
+        if (t->dep_model[d] < 0 || t->dep_model[d] >= M || t->dep_gpu[d] < 0 || t->dep_gpu[d] >= G)
+            return fail(nullptr, HWR_ERR_INVALID_ARG, "deployment %d: model/gpu id out of range", d);
+    }
+    for (int k = 0; k < p->F; ++k) {
+        if (!(p->feat_std[k] != 0.f) || !isfinite(p->feat_std[k]) || !isfinite(p->feat_mean[k]))
+            return fail(nullptr, HWR_ERR_INVALID_ARG, "feature %d: std must be finite and non-zero", k);
+        if (p->feat_xform[k] > 2) return fail(nullptr, HWR_ERR_INVALID_ARG, "feature %d: xform > 2", k);
+    }
+    return HWR_OK;
+}
+
+static hwr_status upload(hwr_ctx *c, void *dst, const void *src, size_t bytes, const char *what) {
+    CK(c, cudaMemcpy(dst, src, bytes, cudaMemcpyHostToDevice), what);
+    return HWR_OK;
+}
+
+#define TRY(x)                          \
+    do {                                \
+        hwr_status s_ = (x);            \
+        if (s_ != HWR_OK) return s_;    \
+    } while (0)
+
+static hwr_status build_ctx(hwr_ctx *c, const hwr_deployment_table *t, const hwr_predictor *p,
+                            const void *memb_in, void *stream) {
+    const int M = c->M, D = c->D, F = c->F, H1 = c->H1, H2 = c->H2, E = c->E;
+    const bool bf = c->dtype == HWR_BF16;
+    if (stream) {
+        c->stream = (cudaStream_t)stream;
+    } else {
+        CK(c, cudaStreamCreateWithFlags(&c->stream, cudaStreamNonBlocking), "create stream");
+        c->own_stream = true;
+    }
+    CK(c, simt_prepare(), "configure SIMT kernels");
+
+    // fp32 copies of every weight (bf16 widened exactly)
+    auto widen = [&](const void *src, size_t n) {
+        std::vector<float> v(n);
+        if (bf) {
+            const uint16_t *s = (const uint16_t *)src;
+            for (size_t i = 0; i < n; ++i) v[i] = bf16_bits_to_f32(s[i]);
+        } else {
+            memcpy(v.data(), src, n * sizeof(float));
+        }
+        return v;
+    };
+    std::vector<float> w1 = widen(p->W1, (size_t)H1 * F), w2 = widen(p->W2, (size_t)H2 * H1),
+                       w3 = widen(p->W3, (size_t)2 * H2), me = widen(memb_in, (size_t)E * M);
+
+    TRY(dev_alloc(c, &c->dep_model, D));
+    TRY(dev_alloc(c, &c->dep_gpu, D));
+    TRY(dev_alloc(c, &c->log10p, M));
+    TRY(dev_alloc(c, &c->W1, w1.size()));
+    TRY(dev_alloc(c, &c->b1, H1));
+    TRY(dev_alloc(c, &c->W2, w2.size()));
+    TRY(dev_alloc(c, &c->b2, H2));
+    TRY(dev_alloc(c, &c->W3, w3.size()));
+    TRY(dev_alloc(c, &c->b3, 2));
+    TRY(dev_alloc(c, &c->mu, F));
+    TRY(dev_alloc(c, &c->sd, F));
+    TRY(dev_alloc(c, &c->xform, F));
+    TRY(dev_alloc(c, &c->memb, me.size()));
+    TRY(dev_alloc(c, &c->W1q, 2 * (size_t)H1));
+    TRY(dev_alloc(c, &c->running, D));
+    TRY(dev_alloc(c, &c->waiting, D));
+    TRY(dev_alloc(c, &c->kv, D));
+    TRY(dev_alloc(c, &c->gpu_util, D));
+    TRY(dev_alloc(c, &c->ttft, D));
+    TRY(dev_alloc(c, &c->tpot, D));
+    TRY(dev_alloc(c, &c->X, (size_t)D * F));
+    TRY(dev_alloc(c, &c->Spre, (size_t)D * H1));
+    TRY(dev_alloc(c, &c->A, (size_t)D * H1));
+
+    TRY(upload(c, c->dep_model, t->dep_model, D * 4, "upload table"));
+    TRY(upload(c, c->dep_gpu, t->dep_gpu, D * 4, "upload table"));
+    TRY(upload(c, c->log10p, t->model_log10_params, M * 4, "upload table"));
+    TRY(upload(c, c->W1, w1.data(), w1.size() * 4, "upload W1"));
+    TRY(upload(c, c->b1, p->b1, H1 * 4, "upload b1"));
+    TRY(upload(c, c->W2, w2.data(), w2.size() * 4, "upload W2"));
+    TRY(upload(c, c->b2, p->b2, H2 * 4, "upload b2"));
+    TRY(upload(c, c->W3, w3.data(), w3.size() * 4, "upload W3"));
+    TRY(upload(c, c->b3, p->b3, 8, "upload b3"));
+    TRY(upload(c, c->mu, p->feat_mean, F * 4, "upload mean"));
+    TRY(upload(c, c->sd, p->feat_std, F * 4, "upload std"));
+    TRY(upload(c, c->xform, p->feat_xform, F, "upload xform"));
+    TRY(upload(c, c->memb, me.data(), me.size() * 4, "upload model embeddings"));
+    std::vector<float> w1q(2 * (size_t)H1);
+    for (int j = 0; j < H1; ++j) {
+        w1q[j] = w1[(size_t)j * F + F - 2];
+        w1q[H1 + j] = w1[(size_t)j * F + F - 1];
+    }
+    TRY(upload(c, c->W1q, w1q.data(), w1q.size() * 4, "upload W1 query columns"));
+    c->mu_in = p->feat_mean[F - 2]; c->sd_in = p->feat_std[F - 2]; c->xf_in = p->feat_xform[F - 2];
+    c->mu_out = p->feat_mean[F - 1]; c->sd_out = p->feat_std[F - 1]; c->xf_out = p->feat_xform[F - 1];
+
+    CK(c, cudaMemset(c->running, 0, D * 4), "zero snapshot");
+    CK(c, cudaMemset(c->waiting, 0, D * 4), "zero snapshot");
+    CK(c, cudaMemset(c->kv, 0, D * 4), "zero snapshot");
+    CK(c, cudaMemset(c->gpu_util, 0, D * 4), "zero snapshot");
+    CK(c, cudaMemset(c->ttft, 0, D * 4), "zero snapshot");
+    CK(c, cudaMemset(c->tpot, 0, D * 4), "zero snapshot");
+
+    // tensor-core images (bf16 only)
+    c->Mpad = M <= 16 ? 16 : 32;
+    c->Epad = (E + 63) / 64 * 64;
+    c->tc_ok = bf && tc_supported(M, H1, H2, E);
+    if (c->tc_ok) {
+        CK(c, tc_prepare(), "configure tensor-core kernels");
+        std::vector<uint16_t> img(tc_w2img_elems(H1, H2));
+        tc_build_w2img((const uint16_t *)p->W2, H1, H2, img.data());
+        TRY(dev_alloc(c, &c->W2img, img.size()));
+        TRY(upload(c, c->W2img, img.data(), img.size() * 2, "upload W2 image"));
+        std::vector<uint16_t> mimg(tc_membimg_elems(c->Mpad, c->Epad));
+        tc_build_membimg((const uint16_t *)memb_in, E, M, c->Mpad, c->Epad, mimg.data());
+        TRY(dev_alloc(c, &c->membimg, mimg.size()));
+        TRY(upload(c, c->membimg, mimg.data(), mimg.size() * 2, "upload memb image"));
+    }
+
+    // status word: mapped pinned host memory the kernels write directly
+    if (hook_fires(c)) return fail(c, HWR_ERR_OOM, "allocation %ld failed (test hook)", c->hook.count);
+    CK(c, cudaHostAlloc((void **)&c->status_h, 64, cudaHostAllocMapped), "alloc status word");
+    memset(c->status_h, 0, 64);
+    CK(c, cudaHostGetDevicePointer((void **)&c->status_d, c->status_h, 0), "map status word");
+
+    // snapshot staging: 6 arrays of D 4-byte values
+    if (hook_fires(c)) return fail(c, HWR_ERR_OOM, "allocation %ld failed (test hook)", c->hook.count);
+    CK(c, cudaHostAlloc(&c->snap_h, 6 * (size_t)D * 4, cudaHostAllocDefault), "alloc snapshot staging");
+    TRY(dev_alloc(c, (char **)&c->snap_d, 6 * (size_t)D * 4));
+    CK(c, cudaEventCreateWithFlags(&c->snap_ev, cudaEventDisableTiming), "create event");
+    CK(c, cudaEventCreateWithFlags(&c->pin_ev, cudaEventDisableTiming), "create event");
+
+    c->seq_qs = seq_chunk(model_view(c));
+    CK(c, cudaDeviceSynchronize(), "create");
+    return HWR_OK;
+}
+
+static void free_ctx(hwr_ctx *c) {
+    if (c->stream) cudaStreamSynchronize(c->stream);
+    for (auto &p : c->pending) {
+        cudaEventDestroy(p.a);
+        cudaEventDestroy(p.b);
+    }
+    for (auto e : c->ev_pool) cudaEventDestroy(e);
+    for (void *p : c->allocs) cudaFree(p);
+    c->allocs.clear();
+    if (c->status_h) cudaFreeHost(c->status_h);
+    if (c->snap_h) cudaFreeHost(c->snap_h);
+    if (c->pin_h) cudaFreeHost(c->pin_h);
+    if (c->snap_ev) cudaEventDestroy(c->snap_ev);
+    if (c->pin_ev) cudaEventDestroy(c->pin_ev);
+    if (c->own_stream && c->stream) cudaStreamDestroy(c->stream);
+    cudaGetLastError();
+    delete c;
+}
+
+extern "C" hwr_status hwr_create(const hwr_deployment_table *table, const hwr_predictor *pred,
+                                 const void *model_emb, int32_t E, hwr_dtype emb_dtype,
+                                 void *cuda_stream, hwr_ctx **out) {
+    if (!out) return fail(nullptr, HWR_ERR_INVALID_ARG, "out is NULL");
+    *out = nullptr;
+    g_create_error.clear();
+    hwr_status s = validate_create(table, pred, model_emb, E, emb_dtype);
+    if (s != HWR_OK) return s;
+    hwr_ctx *c = new (std::nothrow) hwr_ctx();
+    if (!c) return fail(nullptr, HWR_ERR_OOM, "host allocation failed");
+    memset(&c->stats, 0, sizeof c->stats);
+    c->M = table->n_models; c->G = table->n_gpu_types; c->D = table->n_deployments;
+    c->F = pred->F; c->H1 = pred->H1; c->H2 = pred->H2; c->E = E; c->P = c->M + c->G;
+    c->dtype = pred->dtype;
+    if (const char *h = getenv("HWR_TEST_FAIL_ALLOC")) c->hook.fail_at = atol(h);
+    s = build_ctx(c, table, pred, model_emb, cuda_stream);
+    if (s != HWR_OK) {
+        g_create_error = c->err;
+        free_ctx(c);
+        return s;
+    }
+    *out = c;
+    return HWR_OK;
+}
+
+extern "C" hwr_status hwr_destroy(hwr_ctx *c) {
+    if (c) free_ctx(c);
+    return HWR_OK;
+}
+
+// ---------------------------------------------------------------------------
+// snapshot
+
+extern "C" hwr_status hwr_update_snapshot(hwr_ctx *c, const hwr_snapshot *s) {
+    if (!c) return fail(nullptr, HWR_ERR_INVALID_ARG, "ctx is NULL");
+    if (c->broken) return HWR_ERR_STATE;
+    if (!s || !s->running || !s->waiting || !s->kv_util || !s->gpu_util || !s->ttft_avg ||
+        !s->tpot_avg)
+        return fail(c, HWR_ERR_INVALID_ARG, "NULL snapshot array");
+    const size_t n = (size_t)c->D * 4;
+    // the previous snapshot copy must have left the staging buffer
+    CK(c, cudaEventSynchronize(c->snap_ev), "wait for snapshot staging");
+    char *h = (char *)c->snap_h;
+    memcpy(h + 0 * n, s->running, n);
+    memcpy(h + 1 * n, s->waiting, n);
+    memcpy(h + 2 * n, s->kv_util, n);
+    memcpy(h + 3 * n, s->gpu_util, n);
+    memcpy(h + 4 * n, s->ttft_avg, n);
+    memcpy(h + 5 * n, s->tpot_avg, n);
+    CK(c, cudaMemcpyAsync(c->snap_d, h, 6 * n, cudaMemcpyHostToDevice, c->stream), "copy snapshot");
+    CK(c, cudaEventRecord(c->snap_ev, c->stream), "record");
+    const char *d = (const char *)c->snap_d;
+    CK(c, cudaMemcpyAsync(c->running, d + 0 * n, n, cudaMemcpyDeviceToDevice, c->stream), "snapshot");
+    CK(c, cudaMemcpyAsync(c->waiting, d + 1 * n, n, cudaMemcpyDeviceToDevice, c->stream), "snapshot");
+    CK(c, cudaMemcpyAsync(c->kv, d + 2 * n, n, cudaMemcpyDeviceToDevice, c->stream), "snapshot");
+    CK(c, cudaMemcpyAsync(c->gpu_util, d + 3 * n, n, cudaMemcpyDeviceToDevice, c->stream), "snapshot");
+    CK(c, cudaMemcpyAsync(c->ttft, d + 4 * n, n, cudaMemcpyDeviceToDevice, c->stream), "snapshot");
+    CK(c, cudaMemcpyAsync(c->tpot, d + 5 * n, n, cudaMemcpyDeviceToDevice, c->stream), "snapshot");
+    LaunchScope ls(c, HWR_K_SNAPSHOT, false);
+    CK(c, launch_snapshot(model_view(c), c->stream), "snapshot kernel");
+    ls.done();
+    c->have_snapshot = true;
+    return HWR_OK;
+}
+
+extern "C" hwr_status hwr_get_snapshot(hwr_ctx *c, int32_t *running_out) {
+    if (!c) return fail(nullptr, HWR_ERR_INVALID_ARG, "ctx is NULL");
+    if (c->broken) return HWR_ERR_STATE;
+    if (!running_out) return fail(c, HWR_ERR_INVALID_ARG, "running_out is NULL");
+    CK(c, cudaMemcpyAsync(running_out, c->running, (size_t)c->D * 4, cudaMemcpyDeviceToHost,
+                          c->stream), "read running counts");
+    CK(c, cudaStreamSynchronize(c->stream), "synchronize");
+    return HWR_OK;
+}
+
+// ---------------------------------------------------------------------------
+// routing
+
+static hwr_status run_kernels(hwr_ctx *c, const Queries &q, uint32_t flags, bool tensor) {
+    const bool prof = flags & HWR_PROFILE;
+    const Model m = model_view(c);
+    if (flags & HWR_SEQUENTIAL) {
+        const int Qs = c->seq_qs;
+        TRY(grow(c, &c->ctab, &c->ctab_cap, seq_table_floats(c->D, Qs)));
+        TRY(grow(c, &c->qseq, &c->qseq_cap, (size_t)Qs * c->M));
+        const size_t es = c->dtype == HWR_BF16 ? 2 : 4;
+        for (int lo = 0; lo < q.Q; lo += Qs) {
+            Queries k = q;
+            const int n = q.Q - lo < Qs ? q.Q - lo : Qs;
+            k.Q = n;
+            k.in_len = q.in_len + lo;
+            k.out_len = q.out_len + lo;
+            k.emb = (const char *)q.emb + (size_t)lo * c->E * es;
+            k.chosen = q.chosen + lo;
+            k.lat = q.lat + lo;
+            k.util = q.util + lo;
+            LaunchScope a(c, HWR_K_SEQ_TABLE, prof);
+            CK(c, launch_seq_table(m, k, n, c->ctab, c->qseq, c->stream), "sequential table");
+            a.done();
+            CK(c, launch_seq_chain(m, k, n, c->ctab, c->qseq, c->stream), "sequential chain");
+            c->stats.kernel_launches++;
+            c->stats.launches[HWR_K_SEQ_TABLE]++;
+        }
+        return HWR_OK;
+    }
+    if (tensor) {
+        const TcModel t = tc_view(c);
+        TRY(grow(c, &c->qual, &c->qual_cap, (size_t)q.Q * c->Mpad));
+        LaunchScope a(c, HWR_K_QUAL_TC, prof);
+        CK(c, launch_qual_tc(t, q, c->qual, c->status_d, c->stream), "quality kernel");
+        a.done();
+        LaunchScope b(c, HWR_K_MLP_TC, prof);
+        CK(c, launch_mlp_tc(t, q, c->qual, c->status_d, c->stream), "predictor kernel");
+        b.done();
+        return HWR_OK;
+    }
+    LaunchScope a(c, HWR_K_ROUTE_SIMT, prof);
+    CK(c, launch_route_simt(m, q, c->stream), "route kernel");
+    a.done();
+    return HWR_OK;
+}
+
+static size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+extern "C" hwr_status hwr_route_batch(hwr_ctx *c, int32_t Q, const float *in_len,
+                                      const float *out_len, const void *q_emb, float slo,
+                                      float lambda, uint32_t flags, int32_t *chosen,
+                                      float *pred_latency, float *utility) {
+    if (!c) return fail(nullptr, HWR_ERR_INVALID_ARG, "ctx is NULL");
+    if (c->broken) return HWR_ERR_STATE;
+    const uint32_t known = HWR_SEQUENTIAL | HWR_DEVICE_PTRS | HWR_ASYNC | HWR_SCORE_CONVEX |
+                           HWR_PATH_SIMT | HWR_PATH_TENSOR | HWR_PROFILE;
+    if (flags & ~known) return fail(c, HWR_ERR_INVALID_ARG, "unknown flag bits 0x%x", flags & ~known);
+    if (Q < 0) return fail(c, HWR_ERR_INVALID_ARG, "Q=%d < 0", Q);
+    if (Q == 0) return HWR_OK;
+    if (!in_len || !out_len || !q_emb || !chosen || !pred_latency || !utility)
+        return fail(c, HWR_ERR_INVALID_ARG, "NULL input or output array");
+    if (slo != slo) return fail(c, HWR_ERR_INVALID_ARG, "SLO is NaN");
+    if (!isfinite(lambda)) return fail(c, HWR_ERR_INVALID_ARG, "lambda is not finite");
+    if ((flags & HWR_PATH_SIMT) && (flags & HWR_PATH_TENSOR))
+        return fail(c, HWR_ERR_INVALID_ARG, "HWR_PATH_SIMT and HWR_PATH_TENSOR together");
+    if (!c->have_snapshot)
+        return fail(c, HWR_ERR_INVALID_ARG, "route before the first hwr_update_snapshot");
+    const bool seq = flags & HWR_SEQUENTIAL;
+    if ((flags & HWR_PATH_TENSOR) && (seq || !c->tc_ok))
+        return fail(c, HWR_ERR_UNSUPPORTED, "tensor-core path unavailable for this %s",
+                    seq ? "sequential call" : "context (fp32 or unsupported shape)");
+    const bool tensor = !seq && c->tc_ok &&
+                        ((flags & HWR_PATH_TENSOR) || (!(flags & HWR_PATH_SIMT) && Q >= TC_MIN_Q));
+    const bool dev = flags & HWR_DEVICE_PTRS;
+    const size_t es = c->dtype == HWR_BF16 ? 2 : 4;
+    if (dev && tensor && ((uintptr_t)q_emb & 15))
+        return fail(c, HWR_ERR_INVALID_ARG, "device q_emb must be 16-byte aligned");
+
+    Queries q;
+    q.Q = Q;
+    q.emb_bf16 = c->dtype == HWR_BF16;
+    q.slo = slo;
+    q.lam = lambda;
+    q.wq = (flags & HWR_SCORE_CONVEX) ? 1.0f - lambda : 1.0f;
+
+    const size_t emb_b = (size_t)Q * c->E * es, len_b = (size_t)Q * 4;
+    const size_t off_in = align_up(emb_b, 256), off_out = off_in + align_up(len_b, 256);
+    const size_t in_total = off_out + len_b;
+    const size_t o_lat = align_up(len_b, 256), o_util = o_lat + align_up(len_b, 256);
+    const size_t out_total = o_util + len_b;
+    const bool packed = !dev && !(flags & HWR_ASYNC) && in_total <= ((size_t)1 << 20);
+
+    if (dev) {
+        q.in_len = in_len; q.out_len = out_len; q.emb = q_emb;
+        q.chosen = chosen; q.lat = pred_latency; q.util = utility;
+    } else {
+        TRY(grow(c, &c->io_d, &c->io_cap, in_total));
+        TRY(grow(c, &c->out_d, &c->out_cap, out_total));
+        if (packed) {
+            TRY(pin_grow(c, in_total > out_total ? in_total : out_total));
+            CK(c, cudaEventSynchronize(c->pin_ev), "wait for staging");
+            memcpy(c->pin_h, q_emb, emb_b);
+            memcpy(c->pin_h + off_in, in_len, len_b);
+            memcpy(c->pin_h + off_out, out_len, len_b);
+            CK(c, cudaMemcpyAsync(c->io_d, c->pin_h, in_total, cudaMemcpyHostToDevice, c->stream),
+               "copy inputs");
+        } else {
+            CK(c, cudaMemcpyAsync(c->io_d, q_emb, emb_b, cudaMemcpyHostToDevice, c->stream), "copy emb");
+            CK(c, cudaMemcpyAsync(c->io_d + off_in, in_len, len_b, cudaMemcpyHostToDevice, c->stream),
+               "copy in_len");
+            CK(c, cudaMemcpyAsync(c->io_d + off_out, out_len, len_b, cudaMemcpyHostToDevice, c->stream),
+               "copy out_len");
+        }
+        q.emb = c->io_d;
+        q.in_len = (const float *)(c->io_d + off_in);
+        q.out_len = (const float *)(c->io_d + off_out);
+        q.chosen = (int32_t *)c->out_d;
+        q.lat = (float *)(c->out_d + o_lat);
+        q.util = (float *)(c->out_d + o_util);
+    }
+
+    TRY(run_kernels(c, q, flags, tensor));
+
+    bool synced = false;
+    if (!dev) {
+        if (packed) {
+            CK(c, cudaMemcpyAsync(c->pin_h, c->out_d, out_total, cudaMemcpyDeviceToHost, c->stream),
+               "copy outputs");
+            CK(c, cudaEventRecord(c->pin_ev, c->stream), "record");
+            CK(c, cudaStreamSynchronize(c->stream), "synchronize");
+            synced = true;
+            memcpy(chosen, c->pin_h, len_b);
+            memcpy(pred_latency, c->pin_h + o_lat, len_b);
+            memcpy(utility, c->pin_h + o_util, len_b);
+        } else {
+            CK(c, cudaMemcpyAsync(chosen, c->out_d, len_b, cudaMemcpyDeviceToHost, c->stream), "copy chosen");
+            CK(c, cudaMemcpyAsync(pred_latency, c->out_d + o_lat, len_b, cudaMemcpyDeviceToHost, c->stream),
+               "copy latency");
+            CK(c, cudaMemcpyAsync(utility, c->out_d + o_util, len_b, cudaMemcpyDeviceToHost, c->stream),
+               "copy utility");
+        }
+    }
+    c->stats.queries_routed += Q;
+    if ((flags & HWR_ASYNC) && !synced) return HWR_OK;
+    if (!synced) CK(c, cudaStreamSynchronize(c->stream), "synchronize");
+    CK(c, cudaGetLastError(), "kernel");
+    if (tensor) TRY(check_status_word(c));
+    return HWR_OK;
+}
+
+extern "C" hwr_status hwr_synchronize(hwr_ctx *c) {
+    if (!c) return fail(nullptr, HWR_ERR_INVALID_ARG, "ctx is NULL");
+    if (c->broken) return HWR_ERR_STATE;
+    CK(c, cudaStreamSynchronize(c->stream), "synchronize");
+    return check_status_word(c);
+}
+
+extern "C" hwr_status hwr_get_stats(hwr_ctx *c, hwr_stats *out, int reset) {
+    if (!c || !out) return fail(c, HWR_ERR_INVALID_ARG, "NULL argument");
+    if (!c->broken) TRY(collect_profile(c));
+    *out = c->stats;
+    if (reset) {
+        for (int k = 0; k < HWR_K_COUNT; ++k) {
+            c->stats.profiled_ms[k] = 0;
+            c->stats.profiled_launches[k] = 0;
+        }
+    }
+    return HWR_OK;
+}
+
+extern "C" const char *hwr_status_string(hwr_status s) {
+    switch (s) {
+        case HWR_OK: return "ok";
+        case HWR_ERR_INVALID_ARG: return "invalid argument";
+        case HWR_ERR_DTYPE: return "embedding dtype does not match the predictor";
+        case HWR_ERR_OOM: return "out of memory";
+        case HWR_ERR_CUDA: return "CUDA error";
+        case HWR_ERR_TIMEOUT: return "device-side wait timed out";
+        case HWR_ERR_STATE: return "context unusable after an earlier failure";
+        case HWR_ERR_UNSUPPORTED: return "unsupported by this build";
+    }
+    return "unknown status";
+}
+
+extern "C" const char *hwr_last_error(const hwr_ctx *c) {
+    return c ? c->err.c_str() : g_create_error.c_str();
+}

@@ -1,0 +1,100 @@
+// Internal interface between the C-ABI host code (hwr_api.cu) and the CUDA
+// kernels (k_simt.cu: fp32 SIMT kernels, k_tc.cu: bf16 tcgen05 kernels).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "hwr.h"
+
+namespace hwr {
+
+// Device status word, written by kernels whose waits are bounded.
+enum : int32_t { ST_OK = 0, ST_TIMEOUT = 1, ST_BAD_LAUNCH = 2 };
+
+// Largest number of (query, deployment) rows one SIMT tile holds:
+// 8 row groups (one per warp) x RPT rows each.
+constexpr int SIMT_THREADS = 256;
+constexpr int SIMT_KC = 32;          // K chunk of the layer-2 tile
+constexpr int ROUTE_RPT = 8;         // route kernel: rows <= 64
+constexpr int SEQ_RPT = 9;           // sequential table: rows <= 72 (Qs + 1)
+constexpr int MAX_D = 64;
+constexpr int MAX_H = 256;
+constexpr int SEQ_MAX_CHUNK = 64;    // queries per sequential table
+constexpr int SEQ_CHAIN_SMEM = 200 * 1024;
+
+// Read-only device view of the predictor and deployment state.
+struct Model {
+    int M, G, D, F, H1, H2, E, P;
+    const int32_t *dep_model;   // [D]
+    const int32_t *dep_gpu;     // [D]
+    const float *log10p;        // [M]
+    const float *W1, *b1;       // [H1][F], [H1]   fp32 (bf16 widened)
+    const float *W2, *b2;       // [H2][H1], [H2]
+    const float *W3, *b3;       // [2][H2], [2]
+    const float *mu, *sd;       // [F]
+    const uint8_t *xform;       // [F]
+    const float *memb;          // [E][M] fp32 (bf16 widened)
+    // snapshot (SoA, [D]) and derived per-deployment state
+    int32_t *running;
+    const int32_t *waiting;
+    const float *kv, *gpu_util, *ttft, *tpot;
+    float *X;                   // [D][F] standardised deployment features
+    float *Spre;                // [D][H1] layer-1 chain through slot P
+    float *A;                   // [D][H1] layer-1 chain through slot F-3
+};
+
+struct Queries {
+    int Q;
+    const float *in_len, *out_len;
+    const void *emb;            // [Q][E], fp32 or bf16 bits
+    int emb_bf16;
+    float slo, lam, wq;         // wq = 1 or (1 - lambda)
+    int32_t *chosen;
+    float *lat, *util;
+};
+
+// ---- SIMT kernels (k_simt.cu) -------------------------------------------
+cudaError_t launch_snapshot(const Model &m, cudaStream_t s);
+// Fused gather -> MLP -> mask -> argmax for a batch.
+cudaError_t launch_route_simt(const Model &m, const Queries &q, cudaStream_t s);
+// Sequential mode over one chunk of Qs <= seq_chunk(m) queries: the score
+// table (every (picks c, deployment d, query i >= c)), then the serial chain.
+//   ctab: scratch of seq_table_floats(D, Qs) floats; qual: Qs * M floats.
+cudaError_t launch_seq_table(const Model &m, const Queries &q, int Qs,
+                             float *ctab, float *qual, cudaStream_t s);
+cudaError_t launch_seq_chain(const Model &m, const Queries &q, int Qs,
+                             const float *ctab, const float *qual, cudaStream_t s);
+int seq_chunk(const Model &m);
+size_t seq_table_floats(int D, int Qs);
+size_t route_simt_smem(const Model &m);
+size_t seq_table_smem(const Model &m);
+cudaError_t simt_prepare();   // one-time smem opt-in
+
+// ---- tcgen05 kernels (k_tc.cu) -------------------------------------------
+struct TcModel {
+    int M, Mpad, D, H1, H2, E, Epad;
+    const uint16_t *W2img;      // bf16 W2 in the UMMA shared-memory image
+    const uint16_t *membimg;    // bf16 memb^T in the UMMA shared-memory image
+    const float *A;             // [D][H1]
+    const float *W1q;           // [2][H1]: W1 columns of the two query slots
+    const float *b2, *W3, *b3;  // fp32
+    const int32_t *dep_model;
+    float mu_in, sd_in, mu_out, sd_out;
+    uint8_t xf_in, xf_out;
+};
+bool tc_supported(int M, int H1, int H2, int E);
+size_t tc_w2img_elems(int H1, int H2);
+size_t tc_membimg_elems(int Mpad, int Epad);
+// Host-side construction of the shared-memory images (bf16 bits in/out).
+void tc_build_w2img(const uint16_t *W2, int H1, int H2, uint16_t *img);
+void tc_build_membimg(const uint16_t *memb_EM, int E, int M, int Mpad, int Epad,
+                      uint16_t *img);
+// qual: scratch [Q][Mpad] fp32.  status: device int32 word.
+cudaError_t launch_qual_tc(const TcModel &m, const Queries &q, float *qual,
+                           int32_t *status, cudaStream_t s);
+cudaError_t launch_mlp_tc(const TcModel &m, const Queries &q, const float *qual,
+                          int32_t *status, cudaStream_t s);
+cudaError_t tc_prepare();
+
+}  // namespace hwr

@@ -1,0 +1,209 @@
+"""GPU parity: the CUDA path against the CPU oracle on the same seeded inputs.
+
+fp32 SIMT kernels follow the canonical fp32 order, so their latency, utility
+and chosen index must equal the oracle's canonical-fp32 mode bit for bit (and
+sit within 1e-5 relative of the fp64 oracle).  bf16 contexts routed through
+the SIMT kernels are the same computation on bf16-valued inputs and are held
+to the same bit-exact bar.
+"""
+import numpy as np
+import pytest
+
+import oracle as O
+import workload as W
+import paper_2608_14575_gb300 as H
+
+pytestmark = pytest.mark.gpu
+
+SIMT = H.HWR_PATH_SIMT
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    H.build()
+
+
+def _f32(a):
+    return np.asarray(a, np.float64).astype(np.float32)
+
+
+def assert_exact(got, want, what=""):
+    ch, lat, util = got
+    wch, wlat, wutil = want[:3]
+    bad = np.nonzero(ch != wch)[0]
+    assert bad.size == 0, f"{what}: chosen differs at {bad[:10]} ({ch[bad[:5]]} vs {wch[bad[:5]]})"
+    assert np.array_equal(lat, _f32(wlat), equal_nan=True), what
+    assert np.array_equal(util, _f32(wutil), equal_nan=True), what
+
+
+def assert_close_f64(got, want, tol=1e-5):
+    _, lat, util = got
+    _, wlat, wutil = want[:3]
+    ok = np.isfinite(wlat)
+    assert np.all(np.abs(lat[ok] - wlat[ok]) <= tol * np.maximum(np.abs(wlat[ok]), 1e-3))
+    assert np.all(np.abs(util[ok] - wutil[ok]) <= tol * np.maximum(np.abs(wutil[ok]), 1.0))
+
+
+def route_both(p, flags=0, **kw):
+    r = H.Router(p)
+    got = r.route(flags=flags, **kw)
+    orc = O.Problem(p)
+    conv = bool(flags & H.HWR_SCORE_CONVEX)
+    want = orc.route(mode=O.F32, convex=conv, nthreads=8, **kw)
+    r.close()
+    return got, want, orc
+
+
+@pytest.mark.parametrize("Q", [1, 2, 17, 31, 33, 255, 256])
+def test_tiny_fp32_exact(Q):
+    p = W.make_config(0, Q=Q)
+    got, want, orc = route_both(p)
+    assert_exact(got, want, f"cfg0 Q={Q}")
+    assert_close_f64(got, orc.route(mode=O.F64))
+
+
+@pytest.mark.parametrize("slo,lam", [(0.0, 0.5), (float("inf"), 0.5), (5.0, 0.0),
+                                     (1.0, 4.0), (float("-inf"), 0.5)])
+def test_tiny_fp32_degenerate_budgets(slo, lam):
+    p = W.make_config(0, Q=97)
+    got, want, _ = route_both(p, slo=slo, lam=lam)
+    assert_exact(got, want, f"slo={slo} lam={lam}")
+
+
+def test_convex_score_exact():
+    p = W.make_config(0, Q=129)
+    got, want, _ = route_both(p, flags=H.HWR_SCORE_CONVEX, lam=0.25)
+    assert_exact(got, want, "convex")
+
+
+@pytest.mark.parametrize("c,Q", [(1, 300), (3, 40), (4, 65)])
+def test_bf16_contexts_simt_exact(c, Q):
+    p = W.make_config(c, Q=Q)
+    got, want, orc = route_both(p, flags=SIMT)
+    assert_exact(got, want, f"cfg{c} simt")
+    assert_close_f64(got, orc.route(mode=O.F64, nthreads=8))
+
+
+@pytest.mark.parametrize("shape", [
+    dict(M=1, G=1, F=12, H1=8, H2=8, E=8),      # D = 1
+    dict(M=3, G=1, F=16, H1=40, H2=24, E=16),   # odd widths, K not a chunk multiple
+    dict(M=5, G=3, F=24, H1=96, H2=200, E=40),  # D = 15, H2 not a multiple of 32
+    dict(M=16, G=4, F=48, H1=256, H2=256, E=64),  # D = 64, widest tile
+])
+def test_shapes_with_biases_exact(shape):
+    p = W.make_problem(Q=77, dtype="f32", lam=0.4, slo=2.0, seed=31, bias_std=0.3,
+                       **shape)
+    got, want, _ = route_both(p)
+    assert_exact(got, want, str(shape))
+
+
+def test_device_pointers_match_host():
+    import torch
+    p = W.make_config(0, Q=200)
+    stream = torch.cuda.current_stream().cuda_stream
+    r = H.Router(p, stream=stream)
+    host = r.route()
+    dev = torch.device("cuda:0")
+    il = torch.from_numpy(p["in_len"]).to(dev)
+    ol = torch.from_numpy(p["out_len"]).to(dev)
+    em = torch.from_numpy(p["emb"]).to(dev)
+    ch = torch.empty(200, dtype=torch.int32, device=dev)
+    lat = torch.empty(200, dtype=torch.float32, device=dev)
+    ut = torch.empty(200, dtype=torch.float32, device=dev)
+    r.route_device(il, ol, em, ch, lat, ut, slo=p["slo"], lam=p["lam"])
+    torch.cuda.synchronize()
+    assert np.array_equal(ch.cpu().numpy(), host[0])
+    assert np.array_equal(lat.cpu().numpy(), host[1])
+    assert np.array_equal(ut.cpu().numpy(), host[2])
+    r.close()
+
+
+def test_deterministic_reruns():
+    p = W.make_config(1, Q=512)
+    r = H.Router(p)
+    first = r.route(flags=SIMT)
+    for _ in range(5):
+        again = r.route(flags=SIMT)
+        for a, b in zip(first, again):
+            assert np.array_equal(a, b)
+    r.close()
+
+
+def test_route_before_snapshot_and_bad_args():
+    p = W.make_config(0, Q=8)
+    r = H.Router(p)
+    with pytest.raises(H.HwrError) as e:
+        r.route(slo=float("nan"))
+    assert e.value.status == 1
+    with pytest.raises(H.HwrError) as e:
+        r.route(flags=H.HWR_PATH_TENSOR)       # fp32 context has no tensor path
+    assert e.value.status == 7
+    # the context stays usable after argument errors
+    got = r.route()
+    assert got[0].shape == (8,)
+    r.close()
+
+
+# ---------------------------------------------------------------------------
+# sequential mode
+
+def test_sequential_single_call_exact():
+    p = W.make_config(2, Q=200)     # several chunks of the sequential table
+    r = H.Router(p)
+    got = r.route(flags=H.HWR_SEQUENTIAL)
+    orc = O.Problem(p)
+    want = orc.route(mode=O.F32, sequential=True, nthreads=8)
+    assert_exact(got, want, "sequential")
+    assert np.array_equal(r.get_snapshot(), want[3])
+    # increments persist until the next snapshot
+    got2 = r.route(flags=H.HWR_SEQUENTIAL)
+    want2 = orc.route(mode=O.F32, sequential=True, running=want[3], nthreads=8)
+    assert_exact(got2, want2, "sequential, second call")
+    # and a batch call afterwards sees the incremented counts
+    snap = dict(p["snap"])
+    snap["running"] = want2[3]
+    got3 = r.route()
+    want3 = O.Problem(p, snap=snap).route(mode=O.F32, nthreads=8)
+    assert_exact(got3, want3, "batch after sequential")
+    r.update_snapshot(p["snap"])
+    assert np.array_equal(r.get_snapshot(), p["snap"]["running"])
+    r.close()
+
+
+def _online(p, n):
+    """Run the online micro-batch loop through the GPU and through the oracle."""
+    r = H.Router(p)
+
+    def gpu_route(snap, lo, hi):
+        r.update_snapshot(snap)
+        return r.route(p["in_len"][lo:hi], p["out_len"][lo:hi], p["emb"][lo:hi],
+                       flags=H.HWR_SEQUENTIAL)[0]
+
+    orc = O.Problem(p)
+
+    def cpu_route(snap, lo, hi):
+        orc.set_snapshot(snap)
+        return orc.route(p["in_len"][lo:hi], p["out_len"][lo:hi], p["emb"][lo:hi],
+                         mode=O.F32, sequential=True, running=snap["running"],
+                         nthreads=8)[0]
+
+    g, _ = W.simulate_online(p, gpu_route, n_requests=n)
+    c, _ = W.simulate_online(p, cpu_route, n_requests=n)
+    r.close()
+    return g, c
+
+
+def test_online_sequential_prefix_exact():
+    p = W.make_config(2, Q=6_432)   # 100 full micro-batches and a ragged one
+    g, c = _online(p, p["Q"])
+    bad = np.nonzero(g != c)[0]
+    assert bad.size == 0, f"first divergence at request {bad[:1]}"
+
+
+@pytest.mark.slow
+def test_online_sequential_full_100k_exact():
+    p = W.make_config(2)
+    g, c = _online(p, p["Q"])
+    bad = np.nonzero(g != c)[0]
+    assert bad.size == 0, f"first divergence at request {bad[:1]}"
+    assert len(np.unique(g)) > 1
