@@ -1,14 +1,60 @@
 // bf16 tensor-core kernels (tcgen05 + TMA) of the route-scoring path.
+//
+// K_qual_tc  quality contraction of Sec. 3.2 "Quality Predictor":
+//            S = Qemb [Q x E] . Memb [E x M] on the tensor cores (M padded to
+//            16 or 32), query tiles streamed by TMA, model embeddings resident
+//            in shared memory, accumulators in TMEM; epilogue sigmoid -> qual
+//            [Q][Mpad] fp32.  Memory bound: it streams the embeddings once.
+// K_mlp_tc   the latency predictor of Eq. 1 for every (query, deployment)
+//            pair, then Eq. 2 and the decision maker of Eq. 3.  Per tile of
+//            128 queries and per deployment d, producer warps build the layer-1
+//            activations relu(A_d + W1[:, in] u_q + W1[:, out] v_q) as bf16
+//            straight into the UMMA operand layout in shared memory (A_d is the
+//            query-independent prefix of layer 1 computed per snapshot); one
+//            thread issues the layer-2 MMA against W2 resident in shared
+//            memory into a double-buffered TMEM accumulator; epilogue warps
+//            (one TMEM lane = one query) apply bias + ReLU, the two output
+//            heads, softplus, the cost, the utility and the SLO mask, and
+//            keep the running argmax over d in registers.
+//
+// Warp roles are fixed per CTA; CTAs are persistent over query tiles.  Every
+// mbarrier wait is bounded (umma.cuh): on a timeout the CTA stops, drains what
+// it issued, frees its TMEM and reports HWR_ERR_TIMEOUT through the status
+// word.
+#include <cuda.h>
+#include <cudaTypedefs.h>
 #include <string.h>
 
 #include "hwr_internal.cuh"
+#include "select.cuh"
+#include "umma.cuh"
 
 namespace hwr {
 
-// Shared-memory operand images for UMMA, K-major with the 128-byte swizzle:
-// the K extent is cut into chunks of 64 bf16 (128 bytes); chunk c holds one
-// 128-byte row per matrix row n, and inside each row the 16-byte granule g
-// is stored at position g ^ (n % 8).  Chunks follow each other.
+using namespace umma;
+
+namespace {
+
+constexpr int BM = 128;                         // queries per tile
+constexpr int KCH = 64;                         // bf16 K elements per 128-byte row
+constexpr uint32_t CHUNK_BYTES = BM * KCH * 2;  // one A chunk: 16 KB
+constexpr int QUAL_THREADS = 192;               // w0 TMA, w1 MMA, w2-5 epilogue
+constexpr int QUAL_STAGES = 8;
+constexpr int MLP_THREADS = 320;                // w0 MMA, w1 -, w2-5 epilogue, w6-9 producers
+constexpr int MLP_MAX_STAGES = 8;
+constexpr uint32_t SMEM_LIMIT = 227 * 1024;
+
+int g_num_sms = 0;
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+
+}  // namespace
+
+// ---------------------------------------------------------------------------
+// host-side shared-memory images (K-major, 128-byte swizzle): the K extent is
+// cut into chunks of 64 bf16 (128 bytes); chunk c holds one 128-byte row per
+// matrix row n, and inside each row the 16-byte granule g is stored at
+// position g ^ (n % 8).  Chunks follow each other.
+
 static inline size_t sw128_index(int rows, int n, int k) {
     const int c = k >> 6, kk = k & 63, g = kk >> 3, e = kk & 7;
     return (size_t)c * rows * 64 + (size_t)n * 64 + (size_t)((g ^ (n & 7)) << 3) + e;
@@ -29,16 +75,495 @@ void tc_build_membimg(const uint16_t *memb_EM, int E, int M, int Mpad, int Epad,
         for (int k = 0; k < E; ++k) img[sw128_index(Mpad, m, k)] = memb_EM[(size_t)k * M + m];
 }
 
-bool tc_supported(int, int, int, int) { return false; }
+// ---------------------------------------------------------------------------
+// shared-memory layouts (byte offsets from a 1024-aligned base)
 
-cudaError_t tc_prepare() { return cudaSuccess; }
+struct QualLayout {
+    uint32_t memb, stages, bars, misc, total;
+};
 
-cudaError_t launch_qual_tc(const TcModel &, const Queries &, float *, int32_t *, cudaStream_t) {
-    return cudaErrorNotSupported;
+__host__ __device__ inline QualLayout qual_layout(int Mpad, int Epad) {
+    QualLayout L;
+    uint32_t o = 0;
+    L.memb = o;
+    o += (uint32_t)Mpad * Epad * 2;
+    o = (o + 1023) & ~1023u;
+    L.stages = o;
+    o += QUAL_STAGES * CHUNK_BYTES;
+    L.bars = o;
+    o += (2 * QUAL_STAGES + 6) * 8;
+    L.misc = o;
+    o += 16;
+    L.total = o + 1024;  // slack for aligning the dynamic base
+    return L;
 }
 
-cudaError_t launch_mlp_tc(const TcModel &, const Queries &, const float *, int32_t *, cudaStream_t) {
-    return cudaErrorNotSupported;
+struct MlpLayout {
+    uint32_t w2, ring, qual, consts, bars, misc, total;
+    int ns;
+};
+
+__host__ __device__ inline MlpLayout mlp_layout(int H1, int H2, int Mpad, int D) {
+    MlpLayout L;
+    uint32_t fixed = (uint32_t)H1 * H2 * 2                  // W2 image
+                     + BM * (Mpad + 1) * 4                  // quality rows
+                     + (3 * H2 + 4) * 4 + D * 4             // b2, W3, b3, dep_model
+                     + (2 * MLP_MAX_STAGES + 6) * 8 + 16    // barriers, misc
+                     + 1024 + 1024;                         // alignment slack
+    int ns = (int)((SMEM_LIMIT - fixed) / CHUNK_BYTES);
+    L.ns = ns > MLP_MAX_STAGES ? MLP_MAX_STAGES : ns;
+    uint32_t o = 0;
+    L.w2 = o;
+    o += (uint32_t)H1 * H2 * 2;
+    o = (o + 1023) & ~1023u;
+    L.ring = o;
+    o += (uint32_t)(L.ns > 0 ? L.ns : 0) * CHUNK_BYTES;
+    L.qual = o;
+    o += BM * (Mpad + 1) * 4;
+    L.consts = o;
+    o += (3 * H2 + 4) * 4 + D * 4;
+    o = (o + 7) & ~7u;
+    L.bars = o;
+    o += (2 * MLP_MAX_STAGES + 6) * 8;
+    L.misc = o;
+    o += 16;
+    L.total = o + 1024;
+    return L;
+}
+
+__device__ __forceinline__ uint8_t *align1024(uint8_t *p) {
+    const uint32_t a = smem_u32(p);
+    return p + (((a + 1023) & ~1023u) - a);
+}
+
+// Bounded wait that ignores the abort flag: used only to drain copies and
+// MMAs this CTA itself issued before it frees its resources.
+__device__ __forceinline__ void drain_wait(uint64_t *bar, uint32_t parity) {
+    const long long t0 = clock64();
+    while (!mbar_try_wait(bar, parity) && clock64() - t0 < WAIT_CYCLES) {
+    }
+}
+
+__device__ __forceinline__ float softplus_fast(float z) {
+    return fmaxf(z, 0.f) + log1pf(__expf(-fabsf(z)));
+}
+
+__device__ __forceinline__ float standardise_fast(uint8_t code, float v, float mu, float sd) {
+    const float t = code == 1 ? log1pf(v) : (code == 2 ? logf(v) : v);
+    return (t - mu) / sd;
+}
+
+// ---------------------------------------------------------------------------
+// K_qual_tc
+
+__global__ void __launch_bounds__(QUAL_THREADS, 1)
+k_qual_tc(const __grid_constant__ CUtensorMap tmap, TcModel m, int Q, float *qual,
+          int32_t *status) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *sm = align1024(smem_raw);
+    const QualLayout L = qual_layout(m.Mpad, m.Epad);
+    uint8_t *membs = sm + L.memb, *stages = sm + L.stages;
+    uint64_t *full = (uint64_t *)(sm + L.bars), *empty = full + QUAL_STAGES;
+    uint64_t *accf = empty + QUAL_STAGES, *acce = accf + 2, *wbar = acce + 2, *dbar = wbar + 1;
+    uint32_t *tslot = (uint32_t *)(sm + L.misc);
+    volatile int *abort_f = (volatile int *)(tslot + 1);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int nch = m.Epad / KCH, ntiles = (Q + BM - 1) / BM, Mpad = m.Mpad;
+    const uint32_t membytes = (uint32_t)Mpad * m.Epad * 2;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < QUAL_STAGES; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&accf[b], 1);
+            mbar_init(&acce[b], 128);
+        }
+        mbar_init(wbar, 1);
+        mbar_init(dbar, 1);
+        *abort_f = 0;
+        fence_mbar_init();
+    }
+    if (warp == 1) {
+        tmem_alloc(tslot, 64);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tslot;
+
+    if (warp == 0 && lane == 0) {
+        // producer: model embeddings once, then query tiles chunk by chunk
+        tma_prefetch_desc(&tmap);
+        mbar_arrive_expect_tx(wbar, membytes);
+        for (uint32_t off = 0; off < membytes; off += 16384)
+            bulk_g2s(membs + off, (const uint8_t *)m.membimg + off,
+                     membytes - off < 16384 ? membytes - off : 16384, wbar);
+        uint32_t n = 0;
+        bool ok = true;
+        for (int t = blockIdx.x; ok && t < ntiles; t += gridDim.x)
+            for (int c = 0; c < nch; ++c, ++n) {
+                const int s = n % QUAL_STAGES;
+                ok = mbar_wait(&empty[s], ((n / QUAL_STAGES) & 1) ^ 1, abort_f, status);
+                if (!ok) break;
+                mbar_arrive_expect_tx(&full[s], CHUNK_BYTES);
+                tma_load_2d(stages + s * CHUNK_BYTES, &tmap, &full[s], c * KCH, t * BM);
+            }
+        // drain the loads still in flight before the CTA can exit
+        const uint32_t first = n > QUAL_STAGES ? n - QUAL_STAGES : 0;
+        for (uint32_t j = first; j < n; ++j) drain_wait(&full[j % QUAL_STAGES], (j / QUAL_STAGES) & 1);
+        drain_wait(wbar, 0);
+    } else if (warp == 1 && lane == 0) {
+        // MMA issuer
+        bool ok = mbar_wait(wbar, 0, abort_f, status);
+        const uint32_t idesc = idesc_bf16_f32(BM, Mpad);
+        uint32_t n = 0, lt = 0;
+        for (int t = blockIdx.x; ok && t < ntiles; t += gridDim.x, ++lt) {
+            const int b = lt & 1;
+            ok = mbar_wait(&acce[b], ((lt >> 1) & 1) ^ 1, abort_f, status);
+            if (!ok) break;
+            tc_fence_after();
+            for (int c = 0; c < nch; ++c, ++n) {
+                const int s = n % QUAL_STAGES;
+                ok = mbar_wait(&full[s], (n / QUAL_STAGES) & 1, abort_f, status);
+                if (!ok) break;
+                tc_fence_after();
+                const uint64_t ad = sdesc_sw128(smem_u32(stages + s * CHUNK_BYTES));
+                const uint64_t bd = sdesc_sw128(smem_u32(membs + (uint32_t)c * Mpad * 128));
+#pragma unroll
+                for (int k = 0; k < 4; ++k)
+                    mma_bf16(tmem + b * 32, ad + 2 * k, bd + 2 * k, idesc, (c | k) != 0);
+                mma_commit(&empty[s]);
+            }
+            if (!ok) break;
+            mma_commit(&accf[b]);
+        }
+        // every MMA this thread issued must land before TMEM is freed
+        mma_commit(dbar);
+        drain_wait(dbar, 0);
+    } else if (warp >= 2) {
+        // epilogue: TMEM lane = query row of the tile
+        const int quad = warp & 3, r = quad * 32 + lane;
+        const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
+        uint32_t lt = 0;
+        bool ok = true;
+        for (int t = blockIdx.x; t < ntiles; t += gridDim.x, ++lt) {
+            const int b = lt & 1;
+            ok = mbar_wait(&accf[b], (lt >> 1) & 1, abort_f, status);
+            ok = __all_sync(0xffffffffu, ok);
+            if (!ok) break;
+            tc_fence_after();
+            uint32_t v[32];
+            uint32_t v16[16];
+            tmem_ld16(tmem + lane_base + b * 32, v16);
+            tmem_wait_ld16(v16);
+#pragma unroll
+            for (int i = 0; i < 16; ++i) v[i] = v16[i];
+            if (Mpad == 32) {
+                tmem_ld16(tmem + lane_base + b * 32 + 16, v16);
+                tmem_wait_ld16(v16);
+#pragma unroll
+                for (int i = 0; i < 16; ++i) v[16 + i] = v16[i];
+            }
+            tc_fence_before();
+            mbar_arrive(&acce[b]);
+            const int row = t * BM + r;
+            if (row < Q) {
+                float4 *dst = (float4 *)(qual + (size_t)row * Mpad);
+                for (int i = 0; i < Mpad; i += 4) {
+                    float4 o;
+                    o.x = i + 0 < m.M ? 1.f / (1.f + expf(-__uint_as_float(v[i + 0]))) : 0.f;
+                    o.y = i + 1 < m.M ? 1.f / (1.f + expf(-__uint_as_float(v[i + 1]))) : 0.f;
+                    o.z = i + 2 < m.M ? 1.f / (1.f + expf(-__uint_as_float(v[i + 2]))) : 0.f;
+                    o.w = i + 3 < m.M ? 1.f / (1.f + expf(-__uint_as_float(v[i + 3]))) : 0.f;
+                    dst[i >> 2] = o;
+                }
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        __syncwarp();
+        tc_fence_after();
+        tmem_dealloc(tmem, 64);
+    }
+}
+
+// ---------------------------------------------------------------------------
+// K_mlp_tc
+
+__global__ void __launch_bounds__(MLP_THREADS, 1)
+k_mlp_tc(TcModel m, Queries q, const float *__restrict__ qual, int32_t *status) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *sm = align1024(smem_raw);
+    const int H1 = m.H1, H2 = m.H2, D = m.D, Mpad = m.Mpad, QS = Mpad + 1;
+    const MlpLayout L = mlp_layout(H1, H2, Mpad, D);
+    const int NS = L.ns;
+    uint8_t *w2s = sm + L.w2, *ring = sm + L.ring;
+    float *qs = (float *)(sm + L.qual);
+    float *b2s = (float *)(sm + L.consts), *w30s = b2s + H2, *w31s = w30s + H2;
+    float *b3s = w31s + H2;
+    int *dms = (int *)(b3s + 4);
+    uint64_t *full = (uint64_t *)(sm + L.bars), *empty = full + MLP_MAX_STAGES;
+    uint64_t *accf = empty + MLP_MAX_STAGES, *acce = accf + 2, *wbar = acce + 2, *dbar = wbar + 1;
+    uint32_t *tslot = (uint32_t *)(sm + L.misc);
+    volatile int *abort_f = (volatile int *)(tslot + 1);
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int nch = H1 / KCH, ntiles = (q.Q + BM - 1) / BM;
+    const uint32_t tcols = 2 * H2 <= 32 ? 32 : 2 * H2 <= 64 ? 64 : 2 * H2 <= 128 ? 128
+                                                : 2 * H2 <= 256 ? 256 : 512;
+
+    if (tid == 0) {
+        for (int s = 0; s < NS; ++s) {
+            mbar_init(&full[s], 128);
+            mbar_init(&empty[s], 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&accf[b], 1);
+            mbar_init(&acce[b], 128);
+        }
+        mbar_init(wbar, 1);
+        mbar_init(dbar, 1);
+        *abort_f = 0;
+        fence_mbar_init();
+    }
+    for (int i = tid; i < H2; i += MLP_THREADS) {
+        b2s[i] = m.b2[i];
+        w30s[i] = m.W3[i];
+        w31s[i] = m.W3[H2 + i];
+    }
+    if (tid < 2) b3s[tid] = m.b3[tid];
+    for (int i = tid; i < D; i += MLP_THREADS) dms[i] = m.dep_model[i];
+    if (warp == 0) {
+        tmem_alloc(tslot, tcols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tslot;
+
+    if (warp == 0 && lane == 0) {
+        // W2 once, then one layer-2 MMA chain per (tile, deployment)
+        const uint32_t wbytes = (uint32_t)H1 * H2 * 2;
+        mbar_arrive_expect_tx(wbar, wbytes);
+        for (uint32_t off = 0; off < wbytes; off += 16384)
+            bulk_g2s(w2s + off, (const uint8_t *)m.W2img + off,
+                     wbytes - off < 16384 ? wbytes - off : 16384, wbar);
+        bool ok = mbar_wait(wbar, 0, abort_f, status);
+        const uint32_t idesc = idesc_bf16_f32(BM, H2);
+        uint32_t n = 0, g = 0;
+        for (int t = blockIdx.x; ok && t < ntiles; t += gridDim.x) {
+            for (int d = 0; d < D; ++d, ++g) {
+                const int b = g & 1;
+                ok = mbar_wait(&acce[b], ((g >> 1) & 1) ^ 1, abort_f, status);
+                if (!ok) break;
+                tc_fence_after();
+                const uint32_t dt = tmem + (uint32_t)b * H2;
+                for (int c = 0; c < nch; ++c, ++n) {
+                    const int s = n % NS;
+                    ok = mbar_wait(&full[s], (n / NS) & 1, abort_f, status);
+                    if (!ok) break;
+                    tc_fence_after();
+                    const uint64_t ad = sdesc_sw128(smem_u32(ring + s * CHUNK_BYTES));
+                    const uint64_t bd = sdesc_sw128(smem_u32(w2s + (uint32_t)c * H2 * 128));
+#pragma unroll
+                    for (int k = 0; k < 4; ++k)
+                        mma_bf16(dt, ad + 2 * k, bd + 2 * k, idesc, (c | k) != 0);
+                    mma_commit(&empty[s]);
+                }
+                if (!ok) break;
+                mma_commit(&accf[b]);
+            }
+        }
+        // everything this thread issued must land before TMEM is freed
+        mma_commit(dbar);
+        drain_wait(dbar, 0);
+        drain_wait(wbar, 0);
+    } else if (warp >= 2 && warp < 6) {
+        // epilogue: TMEM lane = query row of the tile
+        const int quad = warp & 3, r = quad * 32 + lane;
+        const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
+        const float slo = q.slo, lam = q.lam, wq = q.wq, b30 = b3s[0], b31 = b3s[1];
+        uint32_t g = 0;
+        bool ok = true;
+        for (int t = blockIdx.x; ok && t < ntiles; t += gridDim.x) {
+            const int row = t * BM + r;
+            const bool valid = row < q.Q;
+            const float ol = valid ? q.out_len[row] : 0.f;
+            for (int i = 0; i < m.M; ++i)
+                qs[r * QS + i] = valid ? qual[(size_t)row * Mpad + i] : 0.f;
+            Cand best = no_cand();
+            for (int d = 0; d < D; ++d, ++g) {
+                const int b = g & 1;
+                ok = mbar_wait(&accf[b], (g >> 1) & 1, abort_f, status);
+                ok = __all_sync(0xffffffffu, ok);
+                if (!ok) break;
+                tc_fence_after();
+                float t0a = 0.f, t0b = 0.f, t1a = 0.f, t1b = 0.f;
+                for (int cc = 0; cc < H2; cc += 32) {
+                    uint32_t v[32];
+                    tmem_ld32(tmem + lane_base + (uint32_t)b * H2 + cc, v);
+                    tmem_wait_ld32(v);
+#pragma unroll
+                    for (int j = 0; j < 32; j += 2) {
+                        const float2 bb = *(const float2 *)(b2s + cc + j);
+                        const float2 w0 = *(const float2 *)(w30s + cc + j);
+                        const float2 w1 = *(const float2 *)(w31s + cc + j);
+                        const float h0 = fmaxf(__uint_as_float(v[j]) + bb.x, 0.f);
+                        const float h1 = fmaxf(__uint_as_float(v[j + 1]) + bb.y, 0.f);
+                        t0a = fmaf(h0, w0.x, t0a);
+                        t0b = fmaf(h1, w0.y, t0b);
+                        t1a = fmaf(h0, w1.x, t1a);
+                        t1b = fmaf(h1, w1.y, t1b);
+                    }
+                }
+                tc_fence_before();
+                mbar_arrive(&acce[b]);
+                const float ttft = softplus_fast(t0a + t0b + b30);
+                const float tpot = softplus_fast(t1a + t1b + b31);
+                const float C = fmaf(ol, tpot, ttft);
+                const float U = fmaf(-lam, C, wq * qs[r * QS + dms[d]]);
+                const Cand c = make_cand(C, U, d, slo);
+                if (better(c, best)) best = c;
+            }
+            if (ok && valid) {
+                const bool sel = best.cls > 0;
+                q.chosen[row] = sel ? best.d : -1;
+                q.lat[row] = sel ? best.C : __int_as_float(0x7fc00000);
+                q.util[row] = sel ? best.U : __int_as_float(0x7fc00000);
+            }
+        }
+    } else if (warp >= 6) {
+        // producers: layer-1 activations as bf16 in the UMMA operand layout.
+        // Thread p writes granule (p % 8) of rows p / 8 + 16 i, i < 8.
+        const int p = tid - 192, gi = p & 7, rb = p >> 3;
+        uint32_t n = 0;
+        bool ok = true;
+        for (int t = blockIdx.x; ok && t < ntiles; t += gridDim.x) {
+            float u[8], v[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                const int row = t * BM + rb + 16 * i;
+                const bool valid = row < q.Q;
+                u[i] = valid ? standardise_fast(m.xf_in, q.in_len[row], m.mu_in, m.sd_in) : 0.f;
+                v[i] = valid ? standardise_fast(m.xf_out, q.out_len[row], m.mu_out, m.sd_out) : 0.f;
+            }
+            for (int d = 0; ok && d < D; ++d) {
+                const float *Ad = m.A + (size_t)d * H1;
+                for (int c = 0; c < nch; ++c, ++n) {
+                    const int s = n % NS;
+                    ok = mbar_wait(&empty[s], ((n / NS) & 1) ^ 1, abort_f, status);
+                    if (!ok) break;
+                    const int k0 = c * KCH + gi * 8;
+                    const float4 a0 = *(const float4 *)(Ad + k0), a1 = *(const float4 *)(Ad + k0 + 4);
+                    const float4 i0 = *(const float4 *)(m.W1q + k0), i1 = *(const float4 *)(m.W1q + k0 + 4);
+                    const float4 o0 = *(const float4 *)(m.W1q + H1 + k0),
+                                 o1 = *(const float4 *)(m.W1q + H1 + k0 + 4);
+                    const float a[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
+                    const float wi[8] = {i0.x, i0.y, i0.z, i0.w, i1.x, i1.y, i1.z, i1.w};
+                    const float wo[8] = {o0.x, o0.y, o0.z, o0.w, o1.x, o1.y, o1.z, o1.w};
+                    const uint32_t st = smem_u32(ring + s * CHUNK_BYTES);
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) {
+                        const int r = rb + 16 * i;
+                        uint32_t pk[4];
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) {
+                            const float x0 = fmaf(v[i], wo[2 * e], fmaf(u[i], wi[2 * e], a[2 * e]));
+                            const float x1 =
+                                fmaf(v[i], wo[2 * e + 1], fmaf(u[i], wi[2 * e + 1], a[2 * e + 1]));
+                            pk[e] = pack_relu_bf16x2(x0, x1);
+                        }
+                        const uint32_t off = (uint32_t)(r >> 3) * 1024 + (uint32_t)(r & 7) * 128 +
+                                             (uint32_t)((gi ^ (r & 7)) << 4);
+                        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(st + off),
+                                     "r"(pk[0]), "r"(pk[1]), "r"(pk[2]), "r"(pk[3])
+                                     : "memory");
+                    }
+                    fence_proxy_async_smem();
+                    mbar_arrive(&full[s]);
+                }
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) {
+        __syncwarp();
+        tc_fence_after();
+        tmem_dealloc(tmem, tcols);
+    }
+}
+
+// ---------------------------------------------------------------------------
+// host side
+
+bool tc_supported(int M, int H1, int H2, int E) {
+    if (M < 1 || M > 32) return false;
+    if (H1 < 64 || H1 > 256 || H1 % 64) return false;
+    if (H2 < 32 || H2 > 256 || H2 % 32) return false;
+    if (E < 8 || E % 8) return false;
+    const int Mpad = M <= 16 ? 16 : 32, Epad = (E + 63) / 64 * 64;
+    if (qual_layout(Mpad, Epad).total > SMEM_LIMIT) return false;
+    const MlpLayout L = mlp_layout(H1, H2, Mpad, 64);
+    return L.ns >= 2 && L.total <= SMEM_LIMIT;
+}
+
+cudaError_t tc_prepare() {
+    if (!g_num_sms) {
+        int dev = 0;
+        cudaError_t e = cudaGetDevice(&dev);
+        if (e == cudaSuccess) e = cudaDeviceGetAttribute(&g_num_sms, cudaDevAttrMultiProcessorCount, dev);
+        if (e != cudaSuccess) return e;
+    }
+    if (!g_encode) {
+        void *fn = nullptr;
+        cudaDriverEntryPointQueryResult qr;
+        cudaError_t e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000,
+                                                         cudaEnableDefault, &qr);
+        if (e != cudaSuccess) return e;
+        if (qr != cudaDriverEntryPointSuccess || !fn) return cudaErrorNotSupported;
+        g_encode = (PFN_cuTensorMapEncodeTiled_v12000)fn;
+    }
+    cudaError_t e = cudaFuncSetAttribute(k_qual_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         SMEM_LIMIT);
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(k_mlp_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_LIMIT);
+    return e;
+}
+
+cudaError_t launch_qual_tc(const TcModel &m, const Queries &q, float *qual, int32_t *status,
+                           cudaStream_t s) {
+    if (q.Q <= 0) return cudaSuccess;
+    CUtensorMap map;
+    const cuuint64_t dims[2] = {(cuuint64_t)m.E, (cuuint64_t)q.Q};
+    const cuuint64_t strides[1] = {(cuuint64_t)m.E * 2};
+    const cuuint32_t box[2] = {KCH, BM};
+    const cuuint32_t estr[2] = {1, 1};
+    CUresult r = g_encode(&map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(q.emb),
+                          dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                          CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                          CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
+    const int ntiles = (q.Q + BM - 1) / BM;
+    const int grid = ntiles < g_num_sms ? ntiles : g_num_sms;
+    const QualLayout L = qual_layout(m.Mpad, m.Epad);
+    k_qual_tc<<<grid, QUAL_THREADS, L.total, s>>>(map, m, q.Q, qual, status);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_mlp_tc(const TcModel &m, const Queries &q, const float *qual, int32_t *status,
+                          cudaStream_t s) {
+    if (q.Q <= 0) return cudaSuccess;
+    const int ntiles = (q.Q + BM - 1) / BM;
+    const int grid = ntiles < g_num_sms ? ntiles : g_num_sms;
+    const MlpLayout L = mlp_layout(m.H1, m.H2, m.Mpad, m.D);
+    k_mlp_tc<<<grid, MLP_THREADS, L.total, s>>>(m, q, qual, status);
+    return cudaGetLastError();
 }
 
 }  // namespace hwr

@@ -1,0 +1,199 @@
+"""GPU parity of the bf16 tensor-core path (tcgen05 + TMA) against the oracle.
+
+The tensor path rounds the layer-1 activations to bf16 for the layer-2 MMA and
+accumulates in fp32, so it is held to the bf16 tolerance against the fp64
+oracle: predicted latency and utility within 2e-2 relative (utility relative
+to max(|U|, 1)).  Chosen indices must match wherever the decision is not
+within that tolerance of a tie: the oracle's top-2 utility margin (or, with
+no feasible deployment, the top-2 latency margin) exceeds 2e-2 and no
+deployment's latency is within 2e-2 of the SLO.  For the remaining queries
+the chosen deployment must still be a valid near-optimal choice.
+"""
+import numpy as np
+import pytest
+
+import oracle as O
+import workload as W
+import paper_2608_14575_gb300 as H
+
+pytestmark = pytest.mark.gpu
+TOL = 2e-2
+TC = H.HWR_PATH_TENSOR
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    H.build()
+
+
+def check_against_oracle(p, got, idx=None, slo=None, lam=None, convex=False,
+                         min_checked=0.5):
+    """Compare GPU outputs for queries `idx` (all if None) with the fp64 oracle."""
+    ch, lat, util = (np.asarray(a) for a in got)
+    if idx is not None:
+        sub = W.query_subset(p, idx)
+        ch, lat, util = ch[idx], lat[idx], util[idx]
+    else:
+        sub = p
+    slo = p["slo"] if slo is None else slo
+    lam = p["lam"] if lam is None else lam
+    orc = O.Problem(sub)
+    C, U = orc.score_all(lam=lam, convex=convex, nthreads=16)
+    wch, wlat, wutil, _ = orc.route(slo=slo, lam=lam, convex=convex, nthreads=16)
+    ok = wch >= 0
+    assert np.array_equal(ch >= 0, ok)
+    # the chosen deployment may legitimately differ near ties, so compare the
+    # GPU's outputs with the oracle's scores of the deployment the GPU chose
+    qi = np.nonzero(ok)[0]
+    glat = C[qi, ch[ok]]
+    gutil = U[qi, ch[ok]]
+    rl_own = np.abs(lat[ok] - glat) / np.maximum(np.abs(glat), 1e-3)
+    ru_own = np.abs(util[ok] - gutil) / np.maximum(np.abs(gutil), 1.0)
+    assert rl_own.max(initial=0) <= TOL, rl_own.max()
+    assert ru_own.max(initial=0) <= TOL, ru_own.max()
+    # decisions that are clear under the tolerance must match exactly
+    band = TOL * max(abs(slo), 1e-3) if np.isfinite(slo) else 0.0
+    feas = C <= slo
+    sure = C <= slo - band          # feasible under any in-tolerance latency
+    maybe = C <= slo + band         # feasible under some in-tolerance latency
+    near_slo = (sure != maybe).any(axis=1)
+    with np.errstate(invalid="ignore"):
+        Uf = np.where(feas, U, -np.inf)
+        top1 = Uf.max(axis=1)
+        # runner-up: the best utility strictly below the top.  Exact ties (the
+        # GPU types of one model when lambda = 0) are resolved by index on both
+        # sides, so they do not make a decision unclear.
+        top2 = np.where(Uf < top1[:, None], Uf, -np.inf).max(axis=1)
+        margin_u = (top1 - top2) > TOL * np.maximum(np.abs(top1), 1.0)
+    Cs = np.sort(C, axis=1)
+    margin_c = (Cs[:, 1] - Cs[:, 0]) > TOL * np.maximum(Cs[:, 0], 1e-3) if C.shape[1] > 1 \
+        else np.ones(len(C), bool)
+    any_feas = feas.any(axis=1)
+    clear = np.where(any_feas, margin_u, margin_c) & ~near_slo
+    bad = np.nonzero(clear & (ch != wch))[0]
+    assert bad.size == 0, f"{bad.size} clear decisions differ, e.g. query {bad[:5]}"
+    assert clear.mean() >= min_checked, clear.mean()
+    # the rest must still be valid choices: a deployment the GPU may call
+    # feasible is at least as good (within tolerance) as every surely feasible
+    # one; a choice made as "nothing feasible" needs nothing surely feasible
+    # and has the lowest latency within tolerance
+    for q in np.nonzero(~clear & ok)[0]:
+        c = ch[q]
+        if maybe[q, c]:
+            if sure[q].any():
+                best = U[q][sure[q]].max()
+                assert U[q, c] >= best - 2 * TOL * max(abs(best), 1.0), (q, c)
+        else:
+            assert not sure[q].any(), (q, c)
+            assert C[q, c] <= C[q].min() * (1 + 2 * TOL), (q, c)
+    return float(clear.mean())
+
+
+def test_mid_bf16_full():
+    p = W.make_config(1)                   # Q = 4096, D = 12, H = 128, E = 768
+    r = H.Router(p)
+    got = r.route(flags=TC)
+    frac = check_against_oracle(p, got)
+    auto = r.route()                        # Q >= 512 takes the tensor path by default
+    assert all(np.array_equal(a, b) for a, b in zip(got, auto))
+    st = r.stats()
+    assert st["launches"]["mlp_tc"] == 2 and st["launches"]["qual_tc"] == 2
+    r.close()
+    assert frac > 0.6
+
+
+def test_large_bf16_full_size_sampled():
+    p = W.make_config(3)                   # Q = 65,536, D = 64, H = 256, E = 1024
+    r = H.Router(p)
+    got = r.route()
+    assert r.stats()["launches"]["mlp_tc"] == 1
+    idx = np.arange(0, p["Q"], 61)          # sampled outputs, spanning every tile
+    check_against_oracle(p, got, idx=idx)
+    r.close()
+
+
+@pytest.mark.parametrize("Q", [1, 5, 127, 128, 129, 300, 1000])
+def test_forced_tensor_ragged_batches(Q):
+    p = W.make_config(1, Q=Q)
+    r = H.Router(p)
+    check_against_oracle(p, r.route(flags=TC), min_checked=0.0 if Q < 10 else 0.5)
+    r.close()
+
+
+@pytest.mark.parametrize("shape", [
+    dict(M=1, G=1, F=12, H1=64, H2=32, E=40),        # D = 1, E not a multiple of 64
+    dict(M=5, G=3, F=24, H1=192, H2=96, E=1000),     # odd M, Epad > E
+    dict(M=17, G=2, F=40, H1=128, H2=160, E=64),     # Mpad = 32
+    dict(M=32, G=2, F=48, H1=256, H2=256, E=256),    # D = 64, M = 32
+    dict(M=7, G=1, F=24, H1=64, H2=256, E=128),      # D = 7
+])
+def test_tensor_shapes_with_biases(shape):
+    p = W.make_problem(Q=700, dtype="bf16", lam=0.3, slo=4.0, seed=77, bias_std=0.3,
+                       **shape)
+    r = H.Router(p)
+    check_against_oracle(p, r.route(flags=TC), min_checked=0.3)
+    r.close()
+
+
+@pytest.mark.parametrize("slo,lam,convex", [(0.0, 0.3, False), (float("inf"), 0.3, False),
+                                            (10.0, 0.0, False), (10.0, 0.25, True)])
+def test_tensor_budgets(slo, lam, convex):
+    p = W.make_config(3, Q=3000)
+    r = H.Router(p)
+    got = r.route(flags=TC | (H.HWR_SCORE_CONVEX if convex else 0), slo=slo, lam=lam)
+    check_against_oracle(p, got, slo=slo, lam=lam, convex=convex, min_checked=0.3)
+    r.close()
+
+
+def test_tensor_matches_simt_within_tolerance_and_is_deterministic():
+    p = W.make_config(3, Q=2048)
+    r = H.Router(p)
+    tc = r.route(flags=TC)
+    simt = r.route(flags=H.HWR_PATH_SIMT)
+    same = tc[0] == simt[0]
+    assert same.mean() > 0.95
+    assert np.all(np.abs(tc[1] - simt[1])[same] <= TOL * np.abs(simt[1])[same])
+    for _ in range(3):
+        again = r.route(flags=TC)
+        assert all(np.array_equal(a, b) for a, b in zip(tc, again))
+    r.close()
+
+
+def test_tensor_device_pointers():
+    import torch
+    p = W.make_config(4, Q=4096)
+    r = H.Router(p, stream=torch.cuda.current_stream().cuda_stream)
+    host = r.route(flags=TC)
+    dev = torch.device("cuda:0")
+    il = torch.from_numpy(p["in_len"]).to(dev)
+    ol = torch.from_numpy(p["out_len"]).to(dev)
+    em = torch.from_numpy(p["emb"].view(np.int16)).to(dev)
+    ch = torch.empty(p["Q"], dtype=torch.int32, device=dev)
+    lat = torch.empty(p["Q"], dtype=torch.float32, device=dev)
+    ut = torch.empty(p["Q"], dtype=torch.float32, device=dev)
+    r.route_device(il, ol, em, ch, lat, ut, slo=p["slo"], lam=p["lam"], flags=TC)
+    torch.cuda.synchronize()
+    assert np.array_equal(ch.cpu().numpy(), host[0])
+    assert np.array_equal(lat.cpu().numpy(), host[1])
+    r.close()
+
+
+@pytest.mark.parametrize("Q", [1, 16, 256, 4096, 65_536])
+def test_batch_sweep_d32(Q):
+    p = W.make_config(4, Q=Q)
+    r = H.Router(p)
+    got = r.route()
+    idx = None if Q <= 4096 else np.arange(0, Q, 67)
+    check_against_oracle(p, got, idx=idx, min_checked=0.0 if Q < 100 else 0.5)
+    r.close()
+
+
+@pytest.mark.slow
+def test_batch_sweep_d32_one_million():
+    p = W.make_config(4, Q=1_048_576)
+    r = H.Router(p)
+    got = r.route()
+    check_against_oracle(p, got, idx=np.arange(0, p["Q"], 1021))
+    # every query got a defined choice
+    assert (got[0] >= 0).all() and (got[0] < p["D"]).all()
+    r.close()
