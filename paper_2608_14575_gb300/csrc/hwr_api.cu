@@ -57,6 +57,7 @@ struct hwr_ctx {
     int32_t *running = nullptr, *waiting = nullptr;
     float *kv = nullptr, *gpu_util = nullptr, *ttft = nullptr, *tpot = nullptr;
     float *X = nullptr, *Spre = nullptr, *A = nullptr;
+    uint16_t *Abf = nullptr;
     // host feature constants for the tensor path
     float mu_in = 0, sd_in = 1, mu_out = 0, sd_out = 1;
     uint8_t xf_in = 0, xf_out = 0;
@@ -71,6 +72,8 @@ struct hwr_ctx {
 
     // grow-only scratch
     float *qual = nullptr;   size_t qual_cap = 0;     // [Q][Mpad]
+    char *part = nullptr;    size_t part_cap = 0;     // split-deployment partials
+    int32_t *count = nullptr; size_t count_cap = 0;   // per-row arrivals (self-resetting)
     float *ctab = nullptr;   size_t ctab_cap = 0;
     float *qseq = nullptr;   size_t qseq_cap = 0;
     int seq_qs = 0;
@@ -200,7 +203,7 @@ static Model model_view(const hwr_ctx *c) {
     m.mu = c->mu; m.sd = c->sd; m.xform = c->xform; m.memb = c->memb;
     m.running = c->running; m.waiting = c->waiting; m.kv = c->kv;
     m.gpu_util = c->gpu_util; m.ttft = c->ttft; m.tpot = c->tpot;
-    m.X = c->X; m.Spre = c->Spre; m.A = c->A;
+    m.X = c->X; m.Spre = c->Spre; m.A = c->A; m.Abf = c->Abf;
     return m;
 }
 
@@ -208,7 +211,7 @@ static TcModel tc_view(const hwr_ctx *c) {
     TcModel t;
     t.M = c->M; t.Mpad = c->Mpad; t.D = c->D; t.H1 = c->H1; t.H2 = c->H2;
     t.E = c->E; t.Epad = c->Epad;
-    t.W2img = c->W2img; t.membimg = c->membimg; t.A = c->A; t.W1q = c->W1q;
+    t.W2img = c->W2img; t.membimg = c->membimg; t.Abf = c->Abf; t.W1q = c->W1q;
     t.b2 = c->b2; t.W3 = c->W3; t.b3 = c->b3; t.dep_model = c->dep_model;
     t.mu_in = c->mu_in; t.sd_in = c->sd_in; t.mu_out = c->mu_out; t.sd_out = c->sd_out;
     t.xf_in = c->xf_in; t.xf_out = c->xf_out;
@@ -377,6 +380,7 @@ static hwr_status build_ctx(hwr_ctx *c, const hwr_deployment_table *t, const hwr
     TRY(dev_alloc(c, &c->X, (size_t)D * F));
     TRY(dev_alloc(c, &c->Spre, (size_t)D * H1));
     TRY(dev_alloc(c, &c->A, (size_t)D * H1));
+    TRY(dev_alloc(c, &c->Abf, (size_t)D * H1));
 
     TRY(upload(c, c->dep_model, t->dep_model, D * 4, "upload table"));
     TRY(upload(c, c->dep_gpu, t->dep_gpu, D * 4, "upload table"));
@@ -568,11 +572,20 @@ static hwr_status run_kernels(hwr_ctx *c, const Queries &q, uint32_t flags, bool
     if (tensor) {
         const TcModel t = tc_view(c);
         TRY(grow(c, &c->qual, &c->qual_cap, (size_t)q.Q * c->Mpad));
+        const int ns = tc_mlp_split(t, q.Q);
+        if (ns > 1) {
+            TRY(grow(c, &c->part, &c->part_cap, (size_t)ns * q.Q * 16));
+            if (c->count_cap < (size_t)q.Q) {
+                TRY(grow(c, &c->count, &c->count_cap, (size_t)q.Q));
+                CK(c, cudaMemsetAsync(c->count, 0, c->count_cap * 4, c->stream), "zero counters");
+            }
+        }
         LaunchScope a(c, HWR_K_QUAL_TC, prof);
         CK(c, launch_qual_tc(t, q, c->qual, c->status_d, c->stream), "quality kernel");
         a.done();
         LaunchScope b(c, HWR_K_MLP_TC, prof);
-        CK(c, launch_mlp_tc(t, q, c->qual, c->status_d, c->stream), "predictor kernel");
+        CK(c, launch_mlp_tc(t, q, c->qual, ns, c->part, c->count, c->status_d, c->stream),
+           "predictor kernel");
         b.done();
         return HWR_OK;
     }

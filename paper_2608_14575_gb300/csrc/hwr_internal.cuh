@@ -42,6 +42,7 @@ struct Model {
     float *X;                   // [D][F] standardised deployment features
     float *Spre;                // [D][H1] layer-1 chain through slot P
     float *A;                   // [D][H1] layer-1 chain through slot F-3
+    uint16_t *Abf;              // [D][H1] A rounded to bf16 (tensor-core path)
 };
 
 struct Queries {
@@ -76,7 +77,7 @@ struct TcModel {
     int M, Mpad, D, H1, H2, E, Epad;
     const uint16_t *W2img;      // bf16 W2 in the UMMA shared-memory image
     const uint16_t *membimg;    // bf16 memb^T in the UMMA shared-memory image
-    const float *A;             // [D][H1]
+    const uint16_t *Abf;        // [D][H1] bf16 deployment prefix of layer 1
     const float *W1q;           // [2][H1]: W1 columns of the two query slots
     const float *b2, *W3, *b3;  // fp32
     const int32_t *dep_model;
@@ -93,8 +94,13 @@ void tc_build_membimg(const uint16_t *memb_EM, int E, int M, int Mpad, int Epad,
 // qual: scratch [Q][Mpad] fp32.  status: device int32 word.
 cudaError_t launch_qual_tc(const TcModel &m, const Queries &q, float *qual,
                            int32_t *status, cudaStream_t s);
+// Deployments of a tile may be split over `nsplit` units; then `part`
+// (nsplit * Q records of 16 bytes) and `count` (Q int32, zero, self-resetting)
+// are scratch.
+int tc_mlp_split(const TcModel &m, int Q);
 cudaError_t launch_mlp_tc(const TcModel &m, const Queries &q, const float *qual,
-                          int32_t *status, cudaStream_t s);
+                          int nsplit, void *part, int32_t *count, int32_t *status,
+                          cudaStream_t s);
 cudaError_t tc_prepare();
 
 }  // namespace hwr

@@ -19,6 +19,7 @@
 // Method (HW-Router Sec. 3.2): feature assembly and the latency predictor
 // (Eq. 1), cost (Eq. 2), hardware-independent quality, and the decision maker
 // with its SLO constraint (Eq. 3).
+#include <cuda_bf16.h>
 #include <math.h>
 
 #include "hwr_internal.cuh"
@@ -91,6 +92,7 @@ __global__ void __launch_bounds__(SIMT_THREADS) k_snapshot(Model m) {
         m.Spre[(size_t)d * m.H1 + j] = acc;
         for (; k < m.F - 2; ++k) acc = __fmaf_rn(w[k], xs[k], acc);
         m.A[(size_t)d * m.H1 + j] = acc;
+        m.Abf[(size_t)d * m.H1 + j] = __bfloat16_as_ushort(__float2bfloat16_rn(acc));
     }
 }
 
@@ -451,6 +453,7 @@ k_seq_chain(Model m, Queries q, int Qs, const float *ctab, const float *qualS) {
         acc = __fmaf_rn(w[P + 1], xr, acc);
         for (int k = P + 2; k < F - 2; ++k) acc = __fmaf_rn(w[k], x[k], acc);
         m.A[(size_t)d * H1 + j] = acc;
+        m.Abf[(size_t)d * H1 + j] = __bfloat16_as_ushort(__float2bfloat16_rn(acc));
         if (j == 0) m.X[(size_t)d * F + P + 1] = xr;
     }
 }

@@ -22,6 +22,7 @@
 // it issued, frees its TMEM and reports HWR_ERR_TIMEOUT through the status
 // word.
 #include <cuda.h>
+#include <cuda_bf16.h>
 #include <cudaTypedefs.h>
 #include <string.h>
 
@@ -40,7 +41,8 @@ constexpr int KCH = 64;                         // bf16 K elements per 128-byte 
 constexpr uint32_t CHUNK_BYTES = BM * KCH * 2;  // one A chunk: 16 KB
 constexpr int QUAL_THREADS = 192;               // w0 TMA, w1 MMA, w2-5 epilogue
 constexpr int QUAL_STAGES = 8;
-constexpr int MLP_THREADS = 320;                // w0 MMA, w1 -, w2-5 epilogue, w6-9 producers
+constexpr int MLP_THREADS = 416;                // w0 MMA, w1-4 epilogue, w5-12 producers
+constexpr int MLP_PRODUCERS = 256;
 constexpr int MLP_MAX_STAGES = 8;
 constexpr uint32_t SMEM_LIMIT = 227 * 1024;
 
@@ -294,9 +296,58 @@ k_qual_tc(const __grid_constant__ CUtensorMap tmap, TcModel m, int Q, float *qua
 
 // ---------------------------------------------------------------------------
 // K_mlp_tc
+//
+// Work unit = (query tile, part of the deployment range).  With more than one
+// part per tile, each unit leaves its per-row best candidate in `part` and the
+// last of a row's units to arrive (per-row atomic counter) merges them.
+
+struct Unit {
+    int tile, part, d0, d1;
+};
+
+__device__ __forceinline__ Unit unit_of(int u, int ntiles, int nsplit, int D) {
+    Unit x;
+    x.tile = u % ntiles;
+    x.part = u / ntiles;
+    x.d0 = x.part * D / nsplit;
+    x.d1 = (x.part + 1) * D / nsplit;
+    return x;
+}
+
+// bf16 pairs in 32-bit registers: relu(a * b + c), and float pair -> bf16 pair
+__device__ __forceinline__ uint32_t hfma2_relu(uint32_t a, uint32_t b, uint32_t c) {
+    uint32_t d;
+    asm("fma.rn.relu.bf16x2 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(c));
+    return d;
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+    uint32_t d;
+    asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(hi), "f"(lo));
+    return d;
+}
+
+__device__ __forceinline__ void head_pair(const uint32_t *v, int j, const float4 &bb,
+                                          const float4 &w0, const float4 &w1, float2 &t0a,
+                                          float2 &t0b, float2 &t1a, float2 &t1b) {
+    // relu(acc + b2) for four columns, then both output heads as packed FMAs
+    float2 x01 = __fadd2_rn(make_float2(__uint_as_float(v[j]), __uint_as_float(v[j + 1])),
+                            make_float2(bb.x, bb.y));
+    float2 x23 = __fadd2_rn(make_float2(__uint_as_float(v[j + 2]), __uint_as_float(v[j + 3])),
+                            make_float2(bb.z, bb.w));
+    x01.x = fmaxf(x01.x, 0.f);
+    x01.y = fmaxf(x01.y, 0.f);
+    x23.x = fmaxf(x23.x, 0.f);
+    x23.y = fmaxf(x23.y, 0.f);
+    t0a = __ffma2_rn(x01, make_float2(w0.x, w0.y), t0a);
+    t0b = __ffma2_rn(x23, make_float2(w0.z, w0.w), t0b);
+    t1a = __ffma2_rn(x01, make_float2(w1.x, w1.y), t1a);
+    t1b = __ffma2_rn(x23, make_float2(w1.z, w1.w), t1b);
+}
 
 __global__ void __launch_bounds__(MLP_THREADS, 1)
-k_mlp_tc(TcModel m, Queries q, const float *__restrict__ qual, int32_t *status) {
+k_mlp_tc(TcModel m, Queries q, const float *__restrict__ qual, int nsplit, int4 *part,
+         int32_t *count, int32_t *status) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *sm = align1024(smem_raw);
     const int H1 = m.H1, H2 = m.H2, D = m.D, Mpad = m.Mpad, QS = Mpad + 1;
@@ -312,13 +363,13 @@ k_mlp_tc(TcModel m, Queries q, const float *__restrict__ qual, int32_t *status) 
     uint32_t *tslot = (uint32_t *)(sm + L.misc);
     volatile int *abort_f = (volatile int *)(tslot + 1);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int nch = H1 / KCH, ntiles = (q.Q + BM - 1) / BM;
+    const int nch = H1 / KCH, ntiles = (q.Q + BM - 1) / BM, nunits = ntiles * nsplit;
     const uint32_t tcols = 2 * H2 <= 32 ? 32 : 2 * H2 <= 64 ? 64 : 2 * H2 <= 128 ? 128
                                                 : 2 * H2 <= 256 ? 256 : 512;
 
     if (tid == 0) {
         for (int s = 0; s < NS; ++s) {
-            mbar_init(&full[s], 128);
+            mbar_init(&full[s], MLP_PRODUCERS);
             mbar_init(&empty[s], 1);
         }
         for (int b = 0; b < 2; ++b) {
@@ -347,7 +398,7 @@ k_mlp_tc(TcModel m, Queries q, const float *__restrict__ qual, int32_t *status) 
     const uint32_t tmem = *tslot;
 
     if (warp == 0 && lane == 0) {
-        // W2 once, then one layer-2 MMA chain per (tile, deployment)
+        // ---- MMA issuer: W2 once, then one layer-2 MMA chain per step -----
         const uint32_t wbytes = (uint32_t)H1 * H2 * 2;
         mbar_arrive_expect_tx(wbar, wbytes);
         for (uint32_t off = 0; off < wbytes; off += 16384)
@@ -356,8 +407,9 @@ k_mlp_tc(TcModel m, Queries q, const float *__restrict__ qual, int32_t *status) 
         bool ok = mbar_wait(wbar, 0, abort_f, status);
         const uint32_t idesc = idesc_bf16_f32(BM, H2);
         uint32_t n = 0, g = 0;
-        for (int t = blockIdx.x; ok && t < ntiles; t += gridDim.x) {
-            for (int d = 0; d < D; ++d, ++g) {
+        for (int u = blockIdx.x; ok && u < nunits; u += gridDim.x) {
+            const Unit un = unit_of(u, ntiles, nsplit, D);
+            for (int d = un.d0; d < un.d1; ++d, ++g) {
                 const int b = g & 1;
                 ok = mbar_wait(&acce[b], ((g >> 1) & 1) ^ 1, abort_f, status);
                 if (!ok) break;
@@ -383,109 +435,164 @@ k_mlp_tc(TcModel m, Queries q, const float *__restrict__ qual, int32_t *status) 
         mma_commit(dbar);
         drain_wait(dbar, 0);
         drain_wait(wbar, 0);
-    } else if (warp >= 2 && warp < 6) {
-        // epilogue: TMEM lane = query row of the tile
+    } else if (warp >= 1 && warp < 5) {
+        // ---- epilogue: TMEM lane = query row of the tile ---------------------
         const int quad = warp & 3, r = quad * 32 + lane;
         const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
         const float slo = q.slo, lam = q.lam, wq = q.wq, b30 = b3s[0], b31 = b3s[1];
+        const float4 *b2v = (const float4 *)b2s, *w0v = (const float4 *)w30s,
+                     *w1v = (const float4 *)w31s;
+        const int ncol = H2 / 32;
         uint32_t g = 0;
         bool ok = true;
-        for (int t = blockIdx.x; ok && t < ntiles; t += gridDim.x) {
-            const int row = t * BM + r;
+        for (int u = blockIdx.x; ok && u < nunits; u += gridDim.x) {
+            const Unit un = unit_of(u, ntiles, nsplit, D);
+            const int row = un.tile * BM + r;
             const bool valid = row < q.Q;
             const float ol = valid ? q.out_len[row] : 0.f;
             for (int i = 0; i < m.M; ++i)
                 qs[r * QS + i] = valid ? qual[(size_t)row * Mpad + i] : 0.f;
             Cand best = no_cand();
-            for (int d = 0; d < D; ++d, ++g) {
+            for (int d = un.d0; d < un.d1; ++d, ++g) {
                 const int b = g & 1;
                 ok = mbar_wait(&accf[b], (g >> 1) & 1, abort_f, status);
                 ok = __all_sync(0xffffffffu, ok);
                 if (!ok) break;
                 tc_fence_after();
-                float t0a = 0.f, t0b = 0.f, t1a = 0.f, t1b = 0.f;
-                for (int cc = 0; cc < H2; cc += 32) {
-                    uint32_t v[32];
-                    tmem_ld32(tmem + lane_base + (uint32_t)b * H2 + cc, v);
-                    tmem_wait_ld32(v);
+                const uint32_t base = tmem + lane_base + (uint32_t)b * H2;
+                float2 t0a = make_float2(0.f, 0.f), t0b = t0a, t1a = t0a, t1b = t0a;
+                uint32_t va[32], vb[32];
+                tmem_ld32(base, va);
+                for (int c = 0; c < ncol; c += 2) {
+                    tmem_wait_ld32(va);
+                    if (c + 1 < ncol) tmem_ld32(base + (c + 1) * 32, vb);
 #pragma unroll
-                    for (int j = 0; j < 32; j += 2) {
-                        const float2 bb = *(const float2 *)(b2s + cc + j);
-                        const float2 w0 = *(const float2 *)(w30s + cc + j);
-                        const float2 w1 = *(const float2 *)(w31s + cc + j);
-                        const float h0 = fmaxf(__uint_as_float(v[j]) + bb.x, 0.f);
-                        const float h1 = fmaxf(__uint_as_float(v[j + 1]) + bb.y, 0.f);
-                        t0a = fmaf(h0, w0.x, t0a);
-                        t0b = fmaf(h1, w0.y, t0b);
-                        t1a = fmaf(h0, w1.x, t1a);
-                        t1b = fmaf(h1, w1.y, t1b);
+                    for (int j = 0; j < 32; j += 4) {
+                        const int f = (c * 32 + j) >> 2;
+                        head_pair(va, j, b2v[f], w0v[f], w1v[f], t0a, t0b, t1a, t1b);
+                    }
+                    if (c + 1 < ncol) {
+                        tmem_wait_ld32(vb);
+                        if (c + 2 < ncol) tmem_ld32(base + (c + 2) * 32, va);
+#pragma unroll
+                        for (int j = 0; j < 32; j += 4) {
+                            const int f = ((c + 1) * 32 + j) >> 2;
+                            head_pair(vb, j, b2v[f], w0v[f], w1v[f], t0a, t0b, t1a, t1b);
+                        }
                     }
                 }
                 tc_fence_before();
                 mbar_arrive(&acce[b]);
-                const float ttft = softplus_fast(t0a + t0b + b30);
-                const float tpot = softplus_fast(t1a + t1b + b31);
+                const float z0 = (t0a.x + t0a.y) + (t0b.x + t0b.y) + b30;
+                const float z1 = (t1a.x + t1a.y) + (t1b.x + t1b.y) + b31;
+                const float ttft = softplus_fast(z0), tpot = softplus_fast(z1);
                 const float C = fmaf(ol, tpot, ttft);
                 const float U = fmaf(-lam, C, wq * qs[r * QS + dms[d]]);
-                const Cand c = make_cand(C, U, d, slo);
-                if (better(c, best)) best = c;
+                const Cand cd = make_cand(C, U, d, slo);
+                if (better(cd, best)) best = cd;
             }
-            if (ok && valid) {
+            if (!ok || !valid) continue;
+            if (nsplit == 1) {
                 const bool sel = best.cls > 0;
                 q.chosen[row] = sel ? best.d : -1;
                 q.lat[row] = sel ? best.C : __int_as_float(0x7fc00000);
                 q.util[row] = sel ? best.U : __int_as_float(0x7fc00000);
+                continue;
+            }
+            part[(size_t)un.part * q.Q + row] =
+                make_int4(best.cls, best.d, __float_as_int(best.C), __float_as_int(best.U));
+            __threadfence();
+            if (atomicAdd(&count[row], 1) == nsplit - 1) {
+                // last of this row's units: merge the parts (any order gives the
+                // same result: the candidate order is total)
+                __threadfence();
+                Cand acc = no_cand();
+                for (int pp = 0; pp < nsplit; ++pp) {
+                    const int4 x = __ldcg(&part[(size_t)pp * q.Q + row]);
+                    Cand c;
+                    c.cls = x.x;
+                    c.d = x.y;
+                    c.C = __int_as_float(x.z);
+                    c.U = __int_as_float(x.w);
+                    if (better(c, acc)) acc = c;
+                }
+                const bool sel = acc.cls > 0;
+                q.chosen[row] = sel ? acc.d : -1;
+                q.lat[row] = sel ? acc.C : __int_as_float(0x7fc00000);
+                q.util[row] = sel ? acc.U : __int_as_float(0x7fc00000);
+                count[row] = 0;
             }
         }
-    } else if (warp >= 6) {
-        // producers: layer-1 activations as bf16 in the UMMA operand layout.
-        // Thread p writes granule (p % 8) of rows p / 8 + 16 i, i < 8.
-        const int p = tid - 192, gi = p & 7, rb = p >> 3;
+    } else if (warp >= 5) {
+        // ---- producers: layer-1 activations as bf16 UMMA operand tiles ------
+        // Thread p owns granule gi = p % 8 (8 consecutive K) of every 64-wide K
+        // chunk, for rows rb + 32 i (i < 4).  The query part of layer 1,
+        // W1[:, in] u + W1[:, out] v, does not depend on the deployment: it is
+        // built once per unit in registers (bf16 pairs) and every step then
+        // needs one fused add + ReLU per pair: relu(1 * B + A_d).
+        const int p = tid - 160, gi = p & 7, rb = p >> 3;
+        uint32_t offs[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const int r = rb + 32 * i;
+            offs[i] = (uint32_t)(r >> 3) * 1024 + (uint32_t)(r & 7) * 128 +
+                      (uint32_t)((gi ^ (r & 7)) << 4);
+        }
+        const uint32_t one2 = 0x3F803F80u;  // (1.0, 1.0) in bf16
+        uint32_t Bq[4][4][4];
         uint32_t n = 0;
         bool ok = true;
-        for (int t = blockIdx.x; ok && t < ntiles; t += gridDim.x) {
-            float u[8], v[8];
+        for (int u = blockIdx.x; ok && u < nunits; u += gridDim.x) {
+            const Unit un = unit_of(u, ntiles, nsplit, D);
 #pragma unroll
-            for (int i = 0; i < 8; ++i) {
-                const int row = t * BM + rb + 16 * i;
+            for (int i = 0; i < 4; ++i) {
+                const int row = un.tile * BM + rb + 32 * i;
                 const bool valid = row < q.Q;
-                u[i] = valid ? standardise_fast(m.xf_in, q.in_len[row], m.mu_in, m.sd_in) : 0.f;
-                v[i] = valid ? standardise_fast(m.xf_out, q.out_len[row], m.mu_out, m.sd_out) : 0.f;
-            }
-            for (int d = 0; ok && d < D; ++d) {
-                const float *Ad = m.A + (size_t)d * H1;
-                for (int c = 0; c < nch; ++c, ++n) {
-                    const int s = n % NS;
-                    ok = mbar_wait(&empty[s], ((n / NS) & 1) ^ 1, abort_f, status);
-                    if (!ok) break;
-                    const int k0 = c * KCH + gi * 8;
-                    const float4 a0 = *(const float4 *)(Ad + k0), a1 = *(const float4 *)(Ad + k0 + 4);
-                    const float4 i0 = *(const float4 *)(m.W1q + k0), i1 = *(const float4 *)(m.W1q + k0 + 4);
-                    const float4 o0 = *(const float4 *)(m.W1q + H1 + k0),
-                                 o1 = *(const float4 *)(m.W1q + H1 + k0 + 4);
-                    const float a[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
-                    const float wi[8] = {i0.x, i0.y, i0.z, i0.w, i1.x, i1.y, i1.z, i1.w};
-                    const float wo[8] = {o0.x, o0.y, o0.z, o0.w, o1.x, o1.y, o1.z, o1.w};
-                    const uint32_t st = smem_u32(ring + s * CHUNK_BYTES);
+                const float uu = valid ? standardise_fast(m.xf_in, q.in_len[row], m.mu_in, m.sd_in) : 0.f;
+                const float vv = valid ? standardise_fast(m.xf_out, q.out_len[row], m.mu_out, m.sd_out) : 0.f;
 #pragma unroll
-                    for (int i = 0; i < 8; ++i) {
-                        const int r = rb + 16 * i;
-                        uint32_t pk[4];
+                for (int c = 0; c < 4; ++c) {
+                    if (c < nch) {
+                        const int k0 = c * KCH + gi * 8;
 #pragma unroll
                         for (int e = 0; e < 4; ++e) {
-                            const float x0 = fmaf(v[i], wo[2 * e], fmaf(u[i], wi[2 * e], a[2 * e]));
-                            const float x1 =
-                                fmaf(v[i], wo[2 * e + 1], fmaf(u[i], wi[2 * e + 1], a[2 * e + 1]));
-                            pk[e] = pack_relu_bf16x2(x0, x1);
+                            const float2 wi = *(const float2 *)(m.W1q + k0 + 2 * e);
+                            const float2 wo = *(const float2 *)(m.W1q + H1 + k0 + 2 * e);
+                            Bq[i][c][e] = pack_bf16x2(fmaf(vv, wo.x, uu * wi.x),
+                                                      fmaf(vv, wo.y, uu * wi.y));
                         }
-                        const uint32_t off = (uint32_t)(r >> 3) * 1024 + (uint32_t)(r & 7) * 128 +
-                                             (uint32_t)((gi ^ (r & 7)) << 4);
-                        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(st + off),
-                                     "r"(pk[0]), "r"(pk[1]), "r"(pk[2]), "r"(pk[3])
-                                     : "memory");
                     }
-                    fence_proxy_async_smem();
-                    mbar_arrive(&full[s]);
+                }
+            }
+            for (int d = un.d0; ok && d < un.d1; ++d) {
+                const uint4 *Ad = (const uint4 *)(m.Abf + (size_t)d * H1);
+                uint4 a[4];
+#pragma unroll
+                for (int c = 0; c < 4; ++c)
+                    if (c < nch) a[c] = __ldg(Ad + c * 8 + gi);
+#pragma unroll
+                for (int c = 0; c < 4; ++c) {
+                    if (c < nch && ok) {
+                        const int s = n % NS;
+                        ok = mbar_wait(&empty[s], ((n / NS) & 1) ^ 1, abort_f, status);
+                        if (ok) {
+                            const uint32_t st = smem_u32(ring + s * CHUNK_BYTES);
+#pragma unroll
+                            for (int i = 0; i < 4; ++i) {
+                                const uint32_t h0 = hfma2_relu(Bq[i][c][0], one2, a[c].x);
+                                const uint32_t h1 = hfma2_relu(Bq[i][c][1], one2, a[c].y);
+                                const uint32_t h2 = hfma2_relu(Bq[i][c][2], one2, a[c].z);
+                                const uint32_t h3 = hfma2_relu(Bq[i][c][3], one2, a[c].w);
+                                asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(
+                                                 st + offs[i]),
+                                             "r"(h0), "r"(h1), "r"(h2), "r"(h3)
+                                             : "memory");
+                            }
+                            fence_proxy_async_smem();
+                            mbar_arrive(&full[s]);
+                            ++n;
+                        }
+                    }
                 }
             }
         }
@@ -556,13 +663,30 @@ cudaError_t launch_qual_tc(const TcModel &m, const Queries &q, float *qual, int3
     return cudaGetLastError();
 }
 
-cudaError_t launch_mlp_tc(const TcModel &m, const Queries &q, const float *qual, int32_t *status,
-                          cudaStream_t s) {
+// Deployment split per tile that minimises the busiest CTA's step count
+// (each unit also pays about half a step of per-unit setup).
+int tc_mlp_split(const TcModel &m, int Q) {
+    const int ntiles = (Q + BM - 1) / BM, sms = g_num_sms > 0 ? g_num_sms : 1;
+    int best = 1;
+    double best_cost = 1e300;
+    for (int ns = 1; ns <= 8 && ns <= m.D; ++ns) {
+        const long units = (long)ntiles * ns;
+        const double cost = (double)((units + sms - 1) / sms) * ((m.D + ns - 1) / ns + 0.5);
+        if (cost < best_cost - 1e-9) {
+            best_cost = cost;
+            best = ns;
+        }
+    }
+    return best;
+}
+
+cudaError_t launch_mlp_tc(const TcModel &m, const Queries &q, const float *qual, int nsplit,
+                          void *part, int32_t *count, int32_t *status, cudaStream_t s) {
     if (q.Q <= 0) return cudaSuccess;
-    const int ntiles = (q.Q + BM - 1) / BM;
-    const int grid = ntiles < g_num_sms ? ntiles : g_num_sms;
+    const long units = (long)((q.Q + BM - 1) / BM) * nsplit;
+    const int grid = units < g_num_sms ? (int)units : g_num_sms;
     const MlpLayout L = mlp_layout(m.H1, m.H2, m.Mpad, m.D);
-    k_mlp_tc<<<grid, MLP_THREADS, L.total, s>>>(m, q, qual, status);
+    k_mlp_tc<<<grid, MLP_THREADS, L.total, s>>>(m, q, qual, nsplit, (int4 *)part, count, status);
     return cudaGetLastError();
 }
 
