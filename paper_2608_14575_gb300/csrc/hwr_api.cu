@@ -54,6 +54,7 @@ struct hwr_ctx {
     float *memb = nullptr;
     float *W1q = nullptr;            // [2][H1]
     uint16_t *W2img = nullptr, *membimg = nullptr;
+    std::vector<char> head_consts;   // output-layer constants for the tensor path
     int32_t *running = nullptr, *waiting = nullptr;
     float *kv = nullptr, *gpu_util = nullptr, *ttft = nullptr, *tpot = nullptr;
     float *X = nullptr, *Spre = nullptr, *A = nullptr;
@@ -215,6 +216,7 @@ static TcModel tc_view(const hwr_ctx *c) {
     t.b2 = c->b2; t.W3 = c->W3; t.b3 = c->b3; t.dep_model = c->dep_model;
     t.mu_in = c->mu_in; t.sd_in = c->sd_in; t.mu_out = c->mu_out; t.sd_out = c->sd_out;
     t.xf_in = c->xf_in; t.xf_out = c->xf_out;
+    t.head = (const HeadConsts *)c->head_consts.data();
     return t;
 }
 
@@ -425,6 +427,8 @@ static hwr_status build_ctx(hwr_ctx *c, const hwr_deployment_table *t, const hwr
         tc_build_membimg((const uint16_t *)memb_in, E, M, c->Mpad, c->Epad, mimg.data());
         TRY(dev_alloc(c, &c->membimg, mimg.size()));
         TRY(upload(c, c->membimg, mimg.data(), mimg.size() * 2, "upload memb image"));
+        c->head_consts.resize(tc_head_consts_bytes());
+        tc_fill_head_consts(c->head_consts.data(), p->b2, w3.data(), p->b3, H2);
     }
 
     // status word: mapped pinned host memory the kernels write directly

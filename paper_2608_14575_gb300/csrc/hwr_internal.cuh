@@ -73,8 +73,10 @@ size_t seq_table_smem(const Model &m);
 cudaError_t simt_prepare();   // one-time smem opt-in
 
 // ---- tcgen05 kernels (k_tc.cu) -------------------------------------------
+struct HeadConsts;
 struct TcModel {
     int M, Mpad, D, H1, H2, E, Epad;
+    const HeadConsts *head;     // host copy of b2, W3, b3 (kernel parameters)
     const uint16_t *W2img;      // bf16 W2 in the UMMA shared-memory image
     const uint16_t *membimg;    // bf16 memb^T in the UMMA shared-memory image
     const uint16_t *Abf;        // [D][H1] bf16 deployment prefix of layer 1
@@ -102,5 +104,7 @@ cudaError_t launch_mlp_tc(const TcModel &m, const Queries &q, const float *qual,
                           int nsplit, void *part, int32_t *count, int32_t *status,
                           cudaStream_t s);
 cudaError_t tc_prepare();
+size_t tc_head_consts_bytes();
+void tc_fill_head_consts(void *dst, const float *b2, const float *W3, const float *b3, int H2);
 
 }  // namespace hwr

@@ -345,12 +345,21 @@ __device__ __forceinline__ void head_pair(const uint32_t *v, int j, const float4
     t1b = __ffma2_rn(x23, make_float2(w1.z, w1.w), t1b);
 }
 
+// Output-layer constants passed by value: they sit in the kernel-parameter
+// constant bank, so the fully unrolled epilogue reads them as instruction
+// operands instead of shared-memory loads.
+struct HeadConsts {
+    float b2[MAX_H], w0[MAX_H], w1[MAX_H], b3[2];
+};
+
+template <int H2T>
 __global__ void __launch_bounds__(MLP_THREADS, 1)
-k_mlp_tc(TcModel m, Queries q, const float *__restrict__ qual, int nsplit, int4 *part,
-         int32_t *count, int32_t *status) {
+k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
+         const float *__restrict__ qual, int nsplit, int4 *part, int32_t *count, int32_t *status) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *sm = align1024(smem_raw);
-    const int H1 = m.H1, H2 = m.H2, D = m.D, Mpad = m.Mpad, QS = Mpad + 1;
+    constexpr bool FIXED = H2T > 0;
+    const int H1 = m.H1, H2 = FIXED ? H2T : m.H2, D = m.D, Mpad = m.Mpad, QS = Mpad + 1;
     const MlpLayout L = mlp_layout(H1, H2, Mpad, D);
     const int NS = L.ns;
     uint8_t *w2s = sm + L.w2, *ring = sm + L.ring;
@@ -463,21 +472,40 @@ k_mlp_tc(TcModel m, Queries q, const float *__restrict__ qual, int nsplit, int4 
                 float2 t0a = make_float2(0.f, 0.f), t0b = t0a, t1a = t0a, t1b = t0a;
                 uint32_t va[32], vb[32];
                 tmem_ld32(base, va);
-                for (int c = 0; c < ncol; c += 2) {
-                    tmem_wait_ld32(va);
-                    if (c + 1 < ncol) tmem_ld32(base + (c + 1) * 32, vb);
+                if constexpr (FIXED) {
+                    constexpr int NC = H2T / 32;
 #pragma unroll
-                    for (int j = 0; j < 32; j += 4) {
-                        const int f = (c * 32 + j) >> 2;
-                        head_pair(va, j, b2v[f], w0v[f], w1v[f], t0a, t0b, t1a, t1b);
-                    }
-                    if (c + 1 < ncol) {
-                        tmem_wait_ld32(vb);
-                        if (c + 2 < ncol) tmem_ld32(base + (c + 2) * 32, va);
+                    for (int c = 0; c < NC; ++c) {
+                        uint32_t(&cur)[32] = (c & 1) ? vb : va;
+                        uint32_t(&nxt)[32] = (c & 1) ? va : vb;
+                        tmem_wait_ld32(cur);
+                        if (c + 1 < NC) tmem_ld32(base + (c + 1) * 32, nxt);
 #pragma unroll
                         for (int j = 0; j < 32; j += 4) {
-                            const int f = ((c + 1) * 32 + j) >> 2;
-                            head_pair(vb, j, b2v[f], w0v[f], w1v[f], t0a, t0b, t1a, t1b);
+                            const int n = c * 32 + j;
+                            head_pair(cur, j, make_float4(hc.b2[n], hc.b2[n + 1], hc.b2[n + 2], hc.b2[n + 3]),
+                                      make_float4(hc.w0[n], hc.w0[n + 1], hc.w0[n + 2], hc.w0[n + 3]),
+                                      make_float4(hc.w1[n], hc.w1[n + 1], hc.w1[n + 2], hc.w1[n + 3]),
+                                      t0a, t0b, t1a, t1b);
+                        }
+                    }
+                } else {
+                    for (int c = 0; c < ncol; c += 2) {
+                        tmem_wait_ld32(va);
+                        if (c + 1 < ncol) tmem_ld32(base + (c + 1) * 32, vb);
+#pragma unroll
+                        for (int j = 0; j < 32; j += 4) {
+                            const int f = (c * 32 + j) >> 2;
+                            head_pair(va, j, b2v[f], w0v[f], w1v[f], t0a, t0b, t1a, t1b);
+                        }
+                        if (c + 1 < ncol) {
+                            tmem_wait_ld32(vb);
+                            if (c + 2 < ncol) tmem_ld32(base + (c + 2) * 32, va);
+#pragma unroll
+                            for (int j = 0; j < 32; j += 4) {
+                                const int f = ((c + 1) * 32 + j) >> 2;
+                                head_pair(vb, j, b2v[f], w0v[f], w1v[f], t0a, t0b, t1a, t1b);
+                            }
                         }
                     }
                 }
@@ -564,12 +592,18 @@ k_mlp_tc(TcModel m, Queries q, const float *__restrict__ qual, int nsplit, int4 
                     }
                 }
             }
-            for (int d = un.d0; ok && d < un.d1; ++d) {
-                const uint4 *Ad = (const uint4 *)(m.Abf + (size_t)d * H1);
-                uint4 a[4];
+            uint4 a[4], an[4];
 #pragma unroll
-                for (int c = 0; c < 4; ++c)
-                    if (c < nch) a[c] = __ldg(Ad + c * 8 + gi);
+            for (int c = 0; c < 4; ++c)
+                if (c < nch) a[c] = __ldg((const uint4 *)(m.Abf + (size_t)un.d0 * H1) + c * 8 + gi);
+            for (int d = un.d0; ok && d < un.d1; ++d) {
+                // prefetch the next deployment's prefix while this one is built
+                if (d + 1 < un.d1) {
+                    const uint4 *An = (const uint4 *)(m.Abf + (size_t)(d + 1) * H1);
+#pragma unroll
+                    for (int c = 0; c < 4; ++c)
+                        if (c < nch) an[c] = __ldg(An + c * 8 + gi);
+                }
 #pragma unroll
                 for (int c = 0; c < 4; ++c) {
                     if (c < nch && ok) {
@@ -594,6 +628,8 @@ k_mlp_tc(TcModel m, Queries q, const float *__restrict__ qual, int nsplit, int4 
                         }
                     }
                 }
+#pragma unroll
+                for (int c = 0; c < 4; ++c) a[c] = an[c];
             }
         }
     }
@@ -639,7 +675,11 @@ cudaError_t tc_prepare() {
     cudaError_t e = cudaFuncSetAttribute(k_qual_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          SMEM_LIMIT);
     if (e == cudaSuccess)
-        e = cudaFuncSetAttribute(k_mlp_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_LIMIT);
+        e = cudaFuncSetAttribute(k_mlp_tc<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_LIMIT);
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(k_mlp_tc<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_LIMIT);
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(k_mlp_tc<256>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_LIMIT);
     return e;
 }
 
@@ -686,8 +726,28 @@ cudaError_t launch_mlp_tc(const TcModel &m, const Queries &q, const float *qual,
     const long units = (long)((q.Q + BM - 1) / BM) * nsplit;
     const int grid = units < g_num_sms ? (int)units : g_num_sms;
     const MlpLayout L = mlp_layout(m.H1, m.H2, m.Mpad, m.D);
-    k_mlp_tc<<<grid, MLP_THREADS, L.total, s>>>(m, q, qual, nsplit, (int4 *)part, count, status);
+    const HeadConsts &hc = *m.head;
+    if (m.H2 == 256)
+        k_mlp_tc<256><<<grid, MLP_THREADS, L.total, s>>>(m, q, hc, qual, nsplit, (int4 *)part, count, status);
+    else if (m.H2 == 128)
+        k_mlp_tc<128><<<grid, MLP_THREADS, L.total, s>>>(m, q, hc, qual, nsplit, (int4 *)part, count, status);
+    else
+        k_mlp_tc<0><<<grid, MLP_THREADS, L.total, s>>>(m, q, hc, qual, nsplit, (int4 *)part, count, status);
     return cudaGetLastError();
+}
+
+size_t tc_head_consts_bytes() { return sizeof(HeadConsts); }
+
+void tc_fill_head_consts(void *dst, const float *b2, const float *W3, const float *b3, int H2) {
+    HeadConsts *h = (HeadConsts *)dst;
+    memset(h, 0, sizeof *h);
+    for (int i = 0; i < H2; ++i) {
+        h->b2[i] = b2[i];
+        h->w0[i] = W3[i];
+        h->w1[i] = W3[H2 + i];
+    }
+    h->b3[0] = b3[0];
+    h->b3[1] = b3[1];
 }
 
 }  // namespace hwr
