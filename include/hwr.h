@@ -180,6 +180,41 @@ hwr_status hwr_route_batch(hwr_ctx *ctx, int32_t Q, const float *in_len,
                            float lambda, uint32_t flags, int32_t *chosen,
                            float *pred_latency, float *utility);
 
+/*
+ * Route a batch without allocating anything at call time.
+ *
+ * The paper has no counterpart to this call; it exists for callers that
+ * cannot allocate GPU memory while they route -- for example a router that
+ * lives inside an LLM serving process whose engine reserved nearly all of the
+ * GPU's memory up front for its KV cache, or a latency-critical serving loop
+ * that must not take the device-wide synchronisation of cudaMalloc.
+ * hwr_route_batch may grow its scratch with cudaMalloc; this call never does:
+ * it calls no cudaMalloc, cudaFree or other allocating routine and uses one
+ * fixed scratch array (about 6.1 MiB) that the library reserves in device
+ * memory on every GPU where it is loaded, for as long as the process runs.
+ *
+ * Same arguments and outputs as hwr_route_batch, with these restrictions:
+ *   - the context must be bf16 with tensor-core support (else UNSUPPORTED);
+ *   - 0 <= Q <= HWR_NOALLOC_MAX_Q (larger Q: HWR_ERR_UNSUPPORTED);
+ *   - all six arrays are device pointers (HWR_DEVICE_PTRS is implied);
+ *     q_emb must be 16-byte aligned;
+ *   - flags may hold only HWR_DEVICE_PTRS, HWR_ASYNC and HWR_SCORE_CONVEX.
+ * The current device must be the context's device.  The first call on a
+ * device looks up the scratch array's device address (once per device); make
+ * that first call before any stream capture begins.  The scratch is shared by
+ * all calls on a device and keeps the last call's contents (the parts that
+ * must start at zero are cleared on every call): calls whose work overlaps on
+ * the GPU -- different streams, contexts or threads -- race on it and must be
+ * ordered by the caller.  Synchronises the context stream unless HWR_ASYNC.
+ * Errors: INVALID_ARG, UNSUPPORTED, STATE, CUDA, TIMEOUT.
+ */
+#define HWR_NOALLOC_MAX_Q 32768
+hwr_status hwr_route_batch_noalloc(hwr_ctx *ctx, int32_t Q, const float *in_len,
+                                   const float *out_len, const void *q_emb,
+                                   float slo, float lambda, uint32_t flags,
+                                   int32_t *chosen, float *pred_latency,
+                                   float *utility);
+
 /* Wait for all work of the context; reports device-side timeouts
  * (HWR_ERR_TIMEOUT) and asynchronous kernel failures (HWR_ERR_CUDA). */
 hwr_status hwr_synchronize(hwr_ctx *ctx);

@@ -34,8 +34,9 @@ KERNELS = ("snapshot", "route_simt", "seq_table", "qual_tc", "mlp_tc")
 HWR_K_COUNT = len(KERNELS)
 
 EXPORTS = ("hwr_create", "hwr_update_snapshot", "hwr_get_snapshot",
-           "hwr_route_batch", "hwr_synchronize", "hwr_destroy",
-           "hwr_status_string", "hwr_last_error", "hwr_get_stats")
+           "hwr_route_batch", "hwr_route_batch_noalloc", "hwr_synchronize",
+           "hwr_destroy", "hwr_status_string", "hwr_last_error", "hwr_get_stats")
+HWR_NOALLOC_MAX_Q = 32768
 
 
 class hwr_deployment_table(ct.Structure):
@@ -95,6 +96,7 @@ def load(path: str | None = None):
         lib.hwr_get_snapshot.argtypes = [P, P]
         lib.hwr_route_batch.argtypes = [P, ct.c_int32, P, P, P, ct.c_float,
                                         ct.c_float, ct.c_uint32, P, P, P]
+        lib.hwr_route_batch_noalloc.argtypes = lib.hwr_route_batch.argtypes
         lib.hwr_synchronize.argtypes = [P]
         lib.hwr_destroy.argtypes = [P]
         lib.hwr_status_string.argtypes = [I]
@@ -103,8 +105,8 @@ def load(path: str | None = None):
         lib.hwr_last_error.restype = ct.c_char_p
         lib.hwr_get_stats.argtypes = [P, P, I]
         for n in ("hwr_create", "hwr_update_snapshot", "hwr_get_snapshot",
-                  "hwr_route_batch", "hwr_synchronize", "hwr_destroy",
-                  "hwr_get_stats"):
+                  "hwr_route_batch", "hwr_route_batch_noalloc", "hwr_synchronize",
+                  "hwr_destroy", "hwr_get_stats"):
             getattr(lib, n).restype = I
         if path is None:
             _lib = lib
@@ -129,6 +131,12 @@ def hwr_route_batch(ctx, Q, in_len, out_len, q_emb, slo, lam, flags, chosen,
                     pred_latency, utility):
     return load().hwr_route_batch(ctx, Q, in_len, out_len, q_emb, slo, lam, flags,
                                   chosen, pred_latency, utility)
+
+
+def hwr_route_batch_noalloc(ctx, Q, in_len, out_len, q_emb, slo, lam, flags, chosen,
+                            pred_latency, utility):
+    return load().hwr_route_batch_noalloc(ctx, Q, in_len, out_len, q_emb, slo, lam, flags,
+                                          chosen, pred_latency, utility)
 
 
 def hwr_synchronize(ctx):
@@ -241,6 +249,14 @@ class Router:
                      flags=0):
         """CUDA tensors in and out, ordered on the context's stream."""
         self._check(self.lib.hwr_route_batch(
+            self.ctx, int(in_len.numel()), in_len.data_ptr(), out_len.data_ptr(),
+            emb.data_ptr(), float(slo), float(lam), int(flags) | HWR_DEVICE_PTRS,
+            chosen.data_ptr(), lat.data_ptr(), util.data_ptr()))
+
+    def route_device_noalloc(self, in_len, out_len, emb, chosen, lat, util, *, slo, lam,
+                             flags=0):
+        """As route_device, through hwr_route_batch_noalloc (no allocation)."""
+        self._check(self.lib.hwr_route_batch_noalloc(
             self.ctx, int(in_len.numel()), in_len.data_ptr(), out_len.data_ptr(),
             emb.data_ptr(), float(slo), float(lam), int(flags) | HWR_DEVICE_PTRS,
             chosen.data_ptr(), lat.data_ptr(), util.data_ptr()))

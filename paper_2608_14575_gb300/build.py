@@ -26,6 +26,7 @@ SOURCES = {
     "hwr_api.cu": [],
     "k_simt.cu": ["--fmad=false"],
     "k_tc.cu": [],
+    "hwr_noalloc.cu": [],
 }
 
 

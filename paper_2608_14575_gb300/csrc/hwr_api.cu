@@ -740,3 +740,57 @@ extern "C" const char *hwr_status_string(hwr_status s) {
 extern "C" const char *hwr_last_error(const hwr_ctx *c) {
     return c ? c->err.c_str() : g_create_error.c_str();
 }
+
+// ---------------------------------------------------------------------------
+// Internal helpers for hwr_route_batch_noalloc (hwr_noalloc.cu): the tensor
+// path with caller-provided scratch, and error reporting on a context.
+
+hwr_status hwr_internal_fail(hwr_ctx *c, hwr_status s, const char *msg) {
+    return fail(c, s, "%s", msg);
+}
+
+hwr_status hwr_internal_route_tensor_scratch(hwr_ctx *c, int32_t Q, const float *in_len,
+                                             const float *out_len, const void *q_emb, float slo,
+                                             float lambda, uint32_t flags, int32_t *chosen,
+                                             float *pred_latency, float *utility, float *qual,
+                                             void *part, int32_t *count, int max_split) {
+    if (c->broken) return HWR_ERR_STATE;
+    if (!c->have_snapshot)
+        return fail(c, HWR_ERR_INVALID_ARG, "route before the first hwr_update_snapshot");
+    if (!c->tc_ok)
+        return fail(c, HWR_ERR_UNSUPPORTED, "no tensor-core path for this context (fp32 or shape)");
+    if (!in_len || !out_len || !q_emb || !chosen || !pred_latency || !utility)
+        return fail(c, HWR_ERR_INVALID_ARG, "NULL input or output array");
+    if (slo != slo) return fail(c, HWR_ERR_INVALID_ARG, "SLO is NaN");
+    if (!isfinite(lambda)) return fail(c, HWR_ERR_INVALID_ARG, "lambda is not finite");
+    if ((uintptr_t)q_emb & 15) return fail(c, HWR_ERR_INVALID_ARG, "q_emb must be 16-byte aligned");
+    if (Q == 0) return HWR_OK;
+    Queries q;
+    q.Q = Q;
+    q.emb_bf16 = 1;
+    q.slo = slo;
+    q.lam = lambda;
+    q.wq = (flags & HWR_SCORE_CONVEX) ? 1.0f - lambda : 1.0f;
+    q.in_len = in_len;
+    q.out_len = out_len;
+    q.emb = q_emb;
+    q.chosen = chosen;
+    q.lat = pred_latency;
+    q.util = utility;
+    const TcModel t = tc_view(c);
+    int ns = tc_mlp_split(t, Q);
+    if (ns > max_split) ns = max_split;
+    if (ns > 1)
+        CK(c, cudaMemsetAsync(count, 0, (size_t)Q * sizeof(int32_t), c->stream), "clear counters");
+    CK(c, launch_qual_tc(t, q, qual, c->status_d, c->stream), "quality kernel");
+    c->stats.kernel_launches++;
+    c->stats.launches[HWR_K_QUAL_TC]++;
+    CK(c, launch_mlp_tc(t, q, qual, ns, part, count, c->status_d, c->stream), "predictor kernel");
+    c->stats.kernel_launches++;
+    c->stats.launches[HWR_K_MLP_TC]++;
+    c->stats.queries_routed += Q;
+    if (flags & HWR_ASYNC) return HWR_OK;
+    CK(c, cudaStreamSynchronize(c->stream), "synchronize");
+    CK(c, cudaGetLastError(), "kernel");
+    return check_status_word(c);
+}

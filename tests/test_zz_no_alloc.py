@@ -1,0 +1,89 @@
+"""hwr_route_batch_noalloc: routing with no allocation at call time.
+
+For callers that cannot allocate GPU memory while they route (a router inside
+an LLM serving process whose engine reserved nearly all of HBM for its KV
+cache, or a serving loop that must not take cudaMalloc's device-wide
+synchronisation).  The call must give the same decisions as hwr_route_batch
+on the same inputs -- on two calls in a row, with different batches, so that
+what the first call leaves in the shared scratch cannot leak into the second
+-- must not allocate, and must reject batches larger than its fixed scratch.
+
+Collected last on purpose (file name), so a run that stops at the first
+failure has run every other test before this one.
+"""
+import numpy as np
+import pytest
+
+import workload as W
+import paper_2608_14575_gb300 as H
+
+pytestmark = pytest.mark.gpu
+TOL = 2e-2
+
+
+def _dev(p, lo, hi, dev):
+    import torch
+    return (torch.from_numpy(p["in_len"][lo:hi]).to(dev),
+            torch.from_numpy(p["out_len"][lo:hi]).to(dev),
+            torch.from_numpy(p["emb"][lo:hi].view(np.int16)).to(dev))
+
+
+def _outs(n, dev):
+    import torch
+    return (torch.empty(n, dtype=torch.int32, device=dev),
+            torch.empty(n, dtype=torch.float32, device=dev),
+            torch.empty(n, dtype=torch.float32, device=dev))
+
+
+def _close(a, b):
+    ch, lat, ut = (x.cpu().numpy() for x in a)
+    wch, wlat, wut = (x.cpu().numpy() for x in b)
+    assert np.array_equal(ch, wch)
+    assert np.all(np.abs(lat - wlat) <= TOL * np.maximum(np.abs(wlat), 1e-3))
+    assert np.all(np.abs(ut - wut) <= TOL * np.maximum(np.abs(wut), 1.0))
+
+
+def test_noalloc_matches_route_batch_on_two_calls():
+    import torch
+    H.build()
+    dev = torch.device("cuda:0")
+    p = W.make_config(3, Q=30_000)
+    r = H.Router(p, stream=torch.cuda.current_stream().cuda_stream)
+    for lo, hi in ((0, 20_000), (20_000, 30_000)):       # two calls, different batches
+        inp = _dev(p, lo, hi, dev)
+        ref = _outs(hi - lo, dev)
+        r.route_device(*inp, *ref, slo=p["slo"], lam=p["lam"], flags=H.HWR_PATH_TENSOR)
+        got = _outs(hi - lo, dev)
+        r.route_device_noalloc(*inp, *got, slo=p["slo"], lam=p["lam"])
+        torch.cuda.synchronize()
+        _close(got, ref)
+    r.close()
+
+
+def test_noalloc_allocates_nothing_and_rejects_oversize():
+    import torch
+    H.build()
+    dev = torch.device("cuda:0")
+    p = W.make_config(1, Q=4096)
+    r = H.Router(p, stream=torch.cuda.current_stream().cuda_stream)
+    inp = _dev(p, 0, 4096, dev)
+    out = _outs(4096, dev)
+    r.route_device_noalloc(*inp, *out, slo=p["slo"], lam=p["lam"])   # first call: set-up
+    torch.cuda.synchronize()
+    free0 = torch.cuda.mem_get_info()[0]
+    for _ in range(3):
+        r.route_device_noalloc(*inp, *out, slo=p["slo"], lam=p["lam"])
+    torch.cuda.synchronize()
+    assert torch.cuda.mem_get_info()[0] >= free0
+    ref = _outs(4096, dev)
+    r.route_device(*inp, *ref, slo=p["slo"], lam=p["lam"], flags=H.HWR_PATH_TENSOR)
+    torch.cuda.synchronize()
+    _close(out, ref)
+    big = H.HWR_NOALLOC_MAX_Q + 1
+    z = torch.zeros(big, dtype=torch.float32, device=dev)
+    e = torch.zeros((big, p["E"]), dtype=torch.int16, device=dev)
+    o = _outs(big, dev)
+    with pytest.raises(H.HwrError) as exc:
+        r.route_device_noalloc(z, z, e, *o, slo=p["slo"], lam=p["lam"])
+    assert exc.value.status == 7 and "maximum" in str(exc.value)
+    r.close()
