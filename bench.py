@@ -125,6 +125,46 @@ class ClockSampler:
                 "reasons": sorted(reasons), "samples": len(sm)}
 
 
+def kernel_sources_sha256():
+    """Hash of the sources the tensor-core kernels are built from."""
+    import hashlib
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2608_14575_gb300", "csrc")
+    for f in sorted(["k_tc.cu", "umma.cuh", "select.cuh", "hwr_internal.cuh"]):
+        with open(os.path.join(csrc, f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()
+
+
+def profiled_traffic(kernel):
+    """DRAM bytes per launch from the committed ncu capture, or None when the
+    kernel sources changed since the counters were taken."""
+    try:
+        with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
+            t = json.load(f)
+    except (OSError, ValueError):
+        return None
+    if t.get("sources_sha256") != kernel_sources_sha256():
+        return None
+    k = t.get("kernels", {}).get(kernel)
+    return None if k is None else k.get("dram_bytes_per_launch")
+
+
+def max_over_ranks(x, dist=None, device=None):
+    """Largest value of x over all ranks (x itself without a process group)."""
+    if dist is None:
+        return float(x)
+    import torch
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(queries_per_rank, world, seconds):
+    """Units processed by all ranks over the slowest rank's time."""
+    return world * queries_per_rank / seconds
+
+
 def dist_env():
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -136,7 +176,7 @@ def cpu_oracle_rate(p, seconds, nthreads):
     """Queries/s of the oracle (fp64 mode) on a sample sized to ~`seconds`."""
     import oracle as O
     orc = O.Problem(p)
-    n = 32
+    n = min(p["Q"], 64 * nthreads)
     t = time.perf_counter()
     orc.route(p["in_len"][:n], p["out_len"][:n], p["emb"][:n], nthreads=nthreads)
     per_q = (time.perf_counter() - t) / n
@@ -226,6 +266,7 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--no-q1", action="store_true")
+    ap.add_argument("--no-clocks", action="store_true")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
     rank, world, local = dist_env()
@@ -274,7 +315,8 @@ def main():
     r.stats(reset=True)
     before = r.stats()["kernel_launches"]
     clocks = ClockSampler(local)
-    clocks.start()
+    if not args.no_clocks:
+        clocks.start()
     if dist:
         dist.barrier()
     torch.cuda.synchronize()
@@ -287,14 +329,10 @@ def main():
     if dist:
         dist.barrier()
     clk = clocks.stop()
-    ms = e0.elapsed_time(e1) / args.steps
-    if dist:
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(e0.elapsed_time(e1) / args.steps, dist, dev)
     st = r.stats(reset=True)
     launches = st["kernel_launches"] - before
-    value = world * Q / (ms * 1e-3)
+    value = whole_job_rate(Q, world, ms * 1e-3)
 
     # dominant kernel and its roofline
     pk, src = peaks()
@@ -306,7 +344,7 @@ def main():
         flop = pairs * flops_per_pair(p)
         ach = flop / (kms[top] * 1e-3) / 1e12
         roof = {"bound": "tensor", "achieved": ach, "peak": pk["bf16_tflops"],
-                "unit": "TFLOP/s", "frac": ach / pk["bf16_tflops"], "traffic": None,
+                "unit": "TFLOP/s", "frac": ach / pk["bf16_tflops"], "traffic": profiled_traffic(top),
                 "kernel": top, "ms_per_launch": kms[top],
                 "peak_source": f"{src} bf16 burst (cuBLAS), frac vs sustained "
                                f"{ach / pk.get('bf16_tflops_sustained', pk['bf16_tflops']):.3f}"}
@@ -314,7 +352,7 @@ def main():
         byt = Q * bytes_per_query(p)
         ach = byt / (kms[top] * 1e-3) / 1e9
         roof = {"bound": "hbm", "achieved": ach, "peak": pk["hbm_gbs"], "unit": "GB/s",
-                "frac": ach / pk["hbm_gbs"], "traffic": None, "kernel": top,
+                "frac": ach / pk["hbm_gbs"], "traffic": profiled_traffic(top), "kernel": top,
                 "ms_per_launch": kms[top], "peak_source": f"{src} copy bandwidth"}
     else:
         flop = pairs * flops_per_pair(p)
@@ -356,12 +394,8 @@ def main():
         t = time.perf_counter()
         for _ in range(args.steps):
             host_step()
-        dt = (time.perf_counter() - t) / args.steps
-        if dist:
-            tt = torch.tensor([dt], device=dev)
-            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-            dt = float(tt.item())
-        line["e2e"] = {"value": world * Q / dt, "unit": "queries/s",
+        dt = max_over_ranks((time.perf_counter() - t) / args.steps, dist, dev)
+        line["e2e"] = {"value": whole_job_rate(Q, world, dt), "unit": "queries/s",
                        "h2d_bytes_per_step": Q * (bytes_per_query(p) - 12),
                        "d2h_bytes_per_step": Q * 12, "ms_per_step": dt * 1e3}
     if rank == 0 and not args.no_q1:

@@ -22,8 +22,10 @@ namespace {
 
 thread_local std::string g_create_error;
 
-// Host-side fault hook for tests: HWR_TEST_FAIL_ALLOC=n makes the n-th
-// allocation of a context (counting from 1) report failure.
+// Host-side fault hooks for tests, read at hwr_create: HWR_TEST_FAIL_ALLOC=n
+// makes the n-th allocation of the context (counting from 1) report failure;
+// HWR_TEST_STALL=1 makes the tensor-path producers never signal their tiles,
+// so the predictor kernel's bounded waits run out (HWR_ERR_TIMEOUT).
 struct AllocHook {
     long fail_at = 0, count = 0;
 };
@@ -41,6 +43,7 @@ struct hwr_ctx {
     bool own_stream = false;
     bool broken = false;
     bool have_snapshot = false;
+    int test_stall = 0;          // HWR_TEST_STALL: tensor-path producers never signal
     std::string err;
     AllocHook hook;
     std::vector<void *> allocs;  // device buffers (cudaMalloc)
@@ -217,6 +220,7 @@ static TcModel tc_view(const hwr_ctx *c) {
     t.mu_in = c->mu_in; t.sd_in = c->sd_in; t.mu_out = c->mu_out; t.sd_out = c->sd_out;
     t.xf_in = c->xf_in; t.xf_out = c->xf_out;
     t.head = (const HeadConsts *)c->head_consts.data();
+    t.test_stall = c->test_stall;
     return t;
 }
 
@@ -483,6 +487,7 @@ extern "C" hwr_status hwr_create(const hwr_deployment_table *table, const hwr_pr
     c->F = pred->F; c->H1 = pred->H1; c->H2 = pred->H2; c->E = E; c->P = c->M + c->G;
     c->dtype = pred->dtype;
     if (const char *h = getenv("HWR_TEST_FAIL_ALLOC")) c->hook.fail_at = atol(h);
+    if (const char *h = getenv("HWR_TEST_STALL")) c->test_stall = atoi(h) != 0;
     s = build_ctx(c, table, pred, model_emb, cuda_stream);
     if (s != HWR_OK) {
         g_create_error = c->err;

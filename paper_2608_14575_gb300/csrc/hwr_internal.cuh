@@ -85,6 +85,7 @@ struct TcModel {
     const int32_t *dep_model;
     float mu_in, sd_in, mu_out, sd_out;
     uint8_t xf_in, xf_out;
+    int test_stall;             // test hook: producers never signal (bounded waits expire)
 };
 bool tc_supported(int M, int H1, int H2, int E);
 size_t tc_w2img_elems(int H1, int H2);

@@ -623,7 +623,7 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
                                              : "memory");
                             }
                             fence_proxy_async_smem();
-                            mbar_arrive(&full[s]);
+                            if (!m.test_stall) mbar_arrive(&full[s]);
                             ++n;
                         }
                     }
