@@ -30,7 +30,14 @@ struct AllocHook {
     long fail_at = 0, count = 0;
 };
 
-constexpr int TC_MIN_Q = 512;  // below this the fused SIMT kernel is faster
+// Path thresholds, from a sweep of batch sizes on GB300 (defaults;
+// HWR_TC_MIN_PAIRS and HWR_PAIRS_MAX_PAIRS override them at hwr_create):
+// batches of at most pairs_max pairs (Q * D) take the small-batch SIMT
+// kernel; larger bf16 batches of at least tc_min_pairs pairs take the
+// tensor-core kernels; the rest the fused SIMT kernel.
+constexpr int TC_MIN_PAIRS = 513;
+constexpr int PIPE_CHUNK_MIN = 8192;   // smallest chunk of a pipelined host batch
+constexpr int SMALL_MAX_PAIRS = 512;
 
 }  // namespace
 
@@ -44,6 +51,7 @@ struct hwr_ctx {
     bool broken = false;
     bool have_snapshot = false;
     int test_stall = 0;          // HWR_TEST_STALL: tensor-path producers never signal
+    int tc_min_pairs = TC_MIN_PAIRS, pairs_max = SMALL_MAX_PAIRS;
     std::string err;
     AllocHook hook;
     std::vector<void *> allocs;  // device buffers (cudaMalloc)
@@ -56,6 +64,7 @@ struct hwr_ctx {
     uint8_t *xform = nullptr;
     float *memb = nullptr;
     float *W1q = nullptr;            // [2][H1]
+    float *W2T = nullptr;            // [H1][H2] fp32, for the small-batch kernel
     uint16_t *W2img = nullptr, *membimg = nullptr;
     std::vector<char> head_consts;   // output-layer constants for the tensor path
     int32_t *running = nullptr, *waiting = nullptr;
@@ -78,6 +87,7 @@ struct hwr_ctx {
     float *qual = nullptr;   size_t qual_cap = 0;     // [Q][Mpad]
     char *part = nullptr;    size_t part_cap = 0;     // split-deployment partials
     int32_t *count = nullptr; size_t count_cap = 0;   // per-row arrivals (self-resetting)
+    float *pairC = nullptr;  float *pairQ = nullptr;  int32_t *pairN = nullptr;  // small batches
     float *ctab = nullptr;   size_t ctab_cap = 0;
     float *qseq = nullptr;   size_t qseq_cap = 0;
     int seq_qs = 0;
@@ -87,6 +97,11 @@ struct hwr_ctx {
     char *out_d = nullptr;   size_t out_cap = 0;
     char *pin_h = nullptr;   size_t pin_cap = 0;       // pinned host staging
     cudaEvent_t pin_ev = nullptr;
+    // large host-pointer batches: chunked copies on a second stream overlap
+    // the kernels of the previous chunk
+    cudaStream_t copy_stream = nullptr;
+    cudaEvent_t chunk_ev[8] = {};
+    cudaEvent_t io_free_ev = nullptr;   // earlier work on the context stream is done
 
     // profiling
     struct Pending { int k; cudaEvent_t a, b; };
@@ -377,6 +392,10 @@ static hwr_status build_ctx(hwr_ctx *c, const hwr_deployment_table *t, const hwr
     TRY(dev_alloc(c, &c->xform, F));
     TRY(dev_alloc(c, &c->memb, me.size()));
     TRY(dev_alloc(c, &c->W1q, 2 * (size_t)H1));
+    TRY(dev_alloc(c, &c->W2T, (size_t)H1 * H2));
+    TRY(dev_alloc(c, &c->pairC, (size_t)PAIRS_MAX_PAIRS));
+    TRY(dev_alloc(c, &c->pairQ, (size_t)PAIRS_MAX_PAIRS * M));
+    TRY(dev_alloc(c, &c->pairN, (size_t)PAIRS_MAX_PAIRS));
     TRY(dev_alloc(c, &c->running, D));
     TRY(dev_alloc(c, &c->waiting, D));
     TRY(dev_alloc(c, &c->kv, D));
@@ -407,6 +426,11 @@ static hwr_status build_ctx(hwr_ctx *c, const hwr_deployment_table *t, const hwr
         w1q[H1 + j] = w1[(size_t)j * F + F - 1];
     }
     TRY(upload(c, c->W1q, w1q.data(), w1q.size() * 4, "upload W1 query columns"));
+    std::vector<float> w2t((size_t)H1 * H2);
+    for (int n = 0; n < H2; ++n)
+        for (int k = 0; k < H1; ++k) w2t[(size_t)k * H2 + n] = w2[(size_t)n * H1 + k];
+    TRY(upload(c, c->W2T, w2t.data(), w2t.size() * 4, "upload W2 transposed"));
+    CK(c, cudaMemset(c->pairN, 0, PAIRS_MAX_PAIRS * sizeof(int32_t)), "zero counters");
     c->mu_in = p->feat_mean[F - 2]; c->sd_in = p->feat_std[F - 2]; c->xf_in = p->feat_xform[F - 2];
     c->mu_out = p->feat_mean[F - 1]; c->sd_out = p->feat_std[F - 1]; c->xf_out = p->feat_xform[F - 1];
 
@@ -447,6 +471,10 @@ static hwr_status build_ctx(hwr_ctx *c, const hwr_deployment_table *t, const hwr
     TRY(dev_alloc(c, (char **)&c->snap_d, 6 * (size_t)D * 4));
     CK(c, cudaEventCreateWithFlags(&c->snap_ev, cudaEventDisableTiming), "create event");
     CK(c, cudaEventCreateWithFlags(&c->pin_ev, cudaEventDisableTiming), "create event");
+    CK(c, cudaStreamCreateWithFlags(&c->copy_stream, cudaStreamNonBlocking), "create copy stream");
+    for (auto &e : c->chunk_ev)
+        CK(c, cudaEventCreateWithFlags(&e, cudaEventDisableTiming), "create event");
+    CK(c, cudaEventCreateWithFlags(&c->io_free_ev, cudaEventDisableTiming), "create event");
 
     c->seq_qs = seq_chunk(model_view(c));
     CK(c, cudaDeviceSynchronize(), "create");
@@ -467,6 +495,13 @@ static void free_ctx(hwr_ctx *c) {
     if (c->pin_h) cudaFreeHost(c->pin_h);
     if (c->snap_ev) cudaEventDestroy(c->snap_ev);
     if (c->pin_ev) cudaEventDestroy(c->pin_ev);
+    for (auto e : c->chunk_ev)
+        if (e) cudaEventDestroy(e);
+    if (c->io_free_ev) cudaEventDestroy(c->io_free_ev);
+    if (c->copy_stream) {
+        cudaStreamSynchronize(c->copy_stream);
+        cudaStreamDestroy(c->copy_stream);
+    }
     if (c->own_stream && c->stream) cudaStreamDestroy(c->stream);
     cudaGetLastError();
     delete c;
@@ -488,6 +523,9 @@ extern "C" hwr_status hwr_create(const hwr_deployment_table *table, const hwr_pr
     c->dtype = pred->dtype;
     if (const char *h = getenv("HWR_TEST_FAIL_ALLOC")) c->hook.fail_at = atol(h);
     if (const char *h = getenv("HWR_TEST_STALL")) c->test_stall = atoi(h) != 0;
+    if (const char *h = getenv("HWR_TC_MIN_PAIRS")) c->tc_min_pairs = atoi(h) > 1 ? atoi(h) : 1;
+    if (const char *h = getenv("HWR_PAIRS_MAX_PAIRS"))
+        c->pairs_max = atoi(h) < 0 ? 0 : (atoi(h) > PAIRS_MAX_PAIRS ? PAIRS_MAX_PAIRS : atoi(h));
     s = build_ctx(c, table, pred, model_emb, cuda_stream);
     if (s != HWR_OK) {
         g_create_error = c->err;
@@ -599,7 +637,11 @@ static hwr_status run_kernels(hwr_ctx *c, const Queries &q, uint32_t flags, bool
         return HWR_OK;
     }
     LaunchScope a(c, HWR_K_ROUTE_SIMT, prof);
-    CK(c, launch_route_simt(m, q, c->stream), "route kernel");
+    if ((long)q.Q * c->D <= c->pairs_max)
+        CK(c, launch_route_pairs(m, q, c->W2T, c->pairC, c->pairQ, c->pairN, c->stream),
+           "route kernel");
+    else
+        CK(c, launch_route_simt(m, q, c->stream), "route kernel");
     a.done();
     return HWR_OK;
 }
@@ -630,7 +672,9 @@ extern "C" hwr_status hwr_route_batch(hwr_ctx *c, int32_t Q, const float *in_len
         return fail(c, HWR_ERR_UNSUPPORTED, "tensor-core path unavailable for this %s",
                     seq ? "sequential call" : "context (fp32 or unsupported shape)");
     const bool tensor = !seq && c->tc_ok &&
-                        ((flags & HWR_PATH_TENSOR) || (!(flags & HWR_PATH_SIMT) && Q >= TC_MIN_Q));
+                        ((flags & HWR_PATH_TENSOR) ||
+                         (!(flags & HWR_PATH_SIMT) && (long)Q * c->D >= c->tc_min_pairs &&
+                          (long)Q * c->D > c->pairs_max));
     const bool dev = flags & HWR_DEVICE_PTRS;
     const size_t es = c->dtype == HWR_BF16 ? 2 : 4;
     if (dev && tensor && ((uintptr_t)q_emb & 15))
@@ -649,6 +693,11 @@ extern "C" hwr_status hwr_route_batch(hwr_ctx *c, int32_t Q, const float *in_len
     const size_t o_lat = align_up(len_b, 256), o_util = o_lat + align_up(len_b, 256);
     const size_t out_total = o_util + len_b;
     const bool packed = !dev && !(flags & HWR_ASYNC) && in_total <= ((size_t)1 << 20);
+    // Large host batches: copy in chunks on the copy stream while the kernels
+    // of the previous chunk run (the link, not the GPU, bounds this path).
+    const int nchunk = (!dev && !packed && !seq && Q >= 2 * PIPE_CHUNK_MIN)
+                           ? (Q / PIPE_CHUNK_MIN < 8 ? Q / PIPE_CHUNK_MIN : 8) : 1;
+    const bool pipelined = nchunk > 1;
 
     if (dev) {
         q.in_len = in_len; q.out_len = out_len; q.emb = q_emb;
@@ -664,7 +713,7 @@ extern "C" hwr_status hwr_route_batch(hwr_ctx *c, int32_t Q, const float *in_len
             memcpy(c->pin_h + off_out, out_len, len_b);
             CK(c, cudaMemcpyAsync(c->io_d, c->pin_h, in_total, cudaMemcpyHostToDevice, c->stream),
                "copy inputs");
-        } else {
+        } else if (!pipelined) {
             CK(c, cudaMemcpyAsync(c->io_d, q_emb, emb_b, cudaMemcpyHostToDevice, c->stream), "copy emb");
             CK(c, cudaMemcpyAsync(c->io_d + off_in, in_len, len_b, cudaMemcpyHostToDevice, c->stream),
                "copy in_len");
@@ -679,7 +728,37 @@ extern "C" hwr_status hwr_route_batch(hwr_ctx *c, int32_t Q, const float *in_len
         q.util = (float *)(c->out_d + o_util);
     }
 
-    TRY(run_kernels(c, q, flags, tensor));
+    if (pipelined) {
+        // everything already queued on the context stream (earlier calls'
+        // kernels read io_d) must finish before io_d is rewritten
+        CK(c, cudaEventRecord(c->io_free_ev, c->stream), "record");
+        CK(c, cudaStreamWaitEvent(c->copy_stream, c->io_free_ev, 0), "order copies");
+        const int per = ((Q + nchunk - 1) / nchunk + 127) / 128 * 128;
+        int k = 0;
+        for (int lo = 0; lo < Q; lo += per, ++k) {
+            const int n = Q - lo < per ? Q - lo : per;
+            const size_t eo = (size_t)lo * c->E * es, eb = (size_t)n * c->E * es;
+            CK(c, cudaMemcpyAsync(c->io_d + eo, (const char *)q_emb + eo, eb, cudaMemcpyHostToDevice,
+                                  c->copy_stream), "copy emb");
+            CK(c, cudaMemcpyAsync(c->io_d + off_in + (size_t)lo * 4, in_len + lo, (size_t)n * 4,
+                                  cudaMemcpyHostToDevice, c->copy_stream), "copy in_len");
+            CK(c, cudaMemcpyAsync(c->io_d + off_out + (size_t)lo * 4, out_len + lo, (size_t)n * 4,
+                                  cudaMemcpyHostToDevice, c->copy_stream), "copy out_len");
+            CK(c, cudaEventRecord(c->chunk_ev[k], c->copy_stream), "record");
+            CK(c, cudaStreamWaitEvent(c->stream, c->chunk_ev[k], 0), "order kernels");
+            Queries qc = q;
+            qc.Q = n;
+            qc.emb = c->io_d + eo;
+            qc.in_len = q.in_len + lo;
+            qc.out_len = q.out_len + lo;
+            qc.chosen = q.chosen + lo;
+            qc.lat = q.lat + lo;
+            qc.util = q.util + lo;
+            TRY(run_kernels(c, qc, flags, tensor));
+        }
+    } else {
+        TRY(run_kernels(c, q, flags, tensor));
+    }
 
     bool synced = false;
     if (!dev) {

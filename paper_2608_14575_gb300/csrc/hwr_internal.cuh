@@ -59,6 +59,13 @@ struct Queries {
 cudaError_t launch_snapshot(const Model &m, cudaStream_t s);
 // Fused gather -> MLP -> mask -> argmax for a batch.
 cudaError_t launch_route_simt(const Model &m, const Queries &q, cudaStream_t s);
+// Small-batch (latency) variant: one block per (query, deployment) pair plus
+// quality blocks; scratch pairC [Q][D], qualS [Q][M], count [Q] (zeroed once,
+// self-resetting).  W2T is W2 transposed ([H1][H2], fp32).
+constexpr int PAIRS_MAX_PAIRS = 2048;   // default upper bound on Q * D for this kernel
+cudaError_t launch_route_pairs(const Model &m, const Queries &q, const float *W2T, float *pairC,
+                               float *qualS, int32_t *count, cudaStream_t s);
+size_t route_pairs_smem(const Model &m);
 // Sequential mode over one chunk of Qs <= seq_chunk(m) queries: the score
 // table (every (picks c, deployment d, query i >= c)), then the serial chain.
 //   ctab: scratch of seq_table_floats(D, Qs) floats; qual: Qs * M floats.

@@ -459,6 +459,138 @@ k_seq_chain(Model m, Queries q, int Qs, const float *ctab, const float *qualS) {
 }
 
 // ---------------------------------------------------------------------------
+// K_route_pairs: the small-batch (latency) variant.  One block per (query,
+// deployment) pair computes that pair's predictor with one thread per hidden
+// unit (W2 read transposed so a warp's loads are contiguous); quality blocks
+// run the per-(query, model) chains from shared memory; the last block to
+// finish a query (per-query arrival counter, self-resetting) applies the
+// decision maker.  Same canonical order as the kernels above.
+
+struct PairArgs {
+    const float *W2T;   // [H1][H2]: W2 transposed
+    float *pairC;       // [Q][D] scratch
+    float *qualS;       // [Q][M] scratch
+    int32_t *count;     // [Q] arrivals, zero between calls
+    int qblocks;        // quality blocks per query
+};
+
+constexpr int PAIR_MPB = 8;  // models per quality block
+
+__device__ void pair_select(const Model &m, const Queries &q, const PairArgs &a, int qq) {
+    // warp 0 of the last block of query qq: utility, SLO mask, argmax
+    const int lane = threadIdx.x & 31;
+    Cand best = no_cand();
+    for (int d = lane; d < m.D; d += 32) {
+        const float C = __ldcg(&a.pairC[(size_t)qq * m.D + d]);
+        const float Ql = __ldcg(&a.qualS[(size_t)qq * m.M + m.dep_model[d]]);
+        const float U = __fmaf_rn(-q.lam, C, __fmul_rn(q.wq, Ql));
+        Cand c = make_cand(C, U, d, q.slo);
+        if (better(c, best)) best = c;
+    }
+    best = warp_best(best);
+    if (lane == 0) {
+        const bool ok = best.cls > 0;
+        q.chosen[qq] = ok ? best.d : -1;
+        q.lat[qq] = ok ? best.C : __int_as_float(0x7fc00000);
+        q.util[qq] = ok ? best.U : __int_as_float(0x7fc00000);
+        a.count[qq] = 0;
+    }
+}
+
+__global__ void __launch_bounds__(SIMT_THREADS) k_route_pairs(Model m, Queries q, PairArgs a) {
+    extern __shared__ float sm[];
+    __shared__ int s_last;
+    const int tid = threadIdx.x, F = m.F, H1 = m.H1, H2 = m.H2, D = m.D, M = m.M;
+    const int npair = q.Q * D;
+    int qq;
+    if ((int)blockIdx.x < npair) {
+        qq = blockIdx.x / D;
+        const int d = blockIdx.x - qq * D;
+        float *h1 = sm, *h2 = sm + MAX_H;
+        __shared__ float uv[3];
+        if (tid == 0) {
+            const float o = q.out_len[qq];
+            uv[0] = standardise(m.xform[F - 2], (double)q.in_len[qq], m.mu[F - 2], m.sd[F - 2]);
+            uv[1] = standardise(m.xform[F - 1], (double)o, m.mu[F - 1], m.sd[F - 1]);
+            uv[2] = o;
+        }
+        __syncthreads();
+        for (int k = tid; k < H1; k += SIMT_THREADS) {
+            const float *w = m.W1 + (size_t)k * F;
+            float x = m.A[(size_t)d * H1 + k];
+            x = __fmaf_rn(w[F - 2], uv[0], x);
+            x = __fmaf_rn(w[F - 1], uv[1], x);
+            h1[k] = x > 0.f ? x : 0.f;
+        }
+        __syncthreads();
+        float *w3s = sm + 2 * MAX_H;   // W3 [2][H2], staged for the head chains
+        for (int i = tid; i < 2 * H2; i += SIMT_THREADS) w3s[i] = m.W3[i];
+        for (int n = tid; n < H2; n += SIMT_THREADS) {
+            // serial chain over k (canonical order); W2 values fetched 32 at a
+            // time, the next block in flight while this one is accumulated
+            float acc = m.b2[n];
+            float w[32], wn[32];
+#pragma unroll
+            for (int j = 0; j < 32; ++j) w[j] = j < H1 ? a.W2T[(size_t)j * H2 + n] : 0.f;
+            for (int k0 = 0; k0 < H1; k0 += 32) {
+#pragma unroll
+                for (int j = 0; j < 32; ++j)
+                    wn[j] = k0 + 32 + j < H1 ? a.W2T[(size_t)(k0 + 32 + j) * H2 + n] : 0.f;
+#pragma unroll
+                for (int j = 0; j < 32; ++j)
+                    if (k0 + j < H1) acc = __fmaf_rn(w[j], h1[k0 + j], acc);
+#pragma unroll
+                for (int j = 0; j < 32; ++j) w[j] = wn[j];
+            }
+            h2[n] = acc > 0.f ? acc : 0.f;
+        }
+        __syncthreads();
+        if (tid < 64) {
+            // the two heads, one warp each
+            const int o = tid >> 5;
+            if ((tid & 31) == 0) {
+                const float *w3 = w3s + (size_t)o * H2;
+                float z = m.b3[o];
+                for (int n = 0; n < H2; ++n) z = __fmaf_rn(w3[n], h2[n], z);
+                uv[o] = softplus_c(z);   // query features no longer needed
+            }
+        }
+        __syncthreads();
+        if (tid == 0) a.pairC[(size_t)qq * D + d] = __fmaf_rn(uv[2], uv[1], uv[0]);
+    } else {
+        // quality of models [m0, m0 + PAIR_MPB) for one query
+        const int b = blockIdx.x - npair;
+        qq = b / a.qblocks;
+        const int m0 = (b - qq * a.qblocks) * PAIR_MPB, mn = min(PAIR_MPB, M - m0), E = m.E;
+        float *er = sm, *mb = sm + E;   // emb row [E], model columns [mn][E]
+        const size_t row = (size_t)qq * E;
+        for (int k = tid; k < E; k += SIMT_THREADS) {
+            er[k] = emb_at(q.emb, q.emb_bf16, row + k);
+            for (int j = 0; j < mn; ++j) mb[(size_t)j * E + k] = m.memb[(size_t)k * M + m0 + j];
+        }
+        __syncthreads();
+        if (tid < mn) {
+            const float *c = mb + (size_t)tid * E;
+            float s = 0.f;
+#pragma unroll 8
+            for (int k = 0; k < E; ++k) s = __fmaf_rn(er[k], c[k], s);
+            a.qualS[(size_t)qq * M + m0 + tid] = sigmoid_c(s);
+        }
+    }
+    // the last of the query's D + qblocks blocks applies the decision maker
+    __syncthreads();
+    if (tid == 0) {
+        __threadfence();
+        s_last = atomicAdd(&a.count[qq], 1) == D + a.qblocks - 1;
+    }
+    __syncthreads();
+    if (s_last && tid < 32) {
+        __threadfence();
+        pair_select(m, q, a, qq);
+    }
+}
+
+// ---------------------------------------------------------------------------
 // host launchers
 
 static int cpt_for(int H2) { return H2 <= 32 ? 1 : H2 <= 64 ? 2 : H2 <= 128 ? 4 : 8; }
@@ -498,6 +630,7 @@ cudaError_t simt_prepare() {
     if (e == cudaSuccess) e = opt_in(k_seq_table<4>, big);
     if (e == cudaSuccess) e = opt_in(k_seq_table<8>, big);
     if (e == cudaSuccess) e = opt_in(k_seq_chain, SEQ_CHAIN_SMEM + 1024);
+    if (e == cudaSuccess) e = opt_in(k_route_pairs, big);
     return e;
 }
 
@@ -517,6 +650,26 @@ cudaError_t launch_route_simt(const Model &m, const Queries &q, cudaStream_t s) 
         case 4: k_route_simt<4><<<blocks, SIMT_THREADS, smem, s>>>(m, q); break;
         default: k_route_simt<8><<<blocks, SIMT_THREADS, smem, s>>>(m, q); break;
     }
+    return cudaGetLastError();
+}
+
+size_t route_pairs_smem(const Model &m) {
+    const size_t pair = 4 * MAX_H * sizeof(float);
+    const size_t qual = (size_t)m.E * (1 + PAIR_MPB) * sizeof(float);
+    return pair > qual ? pair : qual;
+}
+
+cudaError_t launch_route_pairs(const Model &m, const Queries &q, const float *W2T, float *pairC,
+                               float *qualS, int32_t *count, cudaStream_t s) {
+    if (q.Q <= 0) return cudaSuccess;
+    PairArgs a;
+    a.W2T = W2T;
+    a.pairC = pairC;
+    a.qualS = qualS;
+    a.count = count;
+    a.qblocks = (m.M + PAIR_MPB - 1) / PAIR_MPB;
+    const int blocks = q.Q * (m.D + a.qblocks);
+    k_route_pairs<<<blocks, SIMT_THREADS, route_pairs_smem(m), s>>>(m, q, a);
     return cudaGetLastError();
 }
 
