@@ -88,6 +88,10 @@ def _declare(lib):
                               P, P, P, I]
     lib.orc_route.restype = I
     lib.orc_score_all.argtypes = [P, P, ct.c_int32, P, P, P, I, F, I, I, P, P, I]
+    lib.orc_route_q.argtypes = [P, P, ct.c_int32, P, P, P, I, P, F, I, I, I, P, P, P, P, I]
+    lib.orc_route_q.restype = I
+    lib.orc_slo_budget.argtypes = [F, F, F, F, F, F, I]
+    lib.orc_slo_budget.restype = D_
     lib.orc_score_all.restype = I
     lib.orc_features.argtypes = [P, P, I, F, F, I, P]
     lib.orc_predict.argtypes = [P, P, I, P, P]
@@ -187,6 +191,31 @@ class Problem:
             raise MemoryError("oracle allocation failed")
         return chosen, lat, util, run
 
+    def route_slo(self, slo_q, in_len=None, out_len=None, emb=None, *, lam=None,
+                  mode=F64, sequential=False, convex=False, running=None):
+        """Route with one SLO budget per query (float32 array of length Q)."""
+        p = self.p
+        il, ol, e, bf = self._queries(p["in_len"] if in_len is None else in_len,
+                                      p["out_len"] if out_len is None else out_len,
+                                      p["emb"] if emb is None else emb)
+        Q = il.size
+        sq = np.ascontiguousarray(slo_q, dtype=np.float32)
+        assert sq.size == Q
+        lam = p["lam"] if lam is None else lam
+        run = np.array(self._snap_arrays[0] if running is None else running,
+                       dtype=np.int32, copy=True)
+        chosen = np.empty(Q, np.int32)
+        lat = np.empty(Q, np.float64)
+        util = np.empty(Q, np.float64)
+        rc = self.lib.orc_route_q(ct.byref(self.model), ct.byref(self.snap), Q,
+                                  il.ctypes.data, ol.ctypes.data, e.ctypes.data, bf,
+                                  sq.ctypes.data, float(lam), int(convex), int(mode),
+                                  int(sequential), run.ctypes.data, chosen.ctypes.data,
+                                  lat.ctypes.data, util.ctypes.data, 1)
+        if rc != 0:
+            raise MemoryError("oracle allocation failed")
+        return chosen, lat, util, run
+
     def score_all(self, in_len=None, out_len=None, emb=None, *, lam=None,
                   mode=F64, convex=False, nthreads=1):
         """Latency and utility of every (query, deployment) pair, [Q][D]."""
@@ -229,6 +258,16 @@ class Problem:
         self.lib.orc_quality(ct.byref(self.model), e.ctypes.data, bf, 0,
                              int(mode), out.ctypes.data)
         return out
+
+
+def slo_budget(a, b, slack, tpot_slo, in_len, out_len, mode=F64, lib=None):
+    """Per-query SLO budgets of Eq. 4-5 (one value per query)."""
+    lib = lib or load()
+    il = np.asarray(in_len, np.float32).ravel()
+    ol = np.asarray(out_len, np.float32).ravel()
+    return np.array([lib.orc_slo_budget(float(a), float(b), float(slack), float(tpot_slo),
+                                        float(x), float(y), int(mode))
+                     for x, y in zip(il, ol)])
 
 
 def select(C, U, slo, mode=F64, lib=None):

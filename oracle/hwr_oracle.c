@@ -265,6 +265,23 @@ int orc_select(int D, const double *C, const double *U, double slo, int mode)
     return best;
 }
 
+/* ---- per-query latency budget (Sec. 4.3, Eq. 4-5) ---------------------- */
+
+/* SLO budget of a query with p input tokens and d expected output tokens:
+ * TTFT_SLO(p) = slack * (a + b p) and the request meets the SLO when its
+ * latency is at most TTFT_SLO(p) + d * TPOT_SLO.  fp32 order:
+ * t = fma(b, p, a); s = slack * t; B = fma(tpot_slo, d, s). */
+double orc_slo_budget(float a, float b, float slack, float tpot_slo, float p, float d,
+                      int mode)
+{
+    if (mode == ORC_F64)
+        return (double)slack * ((double)a + (double)b * (double)p) +
+               (double)d * (double)tpot_slo;
+    float t = fmaf(b, p, a);
+    float s = slack * t;
+    return (double)fmaf(tpot_slo, d, s);
+}
+
 /* ---- one query against every deployment ------------------------------- */
 
 typedef struct {
@@ -399,6 +416,34 @@ int orc_route(const orc_model *m, const orc_snapshot *s, int32_t Q,
     if (ws)
         for (int t = 0; t < nthreads; ++t) work_free(&ws[t]);
     free(ws); free(C); free(U); free(qual);
+    return fail ? -1 : 0;
+}
+
+/* As orc_route in batch or sequential mode, with one SLO budget per query
+ * (slo_q[Q], in the precision of the mode: float values). */
+int orc_route_q(const orc_model *m, const orc_snapshot *s, int32_t Q, const float *in_len,
+                const float *out_len, const void *emb, int emb_bf16, const float *slo_q,
+                float lam, int convex, int mode, int sequential, int32_t *running_io,
+                int32_t *chosen, double *lat, double *util, int nthreads)
+{
+    if (nthreads < 1) nthreads = 1;
+    orc_snapshot cur = *s;
+    if (sequential) cur.running = running_io;
+    int fail = 0;
+    orc_work w;
+    if (!work_alloc(m, &w)) {
+        work_free(&w);
+        return -1;
+    }
+    for (int32_t q = 0; q < Q; ++q) {
+        orc_quality(m, emb, emb_bf16, (size_t)q * m->E, mode, w.qual);
+        for (int d = 0; d < m->D; ++d)
+            score_pair(m, &cur, in_len[q], out_len[q], d, slo_q[q], lam, convex, mode, &w);
+        finish_query(m, &w, slo_q[q], mode, &chosen[q], &lat[q], &util[q]);
+        if (sequential && chosen[q] >= 0) running_io[chosen[q]] += 1;
+    }
+    (void)nthreads;
+    work_free(&w);
     return fail ? -1 : 0;
 }
 

@@ -481,6 +481,64 @@ def check_canonical_fp32_exact(lib):
     assert t == f32(z + math.log1p(math.exp(-z))), t
 
 
+# ---------------------------------------------------------------------------
+# per-query SLO budgets (Sec. 4.3, Eq. 4-5)
+
+def check_slo_budget(lib):
+    # TTFT_SLO(p) = slack (a + b p); budget = TTFT_SLO(p) + d TPOT_SLO
+    # (b = 2^-10 per token and TPOT_SLO = 2^-6 s are exact in float32)
+    got = O.slo_budget(0.5, 2.0 ** -10, 1.25, 2.0 ** -6, [1024.0, 0.0], [64.0, 32.0], O.F64, lib)
+    assert got[0] == 1.25 * (0.5 + 1.0) + 1.0, got
+    assert got[1] == 1.25 * 0.5 + 0.5, got
+    # fp32 order: t = fma(b, p, a); s = slack * t; B = fma(tpot, d, s)
+    # values for which computing b * p + a unfused changes the final budget
+    a, b, sl, tp = 0.4524623453617096, 0.000643032428342849, f32(1.2), f32(0.021)
+    p_, d_ = 31701.0, 110.3285903930664
+    assert fma_f32(tp, d_, mul_f32(sl, f32(f32(b * p_) + a))) != \
+        fma_f32(tp, d_, mul_f32(sl, fma_f32(b, p_, a)))
+    t = fma_f32(b, p_, a)
+    want = fma_f32(tp, d_, mul_f32(sl, t))
+    got = O.slo_budget(a, b, sl, tp, [p_], [d_], O.F32, lib)[0]
+    assert got == want, (got, want)
+
+
+def check_per_query_slo(lib):
+    p = tiny(M=2, G=3, Q=60, seed=12, F=16)
+    pr = O.Problem(p, lib=lib)
+    C, U = pr.score_all()
+    rng = np.random.default_rng(3)
+    budgets = np.quantile(C, rng.uniform(0.0, 1.0, p["Q"])).astype(np.float32)
+    budgets[:5] = np.inf
+    budgets[5:10] = 0.0
+    for mode in (O.F64, O.F32):
+        ch, lat, util, _ = pr.route_slo(budgets, mode=mode)
+        Cm, Um = pr.score_all(mode=mode)
+        for q in range(p["Q"]):
+            feas = Cm[q] <= budgets[q]
+            if feas.any():
+                assert feas[ch[q]] and Um[q, ch[q]] == Um[q][feas].max(), q
+            else:
+                assert Cm[q, ch[q]] == Cm[q].min(), q
+        # one budget per query: equal to routing that query alone with it
+        for q in (0, 7, 33):
+            c1, l1, u1, _ = pr.route(p["in_len"][q:q + 1], p["out_len"][q:q + 1],
+                                     p["emb"][q:q + 1], slo=float(budgets[q]), mode=mode)
+            assert c1[0] == ch[q] and l1[0] == lat[q]
+    # sequential with per-query budgets equals the query-by-query replay
+    ch_s, _, _, run_s = pr.route_slo(budgets, sequential=True)
+    run = p["snap"]["running"].copy()
+    for q in range(p["Q"]):
+        snap = dict(p["snap"])
+        snap["running"] = run
+        c, _, _, _ = O.Problem(p, snap=snap, lib=lib).route(
+            p["in_len"][q:q + 1], p["out_len"][q:q + 1], p["emb"][q:q + 1],
+            slo=float(budgets[q]))
+        assert c[0] == ch_s[q], q
+        run = run.copy()
+        run[c[0]] += 1
+    assert np.array_equal(run, run_s)
+
+
 ALL_CHECKS = [
     check_activations,
     check_closed_form_predictor,
@@ -496,4 +554,6 @@ ALL_CHECKS = [
     check_fp32_near_fp64,
     check_sequential,
     check_canonical_fp32_exact,
+    check_slo_budget,
+    check_per_query_slo,
 ]

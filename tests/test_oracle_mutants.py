@@ -66,6 +66,13 @@ MUTANTS = [
      "for (int k = m->F - 1; k >= 0; --k)\n            acc = fmaf(", 1),
     ("features_not_rounded_f32", "x[k] = mode == ORC_F32 ? (double)(float)v : v;",
      "x[k] = v;", 1),
+    ("budget_drops_slack", "return (double)slack * ((double)a + (double)b * (double)p) +",
+     "return ((double)a + (double)b * (double)p) +", 1),
+    ("budget_order_f32", "float t = fmaf(b, p, a);\n    float s = slack * t;",
+     "float t = b * p + a;\n    float s = slack * t;", 1),
+    ("per_query_slo_first_only", "finish_query(m, &w, slo_q[q], mode,", "finish_query(m, &w, slo_q[0], mode,", 1),
+    ("per_query_seq_no_increment", "if (sequential && chosen[q] >= 0) running_io[chosen[q]] += 1;",
+     "if (sequential && chosen[q] >= 0) running_io[chosen[q]] += 0;", 1),
 ]
 
 
