@@ -181,6 +181,35 @@ hwr_status hwr_route_batch(hwr_ctx *ctx, int32_t Q, const float *in_len,
                            float *pred_latency, float *utility);
 
 /*
+ * Per-query latency budgets (HW-Router Sec. 4.3, Eq. 4-5).  The paper's SLO
+ * for a request with p input tokens and d output tokens is
+ * TTFT_SLO(p) + d * TPOT_SLO with TTFT_SLO(p) = slack * (a + b p); routing
+ * uses the query's expected output length for d.
+ *   budget   [Q] budget per query in seconds (host or device memory, as the
+ *            other arrays of the call), or NULL to use the model below;
+ *   ttft_a, ttft_b, slack, tpot   the model (finite) when budget is NULL;
+ *            evaluated per query on the device in fp32 as
+ *            t = fma(b, p, a); s = slack * t; B = fma(tpot, d, s).
+ * A NaN budget makes every deployment of that query infeasible.
+ */
+typedef struct {
+    const float *budget;
+    float ttft_a, ttft_b, slack, tpot;
+} hwr_slo_spec;
+
+/*
+ * As hwr_route_batch, with the SLO budget B of Eq. 3 given per query by
+ * `slo` instead of one scalar for the batch (all flags and paths apply).
+ * Errors: as hwr_route_batch; INVALID_ARG also for a NULL spec or
+ * non-finite model parameters.
+ */
+hwr_status hwr_route_batch_slo(hwr_ctx *ctx, int32_t Q, const float *in_len,
+                               const float *out_len, const void *q_emb,
+                               const hwr_slo_spec *slo, float lambda,
+                               uint32_t flags, int32_t *chosen,
+                               float *pred_latency, float *utility);
+
+/*
  * Route a batch without allocating anything at call time.
  *
  * The paper has no counterpart to this call; it exists for callers that

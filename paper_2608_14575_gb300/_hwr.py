@@ -34,7 +34,7 @@ KERNELS = ("snapshot", "route_simt", "seq_table", "qual_tc", "mlp_tc")
 HWR_K_COUNT = len(KERNELS)
 
 EXPORTS = ("hwr_create", "hwr_update_snapshot", "hwr_get_snapshot",
-           "hwr_route_batch", "hwr_route_batch_noalloc", "hwr_synchronize",
+           "hwr_route_batch", "hwr_route_batch_slo", "hwr_route_batch_noalloc", "hwr_synchronize",
            "hwr_destroy", "hwr_status_string", "hwr_last_error", "hwr_get_stats")
 HWR_NOALLOC_MAX_Q = 32768
 
@@ -56,6 +56,11 @@ class hwr_predictor(ct.Structure):
 class hwr_snapshot(ct.Structure):
     _fields_ = [(n, ct.c_void_p) for n in
                 ("running", "waiting", "kv_util", "gpu_util", "ttft_avg", "tpot_avg")]
+
+
+class hwr_slo_spec(ct.Structure):
+    _fields_ = [("budget", ct.c_void_p), ("ttft_a", ct.c_float), ("ttft_b", ct.c_float),
+                ("slack", ct.c_float), ("tpot", ct.c_float)]
 
 
 class hwr_stats(ct.Structure):
@@ -97,6 +102,8 @@ def load(path: str | None = None):
         lib.hwr_route_batch.argtypes = [P, ct.c_int32, P, P, P, ct.c_float,
                                         ct.c_float, ct.c_uint32, P, P, P]
         lib.hwr_route_batch_noalloc.argtypes = lib.hwr_route_batch.argtypes
+        lib.hwr_route_batch_slo.argtypes = [P, ct.c_int32, P, P, P, P, ct.c_float,
+                                            ct.c_uint32, P, P, P]
         lib.hwr_synchronize.argtypes = [P]
         lib.hwr_destroy.argtypes = [P]
         lib.hwr_status_string.argtypes = [I]
@@ -105,8 +112,8 @@ def load(path: str | None = None):
         lib.hwr_last_error.restype = ct.c_char_p
         lib.hwr_get_stats.argtypes = [P, P, I]
         for n in ("hwr_create", "hwr_update_snapshot", "hwr_get_snapshot",
-                  "hwr_route_batch", "hwr_route_batch_noalloc", "hwr_synchronize",
-                  "hwr_destroy", "hwr_get_stats"):
+                  "hwr_route_batch", "hwr_route_batch_slo", "hwr_route_batch_noalloc",
+                  "hwr_synchronize", "hwr_destroy", "hwr_get_stats"):
             getattr(lib, n).restype = I
         if path is None:
             _lib = lib
@@ -131,6 +138,12 @@ def hwr_route_batch(ctx, Q, in_len, out_len, q_emb, slo, lam, flags, chosen,
                     pred_latency, utility):
     return load().hwr_route_batch(ctx, Q, in_len, out_len, q_emb, slo, lam, flags,
                                   chosen, pred_latency, utility)
+
+
+def hwr_route_batch_slo(ctx, Q, in_len, out_len, q_emb, slo, lam, flags, chosen,
+                        pred_latency, utility):
+    return load().hwr_route_batch_slo(ctx, Q, in_len, out_len, q_emb, slo, lam, flags,
+                                      chosen, pred_latency, utility)
 
 
 def hwr_route_batch_noalloc(ctx, Q, in_len, out_len, q_emb, slo, lam, flags, chosen,
@@ -237,6 +250,44 @@ class Router:
             float(p["lam"] if lam is None else lam), int(flags) & ~HWR_DEVICE_PTRS,
             chosen.ctypes.data, lat.ctypes.data, util.ctypes.data))
         return chosen, lat, util
+
+    def route_slo(self, in_len=None, out_len=None, emb=None, *, budgets=None,
+                  model=None, lam=None, flags=0):
+        """Host routing with per-query budgets (array) or the Eq. 4-5 model
+        (a, b, slack, tpot)."""
+        p = self.p
+        il = _c(p["in_len"] if in_len is None else in_len, np.float32)
+        ol = _c(p["out_len"] if out_len is None else out_len, np.float32)
+        em = _c(p["emb"] if emb is None else emb, self.wdt)
+        Q = il.size
+        spec, keep = self._spec(budgets, model, Q)
+        chosen = np.empty(Q, np.int32)
+        lat = np.empty(Q, np.float32)
+        util = np.empty(Q, np.float32)
+        self._check(self.lib.hwr_route_batch_slo(
+            self.ctx, Q, il.ctypes.data, ol.ctypes.data, em.ctypes.data, ct.byref(spec),
+            float(p["lam"] if lam is None else lam), int(flags) & ~HWR_DEVICE_PTRS,
+            chosen.ctypes.data, lat.ctypes.data, util.ctypes.data))
+        return chosen, lat, util
+
+    def route_device_slo(self, in_len, out_len, emb, chosen, lat, util, *, budgets=None,
+                         model=None, lam, flags=0):
+        """Device routing with per-query budgets (CUDA tensor) or the model."""
+        spec = hwr_slo_spec(budgets.data_ptr() if budgets is not None else None,
+                            *(model if model is not None else (0.0, 0.0, 1.0, 0.0)))
+        self._check(self.lib.hwr_route_batch_slo(
+            self.ctx, int(in_len.numel()), in_len.data_ptr(), out_len.data_ptr(),
+            emb.data_ptr(), ct.byref(spec), float(lam), int(flags) | HWR_DEVICE_PTRS,
+            chosen.data_ptr(), lat.data_ptr(), util.data_ptr()))
+
+    @staticmethod
+    def _spec(budgets, model, Q):
+        if budgets is not None:
+            b = _c(budgets, np.float32)
+            assert b.size == Q
+            return hwr_slo_spec(b.ctypes.data, 0.0, 0.0, 1.0, 0.0), b
+        a, bb, slack, tpot = model
+        return hwr_slo_spec(None, float(a), float(bb), float(slack), float(tpot)), None
 
     def route_host_ptrs(self, Q, in_len_ptr, out_len_ptr, emb_ptr, chosen_ptr,
                         lat_ptr, util_ptr, *, slo, lam, flags=0):

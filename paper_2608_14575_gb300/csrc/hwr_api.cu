@@ -607,6 +607,7 @@ static hwr_status run_kernels(hwr_ctx *c, const Queries &q, uint32_t flags, bool
             k.chosen = q.chosen + lo;
             k.lat = q.lat + lo;
             k.util = q.util + lo;
+            if (q.slo_q) k.slo_q = q.slo_q + lo;
             LaunchScope a(c, HWR_K_SEQ_TABLE, prof);
             CK(c, launch_seq_table(m, k, n, c->ctab, c->qseq, c->stream), "sequential table");
             a.done();
@@ -648,10 +649,12 @@ static hwr_status run_kernels(hwr_ctx *c, const Queries &q, uint32_t flags, bool
 
 static size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
-extern "C" hwr_status hwr_route_batch(hwr_ctx *c, int32_t Q, const float *in_len,
-                                      const float *out_len, const void *q_emb, float slo,
-                                      float lambda, uint32_t flags, int32_t *chosen,
-                                      float *pred_latency, float *utility) {
+// Shared body of hwr_route_batch and hwr_route_batch_slo.  `spec` (may be
+// NULL) replaces the scalar SLO by per-query budgets or the Eq. 4-5 model.
+static hwr_status route_impl(hwr_ctx *c, int32_t Q, const float *in_len, const float *out_len,
+                             const void *q_emb, float slo, const hwr_slo_spec *spec,
+                             float lambda, uint32_t flags, int32_t *chosen,
+                             float *pred_latency, float *utility) {
     if (!c) return fail(nullptr, HWR_ERR_INVALID_ARG, "ctx is NULL");
     if (c->broken) return HWR_ERR_STATE;
     const uint32_t known = HWR_SEQUENTIAL | HWR_DEVICE_PTRS | HWR_ASYNC | HWR_SCORE_CONVEX |
@@ -661,7 +664,11 @@ extern "C" hwr_status hwr_route_batch(hwr_ctx *c, int32_t Q, const float *in_len
     if (Q == 0) return HWR_OK;
     if (!in_len || !out_len || !q_emb || !chosen || !pred_latency || !utility)
         return fail(c, HWR_ERR_INVALID_ARG, "NULL input or output array");
-    if (slo != slo) return fail(c, HWR_ERR_INVALID_ARG, "SLO is NaN");
+    if (!spec && slo != slo) return fail(c, HWR_ERR_INVALID_ARG, "SLO is NaN");
+    if (spec && !spec->budget &&
+        !(isfinite(spec->ttft_a) && isfinite(spec->ttft_b) && isfinite(spec->slack) &&
+          isfinite(spec->tpot)))
+        return fail(c, HWR_ERR_INVALID_ARG, "SLO model parameters must be finite");
     if (!isfinite(lambda)) return fail(c, HWR_ERR_INVALID_ARG, "lambda is not finite");
     if ((flags & HWR_PATH_SIMT) && (flags & HWR_PATH_TENSOR))
         return fail(c, HWR_ERR_INVALID_ARG, "HWR_PATH_SIMT and HWR_PATH_TENSOR together");
@@ -686,10 +693,19 @@ extern "C" hwr_status hwr_route_batch(hwr_ctx *c, int32_t Q, const float *in_len
     q.slo = slo;
     q.lam = lambda;
     q.wq = (flags & HWR_SCORE_CONVEX) ? 1.0f - lambda : 1.0f;
+    const bool budgets = spec && spec->budget;
+    if (spec) {
+        q.slo_mode = budgets ? 1 : 2;
+        q.slo_a = spec->ttft_a;
+        q.slo_b = spec->ttft_b;
+        q.slo_slack = spec->slack;
+        q.slo_tpot = spec->tpot;
+    }
 
     const size_t emb_b = (size_t)Q * c->E * es, len_b = (size_t)Q * 4;
     const size_t off_in = align_up(emb_b, 256), off_out = off_in + align_up(len_b, 256);
-    const size_t in_total = off_out + len_b;
+    const size_t off_slo = off_out + align_up(len_b, 256);
+    const size_t in_total = (budgets ? off_slo : off_out) + len_b;
     const size_t o_lat = align_up(len_b, 256), o_util = o_lat + align_up(len_b, 256);
     const size_t out_total = o_util + len_b;
     const bool packed = !dev && !(flags & HWR_ASYNC) && in_total <= ((size_t)1 << 20);
@@ -702,6 +718,7 @@ extern "C" hwr_status hwr_route_batch(hwr_ctx *c, int32_t Q, const float *in_len
     if (dev) {
         q.in_len = in_len; q.out_len = out_len; q.emb = q_emb;
         q.chosen = chosen; q.lat = pred_latency; q.util = utility;
+        if (budgets) q.slo_q = spec->budget;
     } else {
         TRY(grow(c, &c->io_d, &c->io_cap, in_total));
         TRY(grow(c, &c->out_d, &c->out_cap, out_total));
@@ -711,6 +728,7 @@ extern "C" hwr_status hwr_route_batch(hwr_ctx *c, int32_t Q, const float *in_len
             memcpy(c->pin_h, q_emb, emb_b);
             memcpy(c->pin_h + off_in, in_len, len_b);
             memcpy(c->pin_h + off_out, out_len, len_b);
+            if (budgets) memcpy(c->pin_h + off_slo, spec->budget, len_b);
             CK(c, cudaMemcpyAsync(c->io_d, c->pin_h, in_total, cudaMemcpyHostToDevice, c->stream),
                "copy inputs");
         } else if (!pipelined) {
@@ -719,8 +737,12 @@ extern "C" hwr_status hwr_route_batch(hwr_ctx *c, int32_t Q, const float *in_len
                "copy in_len");
             CK(c, cudaMemcpyAsync(c->io_d + off_out, out_len, len_b, cudaMemcpyHostToDevice, c->stream),
                "copy out_len");
+            if (budgets)
+                CK(c, cudaMemcpyAsync(c->io_d + off_slo, spec->budget, len_b, cudaMemcpyHostToDevice,
+                                      c->stream), "copy budgets");
         }
         q.emb = c->io_d;
+        if (budgets) q.slo_q = (const float *)(c->io_d + off_slo);
         q.in_len = (const float *)(c->io_d + off_in);
         q.out_len = (const float *)(c->io_d + off_out);
         q.chosen = (int32_t *)c->out_d;
@@ -744,6 +766,10 @@ extern "C" hwr_status hwr_route_batch(hwr_ctx *c, int32_t Q, const float *in_len
                                   cudaMemcpyHostToDevice, c->copy_stream), "copy in_len");
             CK(c, cudaMemcpyAsync(c->io_d + off_out + (size_t)lo * 4, out_len + lo, (size_t)n * 4,
                                   cudaMemcpyHostToDevice, c->copy_stream), "copy out_len");
+            if (budgets)
+                CK(c, cudaMemcpyAsync(c->io_d + off_slo + (size_t)lo * 4, spec->budget + lo,
+                                      (size_t)n * 4, cudaMemcpyHostToDevice, c->copy_stream),
+                   "copy budgets");
             CK(c, cudaEventRecord(c->chunk_ev[k], c->copy_stream), "record");
             CK(c, cudaStreamWaitEvent(c->stream, c->chunk_ev[k], 0), "order kernels");
             Queries qc = q;
@@ -754,6 +780,7 @@ extern "C" hwr_status hwr_route_batch(hwr_ctx *c, int32_t Q, const float *in_len
             qc.chosen = q.chosen + lo;
             qc.lat = q.lat + lo;
             qc.util = q.util + lo;
+            if (q.slo_q) qc.slo_q = q.slo_q + lo;
             TRY(run_kernels(c, qc, flags, tensor));
         }
     } else {
@@ -785,6 +812,24 @@ extern "C" hwr_status hwr_route_batch(hwr_ctx *c, int32_t Q, const float *in_len
     CK(c, cudaGetLastError(), "kernel");
     if (tensor) TRY(check_status_word(c));
     return HWR_OK;
+}
+
+extern "C" hwr_status hwr_route_batch(hwr_ctx *c, int32_t Q, const float *in_len,
+                                      const float *out_len, const void *q_emb, float slo,
+                                      float lambda, uint32_t flags, int32_t *chosen,
+                                      float *pred_latency, float *utility) {
+    return route_impl(c, Q, in_len, out_len, q_emb, slo, nullptr, lambda, flags, chosen,
+                      pred_latency, utility);
+}
+
+extern "C" hwr_status hwr_route_batch_slo(hwr_ctx *c, int32_t Q, const float *in_len,
+                                          const float *out_len, const void *q_emb,
+                                          const hwr_slo_spec *slo, float lambda, uint32_t flags,
+                                          int32_t *chosen, float *pred_latency, float *utility) {
+    if (!c) return fail(nullptr, HWR_ERR_INVALID_ARG, "ctx is NULL");
+    if (!slo) return fail(c, HWR_ERR_INVALID_ARG, "slo specification is NULL");
+    return route_impl(c, Q, in_len, out_len, q_emb, 0.0f, slo, lambda, flags, chosen,
+                      pred_latency, utility);
 }
 
 extern "C" hwr_status hwr_synchronize(hwr_ctx *c) {

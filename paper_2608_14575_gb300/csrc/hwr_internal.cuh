@@ -53,7 +53,25 @@ struct Queries {
     float slo, lam, wq;         // wq = 1 or (1 - lambda)
     int32_t *chosen;
     float *lat, *util;
+    // latency budget per query: 0 = the scalar slo, 1 = slo_q[q],
+    // 2 = the SLO model of Eq. 4-5 from the query's lengths
+    int slo_mode = 0;
+    const float *slo_q = nullptr;
+    float slo_a = 0.f, slo_b = 0.f, slo_slack = 1.f, slo_tpot = 0.f;
 };
+
+#ifdef __CUDACC__
+// Budget B of query `row` (Sec. 4.3, Eq. 4-5 for the model form):
+// t = fma(b, p, a); s = slack * t; B = fma(tpot_slo, d, s).
+__device__ __forceinline__ float query_budget(const Queries &q, int row) {
+    if (q.slo_mode == 1) return q.slo_q[row];
+    if (q.slo_mode == 2) {
+        const float t = __fmaf_rn(q.slo_b, q.in_len[row], q.slo_a);
+        return __fmaf_rn(q.slo_tpot, q.out_len[row], __fmul_rn(q.slo_slack, t));
+    }
+    return q.slo;
+}
+#endif
 
 // ---- SIMT kernels (k_simt.cu) -------------------------------------------
 cudaError_t launch_snapshot(const Model &m, cudaStream_t s);

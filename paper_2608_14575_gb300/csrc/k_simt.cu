@@ -279,8 +279,9 @@ __global__ void __launch_bounds__(SIMT_THREADS) k_route_simt(Model m, Queries q)
         const int qq = q0 + qi;
         if (qq >= q.Q) continue;
         Cand best = no_cand();
+        const float slo = query_budget(q, qq);
         for (int d = lane; d < D; d += 32) {
-            Cand c = make_cand(Cs[qi * D + d], Us[qi * D + d], d, q.slo);
+            Cand c = make_cand(Cs[qi * D + d], Us[qi * D + d], d, slo);
             if (better(c, best)) best = c;
         }
         best = warp_best(best);
@@ -414,6 +415,7 @@ k_seq_chain(Model m, Queries q, int Qs, const float *ctab, const float *qualS) {
         int cA = 0, cB = 0;  // picks so far of deployments lane and lane + 32
         for (int i = 0; i < Qs; ++i) {
             Cand best = no_cand();
+            const float slo = query_budget(q, i);
 #pragma unroll
             for (int t = 0; t < 2; ++t) {
                 const int d = lane + 32 * t;
@@ -421,7 +423,7 @@ k_seq_chain(Model m, Queries q, int Qs, const float *ctab, const float *qualS) {
                     const int c = t ? cB : cA;
                     const float C = tab[tri_off(D, Qs, c) + (size_t)d * (Qs - c) + (i - c)];
                     const float U = __fmaf_rn(-q.lam, C, __fmul_rn(q.wq, qs[i * M + dm[d]]));
-                    Cand cd = make_cand(C, U, d, q.slo);
+                    Cand cd = make_cand(C, U, d, slo);
                     if (better(cd, best)) best = cd;
                 }
             }
@@ -480,11 +482,12 @@ __device__ void pair_select(const Model &m, const Queries &q, const PairArgs &a,
     // warp 0 of the last block of query qq: utility, SLO mask, argmax
     const int lane = threadIdx.x & 31;
     Cand best = no_cand();
+    const float slo = query_budget(q, qq);
     for (int d = lane; d < m.D; d += 32) {
         const float C = __ldcg(&a.pairC[(size_t)qq * m.D + d]);
         const float Ql = __ldcg(&a.qualS[(size_t)qq * m.M + m.dep_model[d]]);
         const float U = __fmaf_rn(-q.lam, C, __fmul_rn(q.wq, Ql));
-        Cand c = make_cand(C, U, d, q.slo);
+        Cand c = make_cand(C, U, d, slo);
         if (better(c, best)) best = c;
     }
     best = warp_best(best);

@@ -459,6 +459,7 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
             const int row = un.tile * BM + r;
             const bool valid = row < q.Q;
             const float ol = valid ? q.out_len[row] : 0.f;
+            const float slo_r = valid ? query_budget(q, row) : slo;
             for (int i = 0; i < m.M; ++i)
                 qs[r * QS + i] = valid ? qual[(size_t)row * Mpad + i] : 0.f;
             Cand best = no_cand();
@@ -516,7 +517,7 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
                 const float ttft = softplus_fast(z0), tpot = softplus_fast(z1);
                 const float C = fmaf(ol, tpot, ttft);
                 const float U = fmaf(-lam, C, wq * qs[r * QS + dms[d]]);
-                const Cand cd = make_cand(C, U, d, slo);
+                const Cand cd = make_cand(C, U, d, slo_r);
                 if (better(cd, best)) best = cd;
             }
             if (!ok || !valid) continue;
