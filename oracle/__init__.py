@@ -69,7 +69,7 @@ def load(path: str | None = None, rebuild: bool = False):
 
 
 class _Model(ct.Structure):
-    _fields_ = [(n, ct.c_int32) for n in ("M", "G", "D", "F", "H1", "H2", "E")] + [
+    _fields_ = [(n, ct.c_int32) for n in ("M", "G", "D", "F", "H1", "H2", "E", "n_heads")] + [
         ("dep_model", ct.c_void_p), ("dep_gpu", ct.c_void_p),
         ("log10p", ct.c_void_p), ("W1", ct.c_void_p), ("b1", ct.c_void_p),
         ("W2", ct.c_void_p), ("b2", ct.c_void_p), ("W3", ct.c_void_p),
@@ -94,7 +94,7 @@ def _declare(lib):
     lib.orc_slo_budget.restype = D_
     lib.orc_score_all.restype = I
     lib.orc_features.argtypes = [P, P, I, F, F, I, P]
-    lib.orc_predict.argtypes = [P, P, I, P, P]
+    lib.orc_predict.argtypes = [P, P, I, P, P, P]
     lib.orc_quality.argtypes = [P, P, I, ct.c_size_t, I, P]
     lib.orc_select.argtypes = [I, P, P, D_, I]
     lib.orc_select.restype = I
@@ -130,6 +130,7 @@ class Problem:
         m = _Model()
         for n in ("M", "G", "D", "F", "H1", "H2", "E"):
             setattr(m, n, int(p[n]))
+        m.n_heads = int(p.get("n_heads", 2))
         m.dep_model = arr(p["dep_model"], np.int32)
         m.dep_gpu = arr(p["dep_gpu"], np.int32)
         m.log10p = arr(p["log10p"], np.float32)
@@ -243,12 +244,13 @@ class Problem:
                               x.ctypes.data)
         return x
 
-    def predict(self, x, mode=F64):
+    def predict(self, x, mode=F64, heads=False):
+        """(TTFT, TPOT), or (TTFT, TPOT, N_out) with heads=True."""
         x = np.ascontiguousarray(x, dtype=np.float64)
-        a, b = ct.c_double(), ct.c_double()
+        a, b, c = ct.c_double(), ct.c_double(), ct.c_double()
         self.lib.orc_predict(ct.byref(self.model), x.ctypes.data, int(mode),
-                             ct.byref(a), ct.byref(b))
-        return a.value, b.value
+                             ct.byref(a), ct.byref(b), ct.byref(c))
+        return (a.value, b.value, c.value) if heads else (a.value, b.value)
 
     def quality(self, emb_row, mode=F64):
         e = np.asarray(emb_row)

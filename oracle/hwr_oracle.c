@@ -14,7 +14,10 @@
  *     h1     = relu(W1 x + b1), h2 = relu(W2 h1 + b2), z = W3 h2 + b3
  *              (two fully connected hidden layers with ReLU, Eq. 1)
  *     TTFT   = softplus(z0), TPOT = softplus(z1)
+ *              (with three heads also N_out = softplus(z2), Eq. 1)
  *     C      = TTFT + N_out * TPOT                      (Eq. 2)
+ *              N_out: the third head, or with two heads the query's given
+ *              expected output length
  *     Qual   = sigmoid(emb_q . memb[:, model(d)])        (Sec. 3.2 "Quality
  *              Predictor": depends on the model only, not on the GPU)
  *     U      = w * Qual - lambda * C, w = 1 or (1 - lambda)   (Sec. 3.1, Eq. 3)
@@ -55,11 +58,12 @@
 
 typedef struct {
     int32_t M, G, D, F, H1, H2, E;
+    int32_t n_heads;                    /* 2: TTFT, TPOT; 3: + N_out (Eq. 1) */
     const int32_t *dep_model, *dep_gpu; /* [D] */
     const float *log10p;                /* [M] */
     const float *W1, *b1;               /* [H1][F], [H1] */
     const float *W2, *b2;               /* [H2][H1], [H2] */
-    const float *W3, *b3;               /* [2][H2], [2] */
+    const float *W3, *b3;               /* [n_heads][H2], [n_heads] */
     const float *mu, *sd;               /* [F] */
     const uint8_t *xform;               /* [F]: 0 identity, 1 log1p, 2 log */
     const float *memb;                  /* [E][M] */
@@ -139,7 +143,7 @@ void orc_features(const orc_model *m, const orc_snapshot *s, int d,
 /* ---- predictor (Eq. 1) ------------------------------------------------- */
 
 static void predict_f64(const orc_model *m, const double *x, double *ttft,
-                        double *tpot, double *h1, double *h2)
+                        double *tpot, double *nout, double *h1, double *h2)
 {
     for (int j = 0; j < m->H1; ++j) {
         double acc = m->b1[j];
@@ -153,8 +157,8 @@ static void predict_f64(const orc_model *m, const double *x, double *ttft,
             acc += (double)m->W2[(size_t)i * m->H1 + j] * h1[j];
         h2[i] = acc > 0.0 ? acc : 0.0;
     }
-    double z[2];
-    for (int o = 0; o < 2; ++o) {
+    double z[3] = {0.0, 0.0, 0.0};
+    for (int o = 0; o < m->n_heads; ++o) {
         double acc = m->b3[o];
         for (int i = 0; i < m->H2; ++i)
             acc += (double)m->W3[(size_t)o * m->H2 + i] * h2[i];
@@ -162,10 +166,11 @@ static void predict_f64(const orc_model *m, const double *x, double *ttft,
     }
     *ttft = orc_softplus_f64(z[0]);
     *tpot = orc_softplus_f64(z[1]);
+    *nout = m->n_heads == 3 ? orc_softplus_f64(z[2]) : 0.0;
 }
 
 static void predict_f32(const orc_model *m, const float *x, float *ttft,
-                        float *tpot, float *h1, float *h2)
+                        float *tpot, float *nout, float *h1, float *h2)
 {
     for (int j = 0; j < m->H1; ++j) {
         float acc = m->b1[j];
@@ -179,8 +184,8 @@ static void predict_f32(const orc_model *m, const float *x, float *ttft,
             acc = fmaf(m->W2[(size_t)i * m->H1 + j], h1[j], acc);
         h2[i] = acc > 0.0f ? acc : 0.0f;
     }
-    float z[2];
-    for (int o = 0; o < 2; ++o) {
+    float z[3] = {0.0f, 0.0f, 0.0f};
+    for (int o = 0; o < m->n_heads; ++o) {
         float acc = m->b3[o];
         for (int i = 0; i < m->H2; ++i)
             acc = fmaf(m->W3[(size_t)o * m->H2 + i], h2[i], acc);
@@ -188,23 +193,25 @@ static void predict_f32(const orc_model *m, const float *x, float *ttft,
     }
     *ttft = orc_softplus_f32(z[0]);
     *tpot = orc_softplus_f32(z[1]);
+    *nout = m->n_heads == 3 ? orc_softplus_f32(z[2]) : 0.0f;
 }
 
 /* Single-evaluation entry point (used by the pins): x has F doubles (in fp32
- * mode they are taken as floats). */
+ * mode they are taken as floats).  nout is the third head (0 with two). */
 void orc_predict(const orc_model *m, const double *x, int mode, double *ttft,
-                 double *tpot)
+                 double *tpot, double *nout)
 {
     double *h = (double *)malloc(sizeof(double) * (size_t)(m->H1 + m->H2));
     if (mode == ORC_F64) {
-        predict_f64(m, x, ttft, tpot, h, h + m->H1);
+        predict_f64(m, x, ttft, tpot, nout, h, h + m->H1);
     } else {
         float *xf = (float *)malloc(sizeof(float) * (size_t)(m->F + m->H1 + m->H2));
-        float a, b;
+        float a, b, c;
         for (int k = 0; k < m->F; ++k) xf[k] = (float)x[k];
-        predict_f32(m, xf, &a, &b, xf + m->F, xf + m->F + m->H1);
+        predict_f32(m, xf, &a, &b, &c, xf + m->F, xf + m->F + m->H1);
         *ttft = a;
         *tpot = b;
+        *nout = c;
         free(xf);
     }
     free(h);
@@ -317,17 +324,20 @@ static void score_pair(const orc_model *m, const orc_snapshot *s, float in_len,
     orc_features(m, s, d, in_len, out_len, mode, w->x);
     double qual = w->qual[m->dep_model[d]];
     if (mode == ORC_F64) {
-        double ttft, tpot;
-        predict_f64(m, w->x, &ttft, &tpot, w->h, w->h + m->H1);
-        double C = ttft + (double)out_len * tpot;
+        double ttft, tpot, nout;
+        predict_f64(m, w->x, &ttft, &tpot, &nout, w->h, w->h + m->H1);
+        /* N_out of Eq. 2: the third head's prediction, else the given length */
+        double n = m->n_heads == 3 ? nout : (double)out_len;
+        double C = ttft + n * tpot;
         double wq = convex ? 1.0 - (double)lam : 1.0;
         w->C[d] = C;
         w->U[d] = wq * qual - (double)lam * C;
     } else {
-        float ttft, tpot;
+        float ttft, tpot, nout;
         for (int k = 0; k < m->F; ++k) w->xf[k] = (float)w->x[k];
-        predict_f32(m, w->xf, &ttft, &tpot, w->hf, w->hf + m->H1);
-        float C = fmaf(out_len, tpot, ttft);
+        predict_f32(m, w->xf, &ttft, &tpot, &nout, w->hf, w->hf + m->H1);
+        float n = m->n_heads == 3 ? nout : out_len;
+        float C = fmaf(n, tpot, ttft);
         float wq = convex ? 1.0f - lam : 1.0f;
         w->C[d] = C;
         w->U[d] = fmaf(-lam, C, wq * (float)qual);

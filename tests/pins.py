@@ -84,10 +84,11 @@ def tiny(M=2, G=2, F=16, H1=4, H2=4, E=8, Q=4, dtype="f32", seed=11,
                           weight_std=weight_std)
 
 
-def blank(M=2, G=2, F=16, H1=4, H2=4, E=8, Q=1):
+def blank(M=2, G=2, F=16, H1=4, H2=4, E=8, Q=1, n_heads=2):
     """A problem with zero weights, zero biases, identity transforms and
     (mu, sd) = (0, 1) on every slot, for hand-set closed-form cases."""
-    p = tiny(M=M, G=G, F=F, H1=H1, H2=H2, E=E, Q=Q)
+    p = W.make_problem(Q=Q, M=M, G=G, F=F, H1=H1, H2=H2, E=E, dtype="f32", lam=0.5,
+                       slo=5.0, seed=11, n_heads=n_heads)
     for n in ("W1", "W2", "W3"):
         p[n] = np.zeros_like(p[n])
     for n in ("b1", "b2", "b3"):
@@ -482,6 +483,43 @@ def check_canonical_fp32_exact(lib):
 
 
 # ---------------------------------------------------------------------------
+# third output head N_out (Eq. 1) entering the cost (Eq. 2)
+
+def check_three_heads(lib):
+    p = blank(n_heads=3)
+    lay = W.feature_layout(p["M"], p["G"], p["F"])
+    k = lay["running"]
+    p["W1"][0, k] = 1.0
+    p["xform"][k] = 1                      # log1p
+    p["snap"]["running"][:] = 3            # x = ln 4
+    p["W2"][0, 0] = 1.0
+    p["W3"][:, 0] = [1.0, -1.0, 1.0]       # TTFT = log 5, TPOT = log 1.25, N_out = log 5
+    for mode, tol in ((O.F64, 1e-12), (O.F32, 2e-6)):
+        for out_len in (7.0, 700.0):       # the given length must not enter Eq. 2
+            p["out_len"][:] = out_len
+            pr = O.Problem(p, lib=lib)
+            x = pr.features(0, p["in_len"][0], p["out_len"][0], mode)
+            t, tp, n = pr.predict(x, mode, heads=True)
+            assert abs(n - math.log(5.0)) <= tol * math.log(5.0), n
+            C, _ = pr.score_all(lam=0.0, mode=mode)
+            want = math.log(5.0) + math.log(5.0) * math.log(1.25)
+            assert np.all(np.abs(C - want) <= tol * want), (C, want)
+    # with a constant third head equal to every query's length, three heads
+    # reduce to two
+    q2 = tiny(Q=10, seed=6)
+    q3 = tiny(Q=10, seed=6)
+    q3["n_heads"] = 3
+    q3["W3"] = np.concatenate([q2["W3"], np.zeros((1, q2["H2"]), np.float32)])
+    n = 150.0
+    q3["b3"] = np.concatenate([q2["b3"], [np.float32(math.log(math.expm1(n)))]])
+    q2["out_len"][:] = n
+    q3["out_len"][:] = n
+    C2, U2 = O.Problem(q2, lib=lib).score_all()
+    C3, U3 = O.Problem(q3, lib=lib).score_all()
+    assert np.allclose(C3, C2, rtol=1e-5), (C2, C3)
+
+
+# ---------------------------------------------------------------------------
 # per-query SLO budgets (Sec. 4.3, Eq. 4-5)
 
 def check_slo_budget(lib):
@@ -556,4 +594,5 @@ ALL_CHECKS = [
     check_canonical_fp32_exact,
     check_slo_budget,
     check_per_query_slo,
+    check_three_heads,
 ]

@@ -31,12 +31,10 @@ MUTANTS = [
     ("softplus_drops_max", "return fmax(z, 0.0) + log1p(exp(-fabs(z)));",
      "return log1p(exp(-fabs(z)));", 1),
     ("sigmoid_sign", "return 1.0 / (1.0 + exp(-s));", "return 1.0 / (1.0 + exp(s));", 1),
-    ("cost_sign", "double C = ttft + (double)out_len * tpot;",
-     "double C = ttft - (double)out_len * tpot;", 1),
-    ("cost_drops_ttft_f32", "float C = fmaf(out_len, tpot, ttft);",
-     "float C = out_len * tpot;", 1),
-    ("cost_uses_in_len", "double C = ttft + (double)out_len * tpot;",
-     "double C = ttft + (double)in_len * tpot;", 1),
+    ("cost_sign", "double C = ttft + n * tpot;", "double C = ttft - n * tpot;", 1),
+    ("cost_drops_ttft_f32", "float C = fmaf(n, tpot, ttft);", "float C = n * tpot;", 1),
+    ("cost_uses_in_len", "double n = m->n_heads == 3 ? nout : (double)out_len;",
+     "double n = m->n_heads == 3 ? nout : (double)in_len;", 1),
     ("utility_sign", "w->U[d] = wq * qual - (double)lam * C;",
      "w->U[d] = wq * qual + (double)lam * C;", 1),
     ("convex_weight", "double wq = convex ? 1.0 - (double)lam : 1.0;",
@@ -71,6 +69,12 @@ MUTANTS = [
     ("budget_order_f32", "float t = fmaf(b, p, a);\n    float s = slack * t;",
      "float t = b * p + a;\n    float s = slack * t;", 1),
     ("per_query_slo_first_only", "finish_query(m, &w, slo_q[q], mode,", "finish_query(m, &w, slo_q[0], mode,", 1),
+    ("third_head_ignored", "double n = m->n_heads == 3 ? nout : (double)out_len;",
+     "double n = (double)out_len;", 1),
+    ("third_head_ignored_f32", "float n = m->n_heads == 3 ? nout : out_len;",
+     "float n = out_len;", 1),
+    ("third_head_reads_ttft", "*nout = m->n_heads == 3 ? orc_softplus_f64(z[2]) : 0.0;",
+     "*nout = m->n_heads == 3 ? orc_softplus_f64(z[0]) : 0.0;", 1),
     ("per_query_seq_no_increment", "if (sequential && chosen[q] >= 0) running_io[chosen[q]] += 1;",
      "if (sequential && chosen[q] >= 0) running_io[chosen[q]] += 0;", 1),
 ]

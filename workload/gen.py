@@ -160,10 +160,13 @@ def _calibration(M, G, F, log10p, run_mean, wait_mean, in_len):
     return mean.astype(np.float32), std.astype(np.float32), xf
 
 
+OUT_LEN_MEDIAN = float(np.exp(5.0))   # median of the expected-output-length prior
+
+
 def make_problem(*, Q, M, G, F, H1, H2, E, dtype, lam, slo, log10p=(9.0, 11.0),
                  run_mean=8.0, wait_mean=3.0, in_len=(5.5, 1.0, 16.0, 4096.0),
                  seed=BASE_SEED, weight_std=0.1, bias_std=0.0,
-                 emb_bf16_values=False, name="custom", cfg=None):
+                 emb_bf16_values=False, name="custom", cfg=None, n_heads=2):
     """Draw one complete routing problem (table, predictor, state, queries)."""
     ss = np.random.SeedSequence(seed).spawn(8)
     rngs = [np.random.Generator(np.random.PCG64(s)) for s in ss]
@@ -179,14 +182,16 @@ def make_problem(*, Q, M, G, F, H1, H2, E, dtype, lam, slo, log10p=(9.0, 11.0),
     W1 = r.normal(0.0, weight_std, size=(H1, F)).astype(np.float32)
     W2 = r.normal(0.0, weight_std, size=(H2, H1)).astype(np.float32)
     W3 = r.normal(0.0, weight_std, size=(2, H2)).astype(np.float32)
+    if n_heads == 3:   # drawn after the others so two-head problems are unchanged
+        W3 = np.concatenate([W3, r.normal(0.0, weight_std, size=(1, H2)).astype(np.float32)])
     if bias_std > 0:
         b1 = r.normal(0.0, bias_std, size=H1).astype(np.float32)
         b2 = r.normal(0.0, bias_std, size=H2).astype(np.float32)
     else:
         b1 = np.zeros(H1, np.float32)
         b2 = np.zeros(H2, np.float32)
-    b3 = np.array([_softplus_inv(TTFT_MEDIAN), _softplus_inv(TPOT_MEDIAN)],
-                  np.float32)
+    b3 = np.array([_softplus_inv(TTFT_MEDIAN), _softplus_inv(TPOT_MEDIAN)]
+                  + ([_softplus_inv(OUT_LEN_MEDIAN)] if n_heads == 3 else []), np.float32)
     mu, sd, xf = calibration(M, G, F, log10p, run_mean, wait_mean, in_len)
 
     r = rngs[_S_MEMB]
@@ -201,7 +206,7 @@ def make_problem(*, Q, M, G, F, H1, H2, E, dtype, lam, slo, log10p=(9.0, 11.0),
     emb = _draw_embeddings(rngs[_S_QEMB], Q, E, bf16 or emb_bf16_values,
                            as_bits=bf16)
 
-    p = dict(name=name, cfg=cfg, Q=Q, M=M, G=G, D=D, F=F, H1=H1, H2=H2, E=E,
+    p = dict(name=name, cfg=cfg, Q=Q, M=M, G=G, D=D, F=F, H1=H1, H2=H2, E=E, n_heads=n_heads,
              dtype=dtype, lam=float(lam), slo=float(slo),
              dep_model=dep_model, dep_gpu=dep_gpu, log10p=log10p_m,
              b1=b1, b2=b2, b3=b3, mu=mu, sd=sd, xform=xf, snap=snap,
