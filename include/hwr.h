@@ -89,18 +89,21 @@ typedef struct {
     const float *model_log10_params;   /* [M] */
 } hwr_deployment_table;
 
-/* Latency predictor f_cost (Eq. 1): F -> H1 -> H2 -> 2 with ReLU after both
- * hidden layers and softplus on the two outputs (TTFT, TPOT).  Weights are
- * row-major [out][in] in `dtype` (fp32, or bf16 bit patterns as uint16):
- * W1 [H1][F], W2 [H2][H1], W3 [2][H2].  Biases and standardisation are fp32.
- * All arrays are host memory. */
+/* Latency predictor f_cost (Eq. 1): F -> H1 -> H2 -> NH with ReLU after
+ * both hidden layers and softplus on the outputs: TTFT, TPOT and, with three
+ * heads, the predicted output length N_out.  The cost of Eq. 2 uses N_out from
+ * the third head when there is one, else the query's given expected output
+ * length.  Weights are row-major [out][in] in `dtype` (fp32, or bf16 bit
+ * patterns as uint16): W1 [H1][F], W2 [H2][H1], W3 [NH][H2].  Biases and
+ * standardisation are fp32.  All arrays are host memory. */
 typedef struct {
     int32_t F, H1, H2;
     hwr_dtype dtype;
     const void *W1, *W2, *W3;
-    const float *b1, *b2, *b3;         /* [H1], [H2], [2] */
+    const float *b1, *b2, *b3;         /* [H1], [H2], [NH] */
     const float *feat_mean, *feat_std; /* [F]; feat_std must be non-zero */
     const uint8_t *feat_xform;         /* [F]: 0 identity, 1 log1p, 2 log */
+    int32_t n_heads;                   /* NH: 2 (or 0, meaning 2) or 3 */
 } hwr_predictor;
 
 /* Runtime signals S_i of one snapshot (Table 2, plus GPU utilisation), one

@@ -50,7 +50,8 @@ class hwr_predictor(ct.Structure):
                 ("dtype", ct.c_int), ("W1", ct.c_void_p), ("W2", ct.c_void_p),
                 ("W3", ct.c_void_p), ("b1", ct.c_void_p), ("b2", ct.c_void_p),
                 ("b3", ct.c_void_p), ("feat_mean", ct.c_void_p),
-                ("feat_std", ct.c_void_p), ("feat_xform", ct.c_void_p)]
+                ("feat_std", ct.c_void_p), ("feat_xform", ct.c_void_p),
+                ("n_heads", ct.c_int32)]
 
 
 class hwr_snapshot(ct.Structure):
@@ -207,7 +208,7 @@ class Router:
                            ptr(p["W3"], self.wdt), ptr(p["b1"], np.float32),
                            ptr(p["b2"], np.float32), ptr(p["b3"], np.float32),
                            ptr(p["mu"], np.float32), ptr(p["sd"], np.float32),
-                           ptr(p["xform"], np.uint8))
+                           ptr(p["xform"], np.uint8), int(p.get("n_heads", 2)))
         ctx = ct.c_void_p()
         st = self.lib.hwr_create(ct.byref(t), ct.byref(pr), ptr(p["memb"], self.wdt),
                                  self.E, HWR_BF16 if self.bf16 else HWR_F32,

@@ -42,7 +42,7 @@ constexpr int SMALL_MAX_PAIRS = 512;
 }  // namespace
 
 struct hwr_ctx {
-    int M = 0, G = 0, D = 0, F = 0, H1 = 0, H2 = 0, E = 0, P = 0;
+    int M = 0, G = 0, D = 0, F = 0, H1 = 0, H2 = 0, E = 0, P = 0, NH = 2;
     int Mpad = 0, Epad = 0;
     hwr_dtype dtype = HWR_F32;
     bool tc_ok = false;
@@ -216,7 +216,7 @@ static float bf16_bits_to_f32(uint16_t b) {
 static Model model_view(const hwr_ctx *c) {
     Model m;
     m.M = c->M; m.G = c->G; m.D = c->D; m.F = c->F; m.H1 = c->H1; m.H2 = c->H2;
-    m.E = c->E; m.P = c->P;
+    m.E = c->E; m.P = c->P; m.NH = c->NH;
     m.dep_model = c->dep_model; m.dep_gpu = c->dep_gpu; m.log10p = c->log10p;
     m.W1 = c->W1; m.b1 = c->b1; m.W2 = c->W2; m.b2 = c->b2; m.W3 = c->W3; m.b3 = c->b3;
     m.mu = c->mu; m.sd = c->sd; m.xform = c->xform; m.memb = c->memb;
@@ -229,7 +229,7 @@ static Model model_view(const hwr_ctx *c) {
 static TcModel tc_view(const hwr_ctx *c) {
     TcModel t;
     t.M = c->M; t.Mpad = c->Mpad; t.D = c->D; t.H1 = c->H1; t.H2 = c->H2;
-    t.E = c->E; t.Epad = c->Epad;
+    t.E = c->E; t.Epad = c->Epad; t.NH = c->NH;
     t.W2img = c->W2img; t.membimg = c->membimg; t.Abf = c->Abf; t.W1q = c->W1q;
     t.b2 = c->b2; t.W3 = c->W3; t.b3 = c->b3; t.dep_model = c->dep_model;
     t.mu_in = c->mu_in; t.sd_in = c->sd_in; t.mu_out = c->mu_out; t.sd_out = c->sd_out;
@@ -338,6 +338,8 @@ static hwr_status validate_create(const hwr_deployment_table *t, const hwr_predi
             return fail(nullptr, HWR_ERR_INVALID_ARG, "feature %d: std must be finite and non-zero", k);
         if (p->feat_xform[k] > 2) return fail(nullptr, HWR_ERR_INVALID_ARG, "feature %d: xform > 2", k);
     }
+    if (p->n_heads != 0 && p->n_heads != 2 && p->n_heads != 3)
+        return fail(nullptr, HWR_ERR_INVALID_ARG, "n_heads=%d (2 or 3)", p->n_heads);
     return HWR_OK;
 }
 
@@ -375,8 +377,9 @@ static hwr_status build_ctx(hwr_ctx *c, const hwr_deployment_table *t, const hwr
         }
         return v;
     };
+    const int NH = c->NH;
     std::vector<float> w1 = widen(p->W1, (size_t)H1 * F), w2 = widen(p->W2, (size_t)H2 * H1),
-                       w3 = widen(p->W3, (size_t)2 * H2), me = widen(memb_in, (size_t)E * M);
+                       w3 = widen(p->W3, (size_t)NH * H2), me = widen(memb_in, (size_t)E * M);
 
     TRY(dev_alloc(c, &c->dep_model, D));
     TRY(dev_alloc(c, &c->dep_gpu, D));
@@ -386,7 +389,7 @@ static hwr_status build_ctx(hwr_ctx *c, const hwr_deployment_table *t, const hwr
     TRY(dev_alloc(c, &c->W2, w2.size()));
     TRY(dev_alloc(c, &c->b2, H2));
     TRY(dev_alloc(c, &c->W3, w3.size()));
-    TRY(dev_alloc(c, &c->b3, 2));
+    TRY(dev_alloc(c, &c->b3, 3));
     TRY(dev_alloc(c, &c->mu, F));
     TRY(dev_alloc(c, &c->sd, F));
     TRY(dev_alloc(c, &c->xform, F));
@@ -415,7 +418,7 @@ static hwr_status build_ctx(hwr_ctx *c, const hwr_deployment_table *t, const hwr
     TRY(upload(c, c->W2, w2.data(), w2.size() * 4, "upload W2"));
     TRY(upload(c, c->b2, p->b2, H2 * 4, "upload b2"));
     TRY(upload(c, c->W3, w3.data(), w3.size() * 4, "upload W3"));
-    TRY(upload(c, c->b3, p->b3, 8, "upload b3"));
+    TRY(upload(c, c->b3, p->b3, (size_t)NH * 4, "upload b3"));
     TRY(upload(c, c->mu, p->feat_mean, F * 4, "upload mean"));
     TRY(upload(c, c->sd, p->feat_std, F * 4, "upload std"));
     TRY(upload(c, c->xform, p->feat_xform, F, "upload xform"));
@@ -456,7 +459,7 @@ static hwr_status build_ctx(hwr_ctx *c, const hwr_deployment_table *t, const hwr
         TRY(dev_alloc(c, &c->membimg, mimg.size()));
         TRY(upload(c, c->membimg, mimg.data(), mimg.size() * 2, "upload memb image"));
         c->head_consts.resize(tc_head_consts_bytes());
-        tc_fill_head_consts(c->head_consts.data(), p->b2, w3.data(), p->b3, H2);
+        tc_fill_head_consts(c->head_consts.data(), p->b2, w3.data(), p->b3, H2, NH);
     }
 
     // status word: mapped pinned host memory the kernels write directly
@@ -521,6 +524,7 @@ extern "C" hwr_status hwr_create(const hwr_deployment_table *table, const hwr_pr
     c->M = table->n_models; c->G = table->n_gpu_types; c->D = table->n_deployments;
     c->F = pred->F; c->H1 = pred->H1; c->H2 = pred->H2; c->E = E; c->P = c->M + c->G;
     c->dtype = pred->dtype;
+    c->NH = pred->n_heads == 3 ? 3 : 2;
     if (const char *h = getenv("HWR_TEST_FAIL_ALLOC")) c->hook.fail_at = atol(h);
     if (const char *h = getenv("HWR_TEST_STALL")) c->test_stall = atoi(h) != 0;
     if (const char *h = getenv("HWR_TC_MIN_PAIRS")) c->tc_min_pairs = atoi(h) > 1 ? atoi(h) : 1;

@@ -26,12 +26,13 @@ constexpr int SEQ_CHAIN_SMEM = 200 * 1024;
 // Read-only device view of the predictor and deployment state.
 struct Model {
     int M, G, D, F, H1, H2, E, P;
+    int NH;                     // output heads: 2 (TTFT, TPOT) or 3 (+ N_out)
     const int32_t *dep_model;   // [D]
     const int32_t *dep_gpu;     // [D]
     const float *log10p;        // [M]
     const float *W1, *b1;       // [H1][F], [H1]   fp32 (bf16 widened)
     const float *W2, *b2;       // [H2][H1], [H2]
-    const float *W3, *b3;       // [2][H2], [2]
+    const float *W3, *b3;       // [NH][H2], [NH]
     const float *mu, *sd;       // [F]
     const uint8_t *xform;       // [F]
     const float *memb;          // [E][M] fp32 (bf16 widened)
@@ -100,7 +101,7 @@ cudaError_t simt_prepare();   // one-time smem opt-in
 // ---- tcgen05 kernels (k_tc.cu) -------------------------------------------
 struct HeadConsts;
 struct TcModel {
-    int M, Mpad, D, H1, H2, E, Epad;
+    int M, Mpad, D, H1, H2, E, Epad, NH;
     const HeadConsts *head;     // host copy of b2, W3, b3 (kernel parameters)
     const uint16_t *W2img;      // bf16 W2 in the UMMA shared-memory image
     const uint16_t *membimg;    // bf16 memb^T in the UMMA shared-memory image
@@ -131,6 +132,7 @@ cudaError_t launch_mlp_tc(const TcModel &m, const Queries &q, const float *qual,
                           cudaStream_t s);
 cudaError_t tc_prepare();
 size_t tc_head_consts_bytes();
-void tc_fill_head_consts(void *dst, const float *b2, const float *W3, const float *b3, int H2);
+void tc_fill_head_consts(void *dst, const float *b2, const float *W3, const float *b3, int H2,
+                         int NH);
 
 }  // namespace hwr

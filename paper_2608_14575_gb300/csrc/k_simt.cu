@@ -100,7 +100,8 @@ __global__ void __launch_bounds__(SIMT_THREADS) k_snapshot(Model m) {
 // The shared SIMT tile: rows are (query, deployment) pairs.  For every row it
 // completes layer 1 from a deployment prefix and the two query features,
 // runs layer 2 (register-tiled, K ascending in chunks of SIMT_KC), layer 3
-// and the softplus heads.  Output: sp[2 r + 0] = TTFT, sp[2 r + 1] = TPOT.
+// and the softplus heads.  Output: sp[NH r + 0] = TTFT, sp[NH r + 1] = TPOT
+// and, with three heads, sp[NH r + 2] = N_out.
 //
 // Thread map: warp w owns rows w + 8 i (i < RPT); lane l owns columns
 // l + 32 j (j < CPT).  Shared memory: h1 [8 RPT][KC + 1] and W2 chunk
@@ -182,8 +183,8 @@ __device__ void pair_mlp(const Model &m, int R, const Rows &rows, const float *u
         }
     }
     __syncthreads();
-    for (int e = tid; e < 2 * R; e += SIMT_THREADS) {
-        const int r = e >> 1, o = e & 1;
+    for (int e = tid; e < m.NH * R; e += SIMT_THREADS) {
+        const int r = e / m.NH, o = e - r * m.NH;
         const float *w3 = m.W3 + (size_t)o * H2;
         float z = m.b3[o];
         for (int n = 0; n < H2; ++n) z = __fmaf_rn(w3[n], h2s[r * w2ld + n], z);
@@ -218,7 +219,7 @@ __host__ __device__ inline RouteLayout route_layout(int D, int M, int H2) {
     L.vs = o; o += 64;
     L.ol = o; o += 64;
     L.qual = o; o += (size_t)L.QB * M;
-    L.sp = o; o += 2 * 64;
+    L.sp = o; o += 3 * 64;
     L.C = o; o += 64;
     L.U = o; o += 64;
     o = (o + 3) & ~(size_t)3;
@@ -268,7 +269,8 @@ __global__ void __launch_bounds__(SIMT_THREADS) k_route_simt(Model m, Queries q)
 
     for (int r = tid; r < R; r += SIMT_THREADS) {
         const int qi = r / D, d = r - qi * D;
-        const float C = __fmaf_rn(ol[qi], sp[2 * r + 1], sp[2 * r]);
+        const float *h = sp + m.NH * r;   // TTFT, TPOT (, N_out)
+        const float C = __fmaf_rn(m.NH == 3 ? h[2] : ol[qi], h[1], h[0]);
         const float Ql = qual[qi * M + m.dep_model[d]];
         Cs[r] = C;
         Us[r] = __fmaf_rn(-q.lam, C, __fmul_rn(q.wq, Ql));
@@ -329,7 +331,7 @@ __host__ __device__ inline SeqLayout seq_layout(int H1, int H2) {
     L.vs = o; o += SEQ_MAX_CHUNK;
     L.ol = o; o += SEQ_MAX_CHUNK;
     L.pre = o; o += 2 * (size_t)H1;
-    L.sp = o; o += 2 * 8 * SEQ_RPT;
+    L.sp = o; o += 3 * 8 * SEQ_RPT;
     o = (o + 3) & ~(size_t)3;
     L.tile = o;
     o += tile_floats_for<SEQ_RPT>(H2);
@@ -391,7 +393,8 @@ k_seq_table(Model m, Queries q, int Qs, int nb_table, float *ctab, float *qualS)
 
     for (int r = tid; r < R; r += SIMT_THREADS) {
         const int c = r < n1 ? c1 : c2, i = rows.query(r);
-        const float C = __fmaf_rn(ol[i], sp[2 * r + 1], sp[2 * r]);
+        const float *h = sp + m.NH * r;
+        const float C = __fmaf_rn(m.NH == 3 ? h[2] : ol[i], h[1], h[0]);
         ctab[tri_off(D, Qs, c) + (size_t)d * (Qs - c) + (i - c)] = C;
     }
 }
@@ -526,8 +529,8 @@ __global__ void __launch_bounds__(SIMT_THREADS) k_route_pairs(Model m, Queries q
             h1[k] = x > 0.f ? x : 0.f;
         }
         __syncthreads();
-        float *w3s = sm + 2 * MAX_H;   // W3 [2][H2], staged for the head chains
-        for (int i = tid; i < 2 * H2; i += SIMT_THREADS) w3s[i] = m.W3[i];
+        float *w3s = sm + 2 * MAX_H;   // W3 [NH][H2], staged for the head chains
+        for (int i = tid; i < m.NH * H2; i += SIMT_THREADS) w3s[i] = m.W3[i];
         for (int n = tid; n < H2; n += SIMT_THREADS) {
             // serial chain over k (canonical order); W2 values fetched 32 at a
             // time, the next block in flight while this one is accumulated
@@ -548,18 +551,21 @@ __global__ void __launch_bounds__(SIMT_THREADS) k_route_pairs(Model m, Queries q
             h2[n] = acc > 0.f ? acc : 0.f;
         }
         __syncthreads();
-        if (tid < 64) {
-            // the two heads, one warp each
+        __shared__ float heads[3];
+        if (tid < 32 * m.NH) {
+            // the output heads, one warp each
             const int o = tid >> 5;
             if ((tid & 31) == 0) {
                 const float *w3 = w3s + (size_t)o * H2;
                 float z = m.b3[o];
                 for (int n = 0; n < H2; ++n) z = __fmaf_rn(w3[n], h2[n], z);
-                uv[o] = softplus_c(z);   // query features no longer needed
+                heads[o] = softplus_c(z);
             }
         }
         __syncthreads();
-        if (tid == 0) a.pairC[(size_t)qq * D + d] = __fmaf_rn(uv[2], uv[1], uv[0]);
+        if (tid == 0)
+            a.pairC[(size_t)qq * D + d] =
+                __fmaf_rn(m.NH == 3 ? heads[2] : uv[2], heads[1], heads[0]);
     } else {
         // quality of models [m0, m0 + PAIR_MPB) for one query
         const int b = blockIdx.x - npair;
@@ -657,7 +663,7 @@ cudaError_t launch_route_simt(const Model &m, const Queries &q, cudaStream_t s) 
 }
 
 size_t route_pairs_smem(const Model &m) {
-    const size_t pair = 4 * MAX_H * sizeof(float);
+    const size_t pair = 5 * MAX_H * sizeof(float);
     const size_t qual = (size_t)m.E * (1 + PAIR_MPB) * sizeof(float);
     return pair > qual ? pair : qual;
 }

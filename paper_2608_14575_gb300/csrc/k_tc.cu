@@ -109,7 +109,7 @@ __host__ __device__ inline MlpLayout mlp_layout(int H1, int H2, int Mpad, int D)
     MlpLayout L;
     uint32_t fixed = (uint32_t)H1 * H2 * 2                  // W2 image
                      + BM * (Mpad + 1) * 4                  // quality rows
-                     + (3 * H2 + 4) * 4 + D * 4             // b2, W3, b3, dep_model
+                     + (4 * H2 + 4) * 4 + D * 4             // b2, W3 (<= 3 rows), b3, dep_model
                      + (2 * MLP_MAX_STAGES + 6) * 8 + 16    // barriers, misc
                      + 1024 + 1024;                         // alignment slack
     int ns = (int)((SMEM_LIMIT - fixed) / CHUNK_BYTES);
@@ -123,7 +123,7 @@ __host__ __device__ inline MlpLayout mlp_layout(int H1, int H2, int Mpad, int D)
     L.qual = o;
     o += BM * (Mpad + 1) * 4;
     L.consts = o;
-    o += (3 * H2 + 4) * 4 + D * 4;
+    o += (4 * H2 + 4) * 4 + D * 4;
     o = (o + 7) & ~7u;
     L.bars = o;
     o += (2 * MLP_MAX_STAGES + 6) * 8;
@@ -327,9 +327,11 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
     return d;
 }
 
+template <int NH>
 __device__ __forceinline__ void head_pair(const uint32_t *v, int j, const float4 &bb,
-                                          const float4 &w0, const float4 &w1, float2 &t0a,
-                                          float2 &t0b, float2 &t1a, float2 &t1b) {
+                                          const float4 &w0, const float4 &w1, const float4 &w2,
+                                          float2 &t0a, float2 &t0b, float2 &t1a, float2 &t1b,
+                                          float2 &t2a, float2 &t2b) {
     // relu(acc + b2) for four columns, then both output heads as packed FMAs
     float2 x01 = __fadd2_rn(make_float2(__uint_as_float(v[j]), __uint_as_float(v[j + 1])),
                             make_float2(bb.x, bb.y));
@@ -343,16 +345,20 @@ __device__ __forceinline__ void head_pair(const uint32_t *v, int j, const float4
     t0b = __ffma2_rn(x23, make_float2(w0.z, w0.w), t0b);
     t1a = __ffma2_rn(x01, make_float2(w1.x, w1.y), t1a);
     t1b = __ffma2_rn(x23, make_float2(w1.z, w1.w), t1b);
+    if constexpr (NH == 3) {
+        t2a = __ffma2_rn(x01, make_float2(w2.x, w2.y), t2a);
+        t2b = __ffma2_rn(x23, make_float2(w2.z, w2.w), t2b);
+    }
 }
 
 // Output-layer constants passed by value: they sit in the kernel-parameter
 // constant bank, so the fully unrolled epilogue reads them as instruction
 // operands instead of shared-memory loads.
 struct HeadConsts {
-    float b2[MAX_H], w0[MAX_H], w1[MAX_H], b3[2];
+    float b2[MAX_H], w0[MAX_H], w1[MAX_H], w2[MAX_H], b3[3];
 };
 
-template <int H2T>
+template <int H2T, int NH>
 __global__ void __launch_bounds__(MLP_THREADS, 1)
 k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
          const float *__restrict__ qual, int nsplit, int4 *part, int32_t *count, int32_t *status) {
@@ -365,7 +371,7 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
     uint8_t *w2s = sm + L.w2, *ring = sm + L.ring;
     float *qs = (float *)(sm + L.qual);
     float *b2s = (float *)(sm + L.consts), *w30s = b2s + H2, *w31s = w30s + H2;
-    float *b3s = w31s + H2;
+    float *w32s = w31s + H2, *b3s = w32s + H2;
     int *dms = (int *)(b3s + 4);
     uint64_t *full = (uint64_t *)(sm + L.bars), *empty = full + MLP_MAX_STAGES;
     uint64_t *accf = empty + MLP_MAX_STAGES, *acce = accf + 2, *wbar = acce + 2, *dbar = wbar + 1;
@@ -394,8 +400,9 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
         b2s[i] = m.b2[i];
         w30s[i] = m.W3[i];
         w31s[i] = m.W3[H2 + i];
+        w32s[i] = NH == 3 ? m.W3[2 * H2 + i] : 0.f;
     }
-    if (tid < 2) b3s[tid] = m.b3[tid];
+    if (tid < NH) b3s[tid] = m.b3[tid];
     for (int i = tid; i < D; i += MLP_THREADS) dms[i] = m.dep_model[i];
     if (warp == 0) {
         tmem_alloc(tslot, tcols);
@@ -449,8 +456,9 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
         const int quad = warp & 3, r = quad * 32 + lane;
         const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
         const float slo = q.slo, lam = q.lam, wq = q.wq, b30 = b3s[0], b31 = b3s[1];
+        const float b32 = NH == 3 ? b3s[2] : 0.f;
         const float4 *b2v = (const float4 *)b2s, *w0v = (const float4 *)w30s,
-                     *w1v = (const float4 *)w31s;
+                     *w1v = (const float4 *)w31s, *w2v = (const float4 *)w32s;
         const int ncol = H2 / 32;
         uint32_t g = 0;
         bool ok = true;
@@ -470,7 +478,8 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
                 if (!ok) break;
                 tc_fence_after();
                 const uint32_t base = tmem + lane_base + (uint32_t)b * H2;
-                float2 t0a = make_float2(0.f, 0.f), t0b = t0a, t1a = t0a, t1b = t0a;
+                float2 t0a = make_float2(0.f, 0.f), t0b = t0a, t1a = t0a, t1b = t0a, t2a = t0a,
+                       t2b = t0a;
                 uint32_t va[32], vb[32];
                 tmem_ld32(base, va);
                 if constexpr (FIXED) {
@@ -484,10 +493,11 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
 #pragma unroll
                         for (int j = 0; j < 32; j += 4) {
                             const int n = c * 32 + j;
-                            head_pair(cur, j, make_float4(hc.b2[n], hc.b2[n + 1], hc.b2[n + 2], hc.b2[n + 3]),
-                                      make_float4(hc.w0[n], hc.w0[n + 1], hc.w0[n + 2], hc.w0[n + 3]),
-                                      make_float4(hc.w1[n], hc.w1[n + 1], hc.w1[n + 2], hc.w1[n + 3]),
-                                      t0a, t0b, t1a, t1b);
+                            head_pair<NH>(cur, j, make_float4(hc.b2[n], hc.b2[n + 1], hc.b2[n + 2], hc.b2[n + 3]),
+                                          make_float4(hc.w0[n], hc.w0[n + 1], hc.w0[n + 2], hc.w0[n + 3]),
+                                          make_float4(hc.w1[n], hc.w1[n + 1], hc.w1[n + 2], hc.w1[n + 3]),
+                                          make_float4(hc.w2[n], hc.w2[n + 1], hc.w2[n + 2], hc.w2[n + 3]),
+                                          t0a, t0b, t1a, t1b, t2a, t2b);
                         }
                     }
                 } else {
@@ -497,7 +507,8 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
 #pragma unroll
                         for (int j = 0; j < 32; j += 4) {
                             const int f = (c * 32 + j) >> 2;
-                            head_pair(va, j, b2v[f], w0v[f], w1v[f], t0a, t0b, t1a, t1b);
+                            head_pair<NH>(va, j, b2v[f], w0v[f], w1v[f], w2v[f], t0a, t0b, t1a, t1b,
+                                          t2a, t2b);
                         }
                         if (c + 1 < ncol) {
                             tmem_wait_ld32(vb);
@@ -505,7 +516,8 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
 #pragma unroll
                             for (int j = 0; j < 32; j += 4) {
                                 const int f = ((c + 1) * 32 + j) >> 2;
-                                head_pair(vb, j, b2v[f], w0v[f], w1v[f], t0a, t0b, t1a, t1b);
+                                head_pair<NH>(vb, j, b2v[f], w0v[f], w1v[f], w2v[f], t0a, t0b, t1a,
+                                              t1b, t2a, t2b);
                             }
                         }
                     }
@@ -514,8 +526,10 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
                 mbar_arrive(&acce[b]);
                 const float z0 = (t0a.x + t0a.y) + (t0b.x + t0b.y) + b30;
                 const float z1 = (t1a.x + t1a.y) + (t1b.x + t1b.y) + b31;
+                const float z2 = (t2a.x + t2a.y) + (t2b.x + t2b.y) + b32;
                 const float ttft = softplus_fast(z0), tpot = softplus_fast(z1);
-                const float C = fmaf(ol, tpot, ttft);
+                // N_out of Eq. 2: the third head, or the query's given length
+                const float C = fmaf(NH == 3 ? softplus_fast(z2) : ol, tpot, ttft);
                 const float U = fmaf(-lam, C, wq * qs[r * QS + dms[d]]);
                 const Cand cd = make_cand(C, U, d, slo_r);
                 if (better(cd, best)) best = cd;
@@ -675,12 +689,13 @@ cudaError_t tc_prepare() {
     }
     cudaError_t e = cudaFuncSetAttribute(k_qual_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          SMEM_LIMIT);
-    if (e == cudaSuccess)
-        e = cudaFuncSetAttribute(k_mlp_tc<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_LIMIT);
-    if (e == cudaSuccess)
-        e = cudaFuncSetAttribute(k_mlp_tc<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_LIMIT);
-    if (e == cudaSuccess)
-        e = cudaFuncSetAttribute(k_mlp_tc<256>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_LIMIT);
+    const auto attr = cudaFuncAttributeMaxDynamicSharedMemorySize;
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_mlp_tc<0, 2>, attr, SMEM_LIMIT);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_mlp_tc<128, 2>, attr, SMEM_LIMIT);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_mlp_tc<256, 2>, attr, SMEM_LIMIT);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_mlp_tc<0, 3>, attr, SMEM_LIMIT);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_mlp_tc<128, 3>, attr, SMEM_LIMIT);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_mlp_tc<256, 3>, attr, SMEM_LIMIT);
     return e;
 }
 
@@ -728,27 +743,35 @@ cudaError_t launch_mlp_tc(const TcModel &m, const Queries &q, const float *qual,
     const int grid = units < g_num_sms ? (int)units : g_num_sms;
     const MlpLayout L = mlp_layout(m.H1, m.H2, m.Mpad, m.D);
     const HeadConsts &hc = *m.head;
-    if (m.H2 == 256)
-        k_mlp_tc<256><<<grid, MLP_THREADS, L.total, s>>>(m, q, hc, qual, nsplit, (int4 *)part, count, status);
-    else if (m.H2 == 128)
-        k_mlp_tc<128><<<grid, MLP_THREADS, L.total, s>>>(m, q, hc, qual, nsplit, (int4 *)part, count, status);
-    else
-        k_mlp_tc<0><<<grid, MLP_THREADS, L.total, s>>>(m, q, hc, qual, nsplit, (int4 *)part, count, status);
+    int4 *pt = (int4 *)part;
+#define HWR_MLP(H2T, NHT) \
+    k_mlp_tc<H2T, NHT><<<grid, MLP_THREADS, L.total, s>>>(m, q, hc, qual, nsplit, pt, count, status)
+    if (m.NH == 3) {
+        if (m.H2 == 256) HWR_MLP(256, 3);
+        else if (m.H2 == 128) HWR_MLP(128, 3);
+        else HWR_MLP(0, 3);
+    } else {
+        if (m.H2 == 256) HWR_MLP(256, 2);
+        else if (m.H2 == 128) HWR_MLP(128, 2);
+        else HWR_MLP(0, 2);
+    }
+#undef HWR_MLP
     return cudaGetLastError();
 }
 
 size_t tc_head_consts_bytes() { return sizeof(HeadConsts); }
 
-void tc_fill_head_consts(void *dst, const float *b2, const float *W3, const float *b3, int H2) {
+void tc_fill_head_consts(void *dst, const float *b2, const float *W3, const float *b3, int H2,
+                         int NH) {
     HeadConsts *h = (HeadConsts *)dst;
     memset(h, 0, sizeof *h);
     for (int i = 0; i < H2; ++i) {
         h->b2[i] = b2[i];
         h->w0[i] = W3[i];
         h->w1[i] = W3[H2 + i];
+        h->w2[i] = NH == 3 ? W3[2 * H2 + i] : 0.f;
     }
-    h->b3[0] = b3[0];
-    h->b3[1] = b3[1];
+    for (int o = 0; o < NH; ++o) h->b3[o] = b3[o];
 }
 
 }  // namespace hwr

@@ -207,3 +207,18 @@ def test_online_sequential_full_100k_exact():
     bad = np.nonzero(g != c)[0]
     assert bad.size == 0, f"first divergence at request {bad[:1]}"
     assert len(np.unique(g)) > 1
+
+
+# ---------------------------------------------------------------------------
+# three output heads: N_out predicted (Eq. 1) and used by the cost (Eq. 2)
+
+@pytest.mark.parametrize("c,Q,flags", [(0, 50, 0), (0, 256, 0), (1, 300, SIMT),
+                                       (2, 120, H.HWR_SEQUENTIAL)])
+def test_three_heads_simt_exact(c, Q, flags):
+    p = W.make_config(c, Q=Q, n_heads=3)
+    r = H.Router(p)
+    got = r.route(flags=flags)
+    want = O.Problem(p).route(mode=O.F32, sequential=bool(flags & H.HWR_SEQUENTIAL),
+                              nthreads=8)
+    assert_exact(got, want, f"three heads cfg{c}")
+    r.close()

@@ -162,3 +162,11 @@ def test_pipelined_host_batch_matches_device_path():
     assert all(np.array_equal(a, b) for a, b in zip(host, again))
     assert np.array_equal(small[0], host[0][:100])
     r.close()
+
+
+@pytest.mark.parametrize("c,Q", [(1, 2000), (3, 3000)])
+def test_three_heads_tensor(c, Q):
+    p = W.make_config(c, Q=Q, n_heads=3)
+    r = H.Router(p)
+    check_against_oracle(p, r.route(flags=TC), min_checked=0.3)
+    r.close()
