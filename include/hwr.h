@@ -213,6 +213,25 @@ hwr_status hwr_route_batch_slo(hwr_ctx *ctx, int32_t Q, const float *in_len,
                                float *pred_latency, float *utility);
 
 /*
+ * Route one batch for K values of lambda at once (1 <= K <= 16): the
+ * predictor and the quality scores are evaluated once and the decision maker
+ * of Eq. 3 is applied for every lambda -- the routing half of the paper's
+ * quality-latency Pareto sweep over lambda (Sec. 5, RQ1).
+ *   lambdas     [K] host array of finite values;
+ *   chosen, pred_latency, utility   [K][Q]: row k holds the results for
+ *               lambdas[k] (host or device memory per HWR_DEVICE_PTRS).
+ * Each row equals what hwr_route_batch returns for that lambda.  Flags as for
+ * hwr_route_batch except HWR_SEQUENTIAL (UNSUPPORTED).
+ * Errors: as hwr_route_batch; INVALID_ARG for K out of range or a
+ * non-finite lambda.
+ */
+hwr_status hwr_route_batch_multi(hwr_ctx *ctx, int32_t Q, const float *in_len,
+                                 const float *out_len, const void *q_emb,
+                                 float slo, const float *lambdas, int32_t K,
+                                 uint32_t flags, int32_t *chosen,
+                                 float *pred_latency, float *utility);
+
+/*
  * Route a batch without allocating anything at call time.
  *
  * The paper has no counterpart to this call; it exists for callers that

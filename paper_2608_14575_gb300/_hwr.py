@@ -34,7 +34,8 @@ KERNELS = ("snapshot", "route_simt", "seq_table", "qual_tc", "mlp_tc")
 HWR_K_COUNT = len(KERNELS)
 
 EXPORTS = ("hwr_create", "hwr_update_snapshot", "hwr_get_snapshot",
-           "hwr_route_batch", "hwr_route_batch_slo", "hwr_route_batch_noalloc", "hwr_synchronize",
+           "hwr_route_batch", "hwr_route_batch_slo", "hwr_route_batch_multi",
+           "hwr_route_batch_noalloc", "hwr_synchronize",
            "hwr_destroy", "hwr_status_string", "hwr_last_error", "hwr_get_stats")
 HWR_NOALLOC_MAX_Q = 32768
 
@@ -105,6 +106,8 @@ def load(path: str | None = None):
         lib.hwr_route_batch_noalloc.argtypes = lib.hwr_route_batch.argtypes
         lib.hwr_route_batch_slo.argtypes = [P, ct.c_int32, P, P, P, P, ct.c_float,
                                             ct.c_uint32, P, P, P]
+        lib.hwr_route_batch_multi.argtypes = [P, ct.c_int32, P, P, P, ct.c_float, P,
+                                              ct.c_int32, ct.c_uint32, P, P, P]
         lib.hwr_synchronize.argtypes = [P]
         lib.hwr_destroy.argtypes = [P]
         lib.hwr_status_string.argtypes = [I]
@@ -113,8 +116,9 @@ def load(path: str | None = None):
         lib.hwr_last_error.restype = ct.c_char_p
         lib.hwr_get_stats.argtypes = [P, P, I]
         for n in ("hwr_create", "hwr_update_snapshot", "hwr_get_snapshot",
-                  "hwr_route_batch", "hwr_route_batch_slo", "hwr_route_batch_noalloc",
-                  "hwr_synchronize", "hwr_destroy", "hwr_get_stats"):
+                  "hwr_route_batch", "hwr_route_batch_slo", "hwr_route_batch_multi",
+                  "hwr_route_batch_noalloc", "hwr_synchronize", "hwr_destroy",
+                  "hwr_get_stats"):
             getattr(lib, n).restype = I
         if path is None:
             _lib = lib
@@ -145,6 +149,12 @@ def hwr_route_batch_slo(ctx, Q, in_len, out_len, q_emb, slo, lam, flags, chosen,
                         pred_latency, utility):
     return load().hwr_route_batch_slo(ctx, Q, in_len, out_len, q_emb, slo, lam, flags,
                                       chosen, pred_latency, utility)
+
+
+def hwr_route_batch_multi(ctx, Q, in_len, out_len, q_emb, slo, lambdas, K, flags, chosen,
+                          pred_latency, utility):
+    return load().hwr_route_batch_multi(ctx, Q, in_len, out_len, q_emb, slo, lambdas, K, flags,
+                                        chosen, pred_latency, utility)
 
 
 def hwr_route_batch_noalloc(ctx, Q, in_len, out_len, q_emb, slo, lam, flags, chosen,
@@ -251,6 +261,34 @@ class Router:
             float(p["lam"] if lam is None else lam), int(flags) & ~HWR_DEVICE_PTRS,
             chosen.ctypes.data, lat.ctypes.data, util.ctypes.data))
         return chosen, lat, util
+
+    def route_multi(self, lambdas, in_len=None, out_len=None, emb=None, *, slo=None,
+                    flags=0):
+        """Host routing for several lambdas; outputs have shape [K][Q]."""
+        p = self.p
+        il = _c(p["in_len"] if in_len is None else in_len, np.float32)
+        ol = _c(p["out_len"] if out_len is None else out_len, np.float32)
+        em = _c(p["emb"] if emb is None else emb, self.wdt)
+        lam = _c(lambdas, np.float32)
+        Q, K = il.size, lam.size
+        chosen = np.empty((K, Q), np.int32)
+        lat = np.empty((K, Q), np.float32)
+        util = np.empty((K, Q), np.float32)
+        self._check(self.lib.hwr_route_batch_multi(
+            self.ctx, Q, il.ctypes.data, ol.ctypes.data, em.ctypes.data,
+            float(p["slo"] if slo is None else slo), lam.ctypes.data, K,
+            int(flags) & ~HWR_DEVICE_PTRS, chosen.ctypes.data, lat.ctypes.data,
+            util.ctypes.data))
+        return chosen, lat, util
+
+    def route_device_multi(self, lambdas, in_len, out_len, emb, chosen, lat, util, *, slo,
+                           flags=0):
+        """Device routing for several lambdas into [K][Q] CUDA tensors."""
+        lam = _c(lambdas, np.float32)
+        self._check(self.lib.hwr_route_batch_multi(
+            self.ctx, int(in_len.numel()), in_len.data_ptr(), out_len.data_ptr(),
+            emb.data_ptr(), float(slo), lam.ctypes.data, int(lam.size),
+            int(flags) | HWR_DEVICE_PTRS, chosen.data_ptr(), lat.data_ptr(), util.data_ptr()))
 
     def route_slo(self, in_len=None, out_len=None, emb=None, *, budgets=None,
                   model=None, lam=None, flags=0):

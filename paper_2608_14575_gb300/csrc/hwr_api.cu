@@ -88,6 +88,8 @@ struct hwr_ctx {
     char *part = nullptr;    size_t part_cap = 0;     // split-deployment partials
     int32_t *count = nullptr; size_t count_cap = 0;   // per-row arrivals (self-resetting)
     float *pairC = nullptr;  float *pairQ = nullptr;  int32_t *pairN = nullptr;  // small batches
+    float *mC = nullptr;     size_t mC_cap = 0;       // multi-lambda: pair costs [Q][D]
+    float *mQ = nullptr;     size_t mQ_cap = 0;       // multi-lambda: quality [Q][M]
     float *ctab = nullptr;   size_t ctab_cap = 0;
     float *qseq = nullptr;   size_t qseq_cap = 0;
     int seq_qs = 0;
@@ -658,7 +660,7 @@ static size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 static hwr_status route_impl(hwr_ctx *c, int32_t Q, const float *in_len, const float *out_len,
                              const void *q_emb, float slo, const hwr_slo_spec *spec,
                              float lambda, uint32_t flags, int32_t *chosen,
-                             float *pred_latency, float *utility) {
+                             float *pred_latency, float *utility, const Lambdas *ml = nullptr) {
     if (!c) return fail(nullptr, HWR_ERR_INVALID_ARG, "ctx is NULL");
     if (c->broken) return HWR_ERR_STATE;
     const uint32_t known = HWR_SEQUENTIAL | HWR_DEVICE_PTRS | HWR_ASYNC | HWR_SCORE_CONVEX |
@@ -688,6 +690,8 @@ static hwr_status route_impl(hwr_ctx *c, int32_t Q, const float *in_len, const f
                           (long)Q * c->D > c->pairs_max));
     const bool dev = flags & HWR_DEVICE_PTRS;
     const size_t es = c->dtype == HWR_BF16 ? 2 : 4;
+    const int K = ml ? ml->K : 1;
+    if (ml && seq) return fail(c, HWR_ERR_UNSUPPORTED, "several lambdas with HWR_SEQUENTIAL");
     if (dev && tensor && ((uintptr_t)q_emb & 15))
         return fail(c, HWR_ERR_INVALID_ARG, "device q_emb must be 16-byte aligned");
 
@@ -710,8 +714,9 @@ static hwr_status route_impl(hwr_ctx *c, int32_t Q, const float *in_len, const f
     const size_t off_in = align_up(emb_b, 256), off_out = off_in + align_up(len_b, 256);
     const size_t off_slo = off_out + align_up(len_b, 256);
     const size_t in_total = (budgets ? off_slo : off_out) + len_b;
-    const size_t o_lat = align_up(len_b, 256), o_util = o_lat + align_up(len_b, 256);
-    const size_t out_total = o_util + len_b;
+    const size_t outs_b = (size_t)K * len_b;   // each output holds K rows of Q
+    const size_t o_lat = align_up(outs_b, 256), o_util = o_lat + align_up(outs_b, 256);
+    const size_t out_total = o_util + outs_b;
     const bool packed = !dev && !(flags & HWR_ASYNC) && in_total <= ((size_t)1 << 20);
     // Large host batches: copy in chunks on the copy stream while the kernels
     // of the previous chunk run (the link, not the GPU, bounds this path).
@@ -754,6 +759,34 @@ static hwr_status route_impl(hwr_ctx *c, int32_t Q, const float *in_len, const f
         q.util = (float *)(c->out_d + o_util);
     }
 
+    const Model mv = model_view(c);
+    if (ml) {
+        TRY(grow(c, &c->mC, &c->mC_cap, (size_t)Q * c->D));
+        TRY(grow(c, &c->mQ, &c->mQ_cap, (size_t)Q * c->M));
+    }
+    // One chunk [lo, lo + n): its kernels, then (several lambdas) the selection
+    // for every lambda from the scores the kernels stored.
+    auto run_chunk = [&](Queries qc, int lo) -> hwr_status {
+        const bool small = !tensor && (long)qc.Q * c->D <= c->pairs_max;
+        if (ml) {
+            qc.pair_C = c->mC;
+            qc.qual_out = c->mQ;
+        }
+        TRY(run_kernels(c, qc, flags, tensor));
+        if (!ml) return HWR_OK;
+        Queries qs = qc;
+        qs.chosen = q.chosen + lo;
+        qs.lat = q.lat + lo;
+        qs.util = q.util + lo;
+        const float *Cs = small ? c->pairC : c->mC;
+        const float *qual = tensor ? c->qual : (small ? c->pairQ : c->mQ);
+        const int qstride = tensor ? c->Mpad : c->M;
+        LaunchScope ls(c, HWR_K_ROUTE_SIMT, flags & HWR_PROFILE);
+        CK(c, launch_select_multi(mv, qs, Cs, qual, qstride, *ml, Q, c->stream), "select kernel");
+        ls.done();
+        return HWR_OK;
+    };
+
     if (pipelined) {
         // everything already queued on the context stream (earlier calls'
         // kernels read io_d) must finish before io_d is rewritten
@@ -785,10 +818,10 @@ static hwr_status route_impl(hwr_ctx *c, int32_t Q, const float *in_len, const f
             qc.lat = q.lat + lo;
             qc.util = q.util + lo;
             if (q.slo_q) qc.slo_q = q.slo_q + lo;
-            TRY(run_kernels(c, qc, flags, tensor));
+            TRY(run_chunk(qc, lo));
         }
     } else {
-        TRY(run_kernels(c, q, flags, tensor));
+        TRY(run_chunk(q, 0));
     }
 
     bool synced = false;
@@ -799,15 +832,16 @@ static hwr_status route_impl(hwr_ctx *c, int32_t Q, const float *in_len, const f
             CK(c, cudaEventRecord(c->pin_ev, c->stream), "record");
             CK(c, cudaStreamSynchronize(c->stream), "synchronize");
             synced = true;
-            memcpy(chosen, c->pin_h, len_b);
-            memcpy(pred_latency, c->pin_h + o_lat, len_b);
-            memcpy(utility, c->pin_h + o_util, len_b);
+            memcpy(chosen, c->pin_h, outs_b);
+            memcpy(pred_latency, c->pin_h + o_lat, outs_b);
+            memcpy(utility, c->pin_h + o_util, outs_b);
         } else {
-            CK(c, cudaMemcpyAsync(chosen, c->out_d, len_b, cudaMemcpyDeviceToHost, c->stream), "copy chosen");
-            CK(c, cudaMemcpyAsync(pred_latency, c->out_d + o_lat, len_b, cudaMemcpyDeviceToHost, c->stream),
-               "copy latency");
-            CK(c, cudaMemcpyAsync(utility, c->out_d + o_util, len_b, cudaMemcpyDeviceToHost, c->stream),
-               "copy utility");
+            CK(c, cudaMemcpyAsync(chosen, c->out_d, outs_b, cudaMemcpyDeviceToHost, c->stream),
+               "copy chosen");
+            CK(c, cudaMemcpyAsync(pred_latency, c->out_d + o_lat, outs_b, cudaMemcpyDeviceToHost,
+                                  c->stream), "copy latency");
+            CK(c, cudaMemcpyAsync(utility, c->out_d + o_util, outs_b, cudaMemcpyDeviceToHost,
+                                  c->stream), "copy utility");
         }
     }
     c->stats.queries_routed += Q;
@@ -824,6 +858,26 @@ extern "C" hwr_status hwr_route_batch(hwr_ctx *c, int32_t Q, const float *in_len
                                       float *pred_latency, float *utility) {
     return route_impl(c, Q, in_len, out_len, q_emb, slo, nullptr, lambda, flags, chosen,
                       pred_latency, utility);
+}
+
+extern "C" hwr_status hwr_route_batch_multi(hwr_ctx *c, int32_t Q, const float *in_len,
+                                            const float *out_len, const void *q_emb, float slo,
+                                            const float *lambdas, int32_t K, uint32_t flags,
+                                            int32_t *chosen, float *pred_latency,
+                                            float *utility) {
+    if (!c) return fail(nullptr, HWR_ERR_INVALID_ARG, "ctx is NULL");
+    if (!lambdas) return fail(c, HWR_ERR_INVALID_ARG, "lambdas is NULL");
+    if (K < 1 || K > MAX_LAMBDAS)
+        return fail(c, HWR_ERR_INVALID_ARG, "K=%d outside [1, %d]", K, MAX_LAMBDAS);
+    Lambdas L;
+    L.K = K;
+    for (int k = 0; k < K; ++k) {
+        if (!isfinite(lambdas[k])) return fail(c, HWR_ERR_INVALID_ARG, "lambda %d not finite", k);
+        L.lam[k] = lambdas[k];
+        L.wq[k] = (flags & HWR_SCORE_CONVEX) ? 1.0f - lambdas[k] : 1.0f;
+    }
+    return route_impl(c, Q, in_len, out_len, q_emb, slo, nullptr, lambdas[0], flags, chosen,
+                      pred_latency, utility, &L);
 }
 
 extern "C" hwr_status hwr_route_batch_slo(hwr_ctx *c, int32_t Q, const float *in_len,

@@ -59,6 +59,17 @@ struct Queries {
     int slo_mode = 0;
     const float *slo_q = nullptr;
     float slo_a = 0.f, slo_b = 0.f, slo_slack = 1.f, slo_tpot = 0.f;
+    // when set, kernels also store every pair's cost C [Q][D] and (SIMT fused
+    // kernel) every query's quality [Q][M] for a later multi-lambda selection
+    float *pair_C = nullptr;
+    float *qual_out = nullptr;
+};
+
+// Several values of lambda applied to one set of scores.
+constexpr int MAX_LAMBDAS = 16;
+struct Lambdas {
+    int K;
+    float lam[MAX_LAMBDAS], wq[MAX_LAMBDAS];
 };
 
 #ifdef __CUDACC__
@@ -92,6 +103,11 @@ cudaError_t launch_seq_table(const Model &m, const Queries &q, int Qs,
                              float *ctab, float *qual, cudaStream_t s);
 cudaError_t launch_seq_chain(const Model &m, const Queries &q, int Qs,
                              const float *ctab, const float *qual, cudaStream_t s);
+// Decision maker for K lambdas from stored scores: C [Q][D], quality
+// qual[q * qstride + model]; outputs [K][ostride] starting at query 0.
+cudaError_t launch_select_multi(const Model &m, const Queries &q, const float *C,
+                                const float *qual, int qstride, const Lambdas &L, int ostride,
+                                cudaStream_t s);
 int seq_chunk(const Model &m);
 size_t seq_table_floats(int D, int Qs);
 size_t route_simt_smem(const Model &m);

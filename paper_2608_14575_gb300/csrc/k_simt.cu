@@ -274,7 +274,11 @@ __global__ void __launch_bounds__(SIMT_THREADS) k_route_simt(Model m, Queries q)
         const float Ql = qual[qi * M + m.dep_model[d]];
         Cs[r] = C;
         Us[r] = __fmaf_rn(-q.lam, C, __fmul_rn(q.wq, Ql));
+        if (q.pair_C && q0 + qi < q.Q) q.pair_C[(size_t)(q0 + qi) * D + d] = C;
     }
+    if (q.qual_out)
+        for (int e = tid; e < QB * M; e += SIMT_THREADS)
+            if (q0 + e / M < q.Q) q.qual_out[(size_t)q0 * M + e] = qual[e];
     __syncthreads();
 
     for (int qi = warp; qi < QB; qi += SIMT_THREADS / 32) {
@@ -600,6 +604,34 @@ __global__ void __launch_bounds__(SIMT_THREADS) k_route_pairs(Model m, Queries q
 }
 
 // ---------------------------------------------------------------------------
+// K_select_multi: the decision maker for several lambdas over stored scores
+// (one warp per (query, lambda)); same candidate order as everywhere else.
+
+__global__ void __launch_bounds__(SIMT_THREADS)
+k_select_multi(Model m, Queries q, const float *C, const float *qual, int qstride, Lambdas L,
+               int ostride) {
+    const int wid = (blockIdx.x * SIMT_THREADS + threadIdx.x) >> 5, lane = threadIdx.x & 31;
+    if (wid >= q.Q * L.K) return;
+    const int k = wid / q.Q, qq = wid - k * q.Q;
+    const float slo = query_budget(q, qq), lam = L.lam[k], wq = L.wq[k];
+    Cand best = no_cand();
+    for (int d = lane; d < m.D; d += 32) {
+        const float c = C[(size_t)qq * m.D + d];
+        const float Ql = qual[(size_t)qq * qstride + m.dep_model[d]];
+        Cand cd = make_cand(c, __fmaf_rn(-lam, c, __fmul_rn(wq, Ql)), d, slo);
+        if (better(cd, best)) best = cd;
+    }
+    best = warp_best(best);
+    if (lane == 0) {
+        const bool ok = best.cls > 0;
+        const size_t o = (size_t)k * ostride + qq;
+        q.chosen[o] = ok ? best.d : -1;
+        q.lat[o] = ok ? best.C : __int_as_float(0x7fc00000);
+        q.util[o] = ok ? best.U : __int_as_float(0x7fc00000);
+    }
+}
+
+// ---------------------------------------------------------------------------
 // host launchers
 
 static int cpt_for(int H2) { return H2 <= 32 ? 1 : H2 <= 64 ? 2 : H2 <= 128 ? 4 : 8; }
@@ -679,6 +711,16 @@ cudaError_t launch_route_pairs(const Model &m, const Queries &q, const float *W2
     a.qblocks = (m.M + PAIR_MPB - 1) / PAIR_MPB;
     const int blocks = q.Q * (m.D + a.qblocks);
     k_route_pairs<<<blocks, SIMT_THREADS, route_pairs_smem(m), s>>>(m, q, a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_select_multi(const Model &m, const Queries &q, const float *C,
+                                const float *qual, int qstride, const Lambdas &L, int ostride,
+                                cudaStream_t s) {
+    if (q.Q <= 0 || L.K <= 0) return cudaSuccess;
+    const long warps = (long)q.Q * L.K;
+    const int blocks = (int)((warps * 32 + SIMT_THREADS - 1) / SIMT_THREADS);
+    k_select_multi<<<blocks, SIMT_THREADS, 0, s>>>(m, q, C, qual, qstride, L, ostride);
     return cudaGetLastError();
 }
 

@@ -531,6 +531,7 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
                 // N_out of Eq. 2: the third head, or the query's given length
                 const float C = fmaf(NH == 3 ? softplus_fast(z2) : ol, tpot, ttft);
                 const float U = fmaf(-lam, C, wq * qs[r * QS + dms[d]]);
+                if (q.pair_C && valid) q.pair_C[(size_t)row * D + d] = C;
                 const Cand cd = make_cand(C, U, d, slo_r);
                 if (better(cd, best)) best = cd;
             }
