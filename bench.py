@@ -18,8 +18,15 @@ Printed (one JSON line, rank 0):
             its CUDA-event duration, against the measured GB300 peak;
   q1_latency_us  p50 / p99 single-query route latency through the C ABI with
             host buffers, at D = 32 (the batch-sweep shape);
-  cpu_baseline   the CPU oracle on a bounded sample of the same workload.
+  cpu_baseline   the CPU oracle on a bounded sample of the same workload;
+  multi_lambda   one hwr_route_batch_multi call for 8 values of lambda on the
+            same batch (the Sec. 5 lambda sweep), next to 8 single routes.
 --impl reference times the CPU oracle (the reference arm for this build).
+--online prints the online evaluation metrics of Sec. 4.3 (SLO attainment,
+queue composition, load/running/waiting skew) for the online sequential
+workload's shapes under each arrival pattern, for the hardware-aware router
+and for the frozen-snapshot static-cost mode, one JSON line each, with the
+wall-clock time of each micro-batch's route call through the C ABI.
 """
 from __future__ import annotations
 
@@ -254,6 +261,90 @@ def q1_latency(H, iters=2000):
             "paper_routing_overhead_us": 200.0}
 
 
+# Online scenarios on the online sequential workload's shapes (D = 12).  The
+# serving world has 16 slots per deployment and 0.5 s mean service, so it
+# completes 384 requests/s with every slot busy.
+ONLINE_SCENARIOS = {
+    "online_sequential": dict(),   # the workload itself: Poisson 200 req/s, batches of 64
+    "poisson": dict(pattern="poisson", rate=200.0, window=0.02, cap=16, drain="per_time",
+                    service_s=0.5),
+    "micro_burst": dict(pattern="micro_burst", rate=150.0, window=0.02, cap=16,
+                        drain="per_time", service_s=0.5, burst_factor=8.0, burst_len=0.05,
+                        period=1.0),
+    "sustained_overload": dict(pattern="sustained_overload", rate=384.0, window=0.02, cap=16,
+                               drain="per_time", service_s=0.5, overload=1.25),
+}
+
+
+def online_report(args):
+    import paper_2608_14575_gb300 as H
+    from paper_2608_14575_gb300 import metrics as MX
+    from paper_2608_14575_gb300.online import OnlineRouter
+    from workload import serve
+    H.build()
+    p = W.make_config(2, Q=args.q or 20_000)
+    for name, world in ONLINE_SCENARIOS.items():
+        for mode, static in (("hw_router", False), ("static_cost", True)):
+            times = []
+            with OnlineRouter(p) as r:
+                def route(snap, lo, hi):
+                    t = time.perf_counter()
+                    out = r.route(snap, lo, hi)
+                    times.append(time.perf_counter() - t)
+                    return out
+                tr = serve.run_online(p, route, r.score, static=static, **world)
+            m = MX.summarize(tr, p["dep_gpu"], p["G"], p["D"])
+            us = np.array(times) * 1e6
+            sizes = tr["batch_end"] - tr["batch_start"]
+            print(json.dumps({
+                "online": name, "mode": mode, "workload": workload_name(p),
+                "world": {k: v for k, v in world.items()}, **m,
+                "route_call_us": {"p50": float(np.percentile(us, 50)),
+                                  "p99": float(np.percentile(us, 99)),
+                                  "mean_batch": float(sizes[sizes > 0].mean()),
+                                  "note": "snapshot upload + sequential route of one "
+                                          "micro-batch, host buffers, wall clock"}}),
+                flush=True)
+
+
+def multi_lambda(H, r, p, bufs, flags, stream, steps=10):
+    """One 8-lambda call against 8 single-lambda calls on the same device batch."""
+    import torch
+    lams = np.linspace(0.05, 2.0, 8).astype(np.float32)
+    Q, K = p["Q"], len(lams)
+    dev = bufs[0][0].device
+    ch = torch.empty((K, Q), dtype=torch.int32, device=dev)
+    lat = torch.empty((K, Q), dtype=torch.float32, device=dev)
+    ut = torch.empty((K, Q), dtype=torch.float32, device=dev)
+    torch.cuda.synchronize()
+    il, ol, em = bufs[0]
+
+    fa = flags | H.HWR_ASYNC
+
+    def multi():
+        r.route_device_multi(lams, il, ol, em, ch, lat, ut, slo=p["slo"], flags=fa)
+
+    def singles():
+        for k in range(K):
+            r.route_device(il, ol, em, ch[k], lat[k], ut[k], slo=p["slo"], lam=float(lams[k]),
+                           flags=fa)
+    res = {}
+    for name, fn in (("multi", multi), ("singles", singles)):
+        for _ in range(3):
+            fn()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(steps):
+            fn()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        r.synchronize()
+        res[name] = e0.elapsed_time(e1) / steps
+    return {"lambdas": K, "ms_per_call": res["multi"], "ms_8_single_calls": res["singles"],
+            "lambda_routes_per_s": Q * K / (res["multi"] * 1e-3)}
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
     ap.add_argument("--gpus", type=int, default=1)
@@ -267,9 +358,16 @@ def main():
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--no-q1", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
+    ap.add_argument("--no-multi", action="store_true")
+    ap.add_argument("--online", action="store_true",
+                    help="print the online evaluation metrics instead of the throughput line")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
     rank, world, local = dist_env()
+    if args.online:
+        if rank == 0:
+            online_report(args)
+        return
 
     if args.impl == "reference":
         if rank == 0:
@@ -289,7 +387,10 @@ def main():
     p = W.make_config(args.config, Q=args.q, seed_offset=rank)
     Q = p["Q"]
     dev = torch.device("cuda", local)
-    stream = torch.cuda.current_stream()
+    # a stream of its own (the default stream's handle is NULL, for which the
+    # library would create a private stream): the CUDA events below are
+    # recorded on the stream the kernels run on
+    stream = torch.cuda.Stream(device=dev)
     r = H.Router(p, stream=stream.cuda_stream)
     flags = {"auto": 0, "simt": H.HWR_PATH_SIMT, "tensor": H.HWR_PATH_TENSOR}[args.path]
 
@@ -303,6 +404,7 @@ def main():
     ch = torch.empty(Q, dtype=torch.int32, device=dev)
     lat = torch.empty(Q, dtype=torch.float32, device=dev)
     ut = torch.empty(Q, dtype=torch.float32, device=dev)
+    torch.cuda.synchronize()      # inputs are written on the default stream
 
     def step(k, extra=0):
         il, ol, em = bufs[k % nbuf]
@@ -322,10 +424,11 @@ def main():
     torch.cuda.synchronize()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
-    for k in range(args.steps):
-        step(k, H.HWR_PROFILE)
+    for k in range(args.steps):     # queued back to back; status checked after
+        step(k, H.HWR_PROFILE | H.HWR_ASYNC)
     e1.record(stream)
     torch.cuda.synchronize()
+    r.synchronize()
     if dist:
         dist.barrier()
     clk = clocks.stop()
@@ -398,6 +501,8 @@ def main():
         line["e2e"] = {"value": whole_job_rate(Q, world, dt), "unit": "queries/s",
                        "h2d_bytes_per_step": Q * (bytes_per_query(p) - 12),
                        "d2h_bytes_per_step": Q * 12, "ms_per_step": dt * 1e3}
+    if not args.no_multi:
+        line["multi_lambda"] = multi_lambda(H, r, p, bufs, flags, stream)
     if rank == 0 and not args.no_q1:
         line["q1_latency_us"] = q1_latency(H)
     if rank == 0 and not args.no_cpu:

@@ -213,6 +213,21 @@ hwr_status hwr_route_batch_slo(hwr_ctx *ctx, int32_t Q, const float *in_len,
                                float *pred_latency, float *utility);
 
 /*
+ * Score one batch without deciding: the cost predictor's C = TTFT + N_out *
+ * TPOT (Eq. 1-2) for every (query, deployment) pair and the quality score of
+ * every (query, model) pair (Sec. 3.2 (3)), under the current snapshot.
+ *   cost     [Q][D] row-major, or NULL;
+ *   quality  [Q][M] row-major, or NULL (not both NULL).
+ * Host or device memory per HWR_DEVICE_PTRS.  Values are those the routing
+ * calls compare: bit-identical to what a route of the same batch on the same
+ * path computes for each pair.  HWR_SCORE_CONVEX is ignored; HWR_SEQUENTIAL
+ * is UNSUPPORTED.  Errors: as hwr_route_batch.
+ */
+hwr_status hwr_score_batch(hwr_ctx *ctx, int32_t Q, const float *in_len,
+                           const float *out_len, const void *q_emb,
+                           uint32_t flags, float *cost, float *quality);
+
+/*
  * Route one batch for K values of lambda at once (1 <= K <= 16): the
  * predictor and the quality scores are evaluated once and the decision maker
  * of Eq. 3 is applied for every lambda -- the routing half of the paper's

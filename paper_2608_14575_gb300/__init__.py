@@ -8,6 +8,7 @@ from ._hwr import (HwrError, Router, load, lib_path, HWR_SEQUENTIAL,
                    HWR_PATH_TENSOR, HWR_PROFILE, HWR_F32, HWR_BF16, KERNELS,
                    hwr_create, hwr_update_snapshot, hwr_get_snapshot,
                    hwr_route_batch, hwr_route_batch_slo, hwr_slo_spec, hwr_route_batch_multi,
+                   hwr_score_batch,
                    hwr_route_batch_noalloc, HWR_NOALLOC_MAX_Q,
                    hwr_synchronize, hwr_destroy,
                    hwr_status_string, hwr_last_error, hwr_get_stats)

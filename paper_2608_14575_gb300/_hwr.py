@@ -35,7 +35,7 @@ HWR_K_COUNT = len(KERNELS)
 
 EXPORTS = ("hwr_create", "hwr_update_snapshot", "hwr_get_snapshot",
            "hwr_route_batch", "hwr_route_batch_slo", "hwr_route_batch_multi",
-           "hwr_route_batch_noalloc", "hwr_synchronize",
+           "hwr_score_batch", "hwr_route_batch_noalloc", "hwr_synchronize",
            "hwr_destroy", "hwr_status_string", "hwr_last_error", "hwr_get_stats")
 HWR_NOALLOC_MAX_Q = 32768
 
@@ -108,6 +108,7 @@ def load(path: str | None = None):
                                             ct.c_uint32, P, P, P]
         lib.hwr_route_batch_multi.argtypes = [P, ct.c_int32, P, P, P, ct.c_float, P,
                                               ct.c_int32, ct.c_uint32, P, P, P]
+        lib.hwr_score_batch.argtypes = [P, ct.c_int32, P, P, P, ct.c_uint32, P, P]
         lib.hwr_synchronize.argtypes = [P]
         lib.hwr_destroy.argtypes = [P]
         lib.hwr_status_string.argtypes = [I]
@@ -117,8 +118,8 @@ def load(path: str | None = None):
         lib.hwr_get_stats.argtypes = [P, P, I]
         for n in ("hwr_create", "hwr_update_snapshot", "hwr_get_snapshot",
                   "hwr_route_batch", "hwr_route_batch_slo", "hwr_route_batch_multi",
-                  "hwr_route_batch_noalloc", "hwr_synchronize", "hwr_destroy",
-                  "hwr_get_stats"):
+                  "hwr_score_batch", "hwr_route_batch_noalloc", "hwr_synchronize",
+                  "hwr_destroy", "hwr_get_stats"):
             getattr(lib, n).restype = I
         if path is None:
             _lib = lib
@@ -155,6 +156,10 @@ def hwr_route_batch_multi(ctx, Q, in_len, out_len, q_emb, slo, lambdas, K, flags
                           pred_latency, utility):
     return load().hwr_route_batch_multi(ctx, Q, in_len, out_len, q_emb, slo, lambdas, K, flags,
                                         chosen, pred_latency, utility)
+
+
+def hwr_score_batch(ctx, Q, in_len, out_len, q_emb, flags, cost, quality):
+    return load().hwr_score_batch(ctx, Q, in_len, out_len, q_emb, flags, cost, quality)
 
 
 def hwr_route_batch_noalloc(ctx, Q, in_len, out_len, q_emb, slo, lam, flags, chosen,
@@ -261,6 +266,28 @@ class Router:
             float(p["lam"] if lam is None else lam), int(flags) & ~HWR_DEVICE_PTRS,
             chosen.ctypes.data, lat.ctypes.data, util.ctypes.data))
         return chosen, lat, util
+
+    def score(self, in_len=None, out_len=None, emb=None, *, flags=0, quality=True):
+        """Cost [Q][D] and quality [Q][M] (None unless `quality`) of a host batch."""
+        p = self.p
+        il = _c(p["in_len"] if in_len is None else in_len, np.float32)
+        ol = _c(p["out_len"] if out_len is None else out_len, np.float32)
+        em = _c(p["emb"] if emb is None else emb, self.wdt)
+        Q = il.size
+        cost = np.empty((Q, p["D"]), np.float32)
+        qual = np.empty((Q, p["M"]), np.float32) if quality else None
+        self._check(self.lib.hwr_score_batch(
+            self.ctx, Q, il.ctypes.data, ol.ctypes.data, em.ctypes.data,
+            int(flags) & ~HWR_DEVICE_PTRS, cost.ctypes.data,
+            qual.ctypes.data if quality else None))
+        return cost, qual
+
+    def score_device(self, in_len, out_len, emb, cost, quality=None, *, flags=0):
+        """Device scoring into CUDA tensors cost [Q][D] and quality [Q][M]."""
+        self._check(self.lib.hwr_score_batch(
+            self.ctx, int(in_len.numel()), in_len.data_ptr(), out_len.data_ptr(),
+            emb.data_ptr(), int(flags) | HWR_DEVICE_PTRS, cost.data_ptr(),
+            None if quality is None else quality.data_ptr()))
 
     def route_multi(self, lambdas, in_len=None, out_len=None, emb=None, *, slo=None,
                     flags=0):

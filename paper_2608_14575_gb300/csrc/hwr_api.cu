@@ -657,10 +657,17 @@ static size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 // Shared body of hwr_route_batch and hwr_route_batch_slo.  `spec` (may be
 // NULL) replaces the scalar SLO by per-query budgets or the Eq. 4-5 model.
+// Score outputs of hwr_score_batch: cost [Q][D] and quality [Q][M] (either may be NULL).
+struct ScoreOut {
+    float *cost;
+    float *quality;
+};
+
 static hwr_status route_impl(hwr_ctx *c, int32_t Q, const float *in_len, const float *out_len,
                              const void *q_emb, float slo, const hwr_slo_spec *spec,
                              float lambda, uint32_t flags, int32_t *chosen,
-                             float *pred_latency, float *utility, const Lambdas *ml = nullptr) {
+                             float *pred_latency, float *utility, const Lambdas *ml = nullptr,
+                             const ScoreOut *so = nullptr) {
     if (!c) return fail(nullptr, HWR_ERR_INVALID_ARG, "ctx is NULL");
     if (c->broken) return HWR_ERR_STATE;
     const uint32_t known = HWR_SEQUENTIAL | HWR_DEVICE_PTRS | HWR_ASYNC | HWR_SCORE_CONVEX |
@@ -668,7 +675,7 @@ static hwr_status route_impl(hwr_ctx *c, int32_t Q, const float *in_len, const f
     if (flags & ~known) return fail(c, HWR_ERR_INVALID_ARG, "unknown flag bits 0x%x", flags & ~known);
     if (Q < 0) return fail(c, HWR_ERR_INVALID_ARG, "Q=%d < 0", Q);
     if (Q == 0) return HWR_OK;
-    if (!in_len || !out_len || !q_emb || !chosen || !pred_latency || !utility)
+    if (!in_len || !out_len || !q_emb || (!so && (!chosen || !pred_latency || !utility)))
         return fail(c, HWR_ERR_INVALID_ARG, "NULL input or output array");
     if (!spec && slo != slo) return fail(c, HWR_ERR_INVALID_ARG, "SLO is NaN");
     if (spec && !spec->budget &&
@@ -691,7 +698,8 @@ static hwr_status route_impl(hwr_ctx *c, int32_t Q, const float *in_len, const f
     const bool dev = flags & HWR_DEVICE_PTRS;
     const size_t es = c->dtype == HWR_BF16 ? 2 : 4;
     const int K = ml ? ml->K : 1;
-    if (ml && seq) return fail(c, HWR_ERR_UNSUPPORTED, "several lambdas with HWR_SEQUENTIAL");
+    if ((ml || so) && seq)
+        return fail(c, HWR_ERR_UNSUPPORTED, "HWR_SEQUENTIAL with several lambdas or scoring");
     if (dev && tensor && ((uintptr_t)q_emb & 15))
         return fail(c, HWR_ERR_INVALID_ARG, "device q_emb must be 16-byte aligned");
 
@@ -728,6 +736,12 @@ static hwr_status route_impl(hwr_ctx *c, int32_t Q, const float *in_len, const f
         q.in_len = in_len; q.out_len = out_len; q.emb = q_emb;
         q.chosen = chosen; q.lat = pred_latency; q.util = utility;
         if (budgets) q.slo_q = spec->budget;
+        if (so) {   // the kernels' own decisions go to scratch
+            TRY(grow(c, &c->out_d, &c->out_cap, out_total));
+            q.chosen = (int32_t *)c->out_d;
+            q.lat = (float *)(c->out_d + o_lat);
+            q.util = (float *)(c->out_d + o_util);
+        }
     } else {
         TRY(grow(c, &c->io_d, &c->io_cap, in_total));
         TRY(grow(c, &c->out_d, &c->out_cap, out_total));
@@ -760,29 +774,49 @@ static hwr_status route_impl(hwr_ctx *c, int32_t Q, const float *in_len, const f
     }
 
     const Model mv = model_view(c);
-    if (ml) {
-        TRY(grow(c, &c->mC, &c->mC_cap, (size_t)Q * c->D));
-        TRY(grow(c, &c->mQ, &c->mQ_cap, (size_t)Q * c->M));
+    // Stored scores: cost [Q][D] and quality [Q][M], for the selection over
+    // several lambdas or as the output of hwr_score_batch.
+    float *SC = nullptr, *SQ = nullptr;
+    if (ml || so) {
+        if (so && dev) {
+            SC = so->cost;
+            SQ = so->quality;
+        } else {
+            TRY(grow(c, &c->mC, &c->mC_cap, (size_t)Q * c->D));
+            TRY(grow(c, &c->mQ, &c->mQ_cap, (size_t)Q * c->M));
+            SC = c->mC;
+            SQ = c->mQ;
+        }
     }
+    const size_t rowC = (size_t)c->D * 4, rowQ = (size_t)c->M * 4;
     // One chunk [lo, lo + n): its kernels, then (several lambdas) the selection
     // for every lambda from the scores the kernels stored.
     auto run_chunk = [&](Queries qc, int lo) -> hwr_status {
-        const bool small = !tensor && (long)qc.Q * c->D <= c->pairs_max;
-        if (ml) {
-            qc.pair_C = c->mC;
-            qc.qual_out = c->mQ;
-        }
+        const int n = qc.Q;
+        const bool small = !tensor && (long)n * c->D <= c->pairs_max;
+        if (SC) qc.pair_C = SC + (size_t)lo * c->D;
+        if (SQ) qc.qual_out = SQ + (size_t)lo * c->M;
         TRY(run_kernels(c, qc, flags, tensor));
+        if (!SC && !SQ) return HWR_OK;
+        // paths that keep their scores in their own scratch: copy them over
+        if (small && SC)
+            CK(c, cudaMemcpyAsync(SC + (size_t)lo * c->D, c->pairC, n * rowC,
+                                  cudaMemcpyDeviceToDevice, c->stream), "copy costs");
+        if (small && SQ)
+            CK(c, cudaMemcpyAsync(SQ + (size_t)lo * c->M, c->pairQ, n * rowQ,
+                                  cudaMemcpyDeviceToDevice, c->stream), "copy quality");
+        if (tensor && SQ)
+            CK(c, cudaMemcpy2DAsync(SQ + (size_t)lo * c->M, rowQ, c->qual, (size_t)c->Mpad * 4,
+                                    rowQ, n, cudaMemcpyDeviceToDevice, c->stream),
+               "copy quality");
         if (!ml) return HWR_OK;
         Queries qs = qc;
         qs.chosen = q.chosen + lo;
         qs.lat = q.lat + lo;
         qs.util = q.util + lo;
-        const float *Cs = small ? c->pairC : c->mC;
-        const float *qual = tensor ? c->qual : (small ? c->pairQ : c->mQ);
-        const int qstride = tensor ? c->Mpad : c->M;
         LaunchScope ls(c, HWR_K_ROUTE_SIMT, flags & HWR_PROFILE);
-        CK(c, launch_select_multi(mv, qs, Cs, qual, qstride, *ml, Q, c->stream), "select kernel");
+        CK(c, launch_select_multi(mv, qs, SC + (size_t)lo * c->D, SQ + (size_t)lo * c->M, c->M,
+                                  *ml, Q, c->stream), "select kernel");
         ls.done();
         return HWR_OK;
     };
@@ -825,7 +859,14 @@ static hwr_status route_impl(hwr_ctx *c, int32_t Q, const float *in_len, const f
     }
 
     bool synced = false;
-    if (!dev) {
+    if (so && !dev) {
+        if (so->cost)
+            CK(c, cudaMemcpyAsync(so->cost, SC, (size_t)Q * rowC, cudaMemcpyDeviceToHost, c->stream),
+               "copy costs");
+        if (so->quality)
+            CK(c, cudaMemcpyAsync(so->quality, SQ, (size_t)Q * rowQ, cudaMemcpyDeviceToHost,
+                                  c->stream), "copy quality");
+    } else if (!dev) {
         if (packed) {
             CK(c, cudaMemcpyAsync(c->pin_h, c->out_d, out_total, cudaMemcpyDeviceToHost, c->stream),
                "copy outputs");
@@ -858,6 +899,16 @@ extern "C" hwr_status hwr_route_batch(hwr_ctx *c, int32_t Q, const float *in_len
                                       float *pred_latency, float *utility) {
     return route_impl(c, Q, in_len, out_len, q_emb, slo, nullptr, lambda, flags, chosen,
                       pred_latency, utility);
+}
+
+extern "C" hwr_status hwr_score_batch(hwr_ctx *c, int32_t Q, const float *in_len,
+                                      const float *out_len, const void *q_emb, uint32_t flags,
+                                      float *cost, float *quality) {
+    if (!c) return fail(nullptr, HWR_ERR_INVALID_ARG, "ctx is NULL");
+    if (!cost && !quality) return fail(c, HWR_ERR_INVALID_ARG, "cost and quality both NULL");
+    ScoreOut so{cost, quality};
+    return route_impl(c, Q, in_len, out_len, q_emb, INFINITY, nullptr, 0.0f,
+                      flags & ~HWR_SCORE_CONVEX, nullptr, nullptr, nullptr, nullptr, &so);
 }
 
 extern "C" hwr_status hwr_route_batch_multi(hwr_ctx *c, int32_t Q, const float *in_len,
