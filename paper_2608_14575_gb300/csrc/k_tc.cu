@@ -314,6 +314,16 @@ __device__ __forceinline__ Unit unit_of(int u, int ntiles, int nsplit, int D) {
     return x;
 }
 
+// 16-byte read-only load issued where it is written (volatile: not sunk to
+// its first use, so a prefetch stays a prefetch)
+__device__ __forceinline__ uint4 ldg_nc_v4(const uint4 *p) {
+    uint4 v;
+    asm volatile("ld.global.nc.v4.u32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "l"(p));
+    return v;
+}
+
 // bf16 pairs in 32-bit registers: relu(a * b + c), and float pair -> bf16 pair
 __device__ __forceinline__ uint32_t hfma2_relu(uint32_t a, uint32_t b, uint32_t c) {
     uint32_t d;
@@ -422,7 +432,8 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
                      wbytes - off < 16384 ? wbytes - off : 16384, wbar);
         bool ok = mbar_wait(wbar, 0, abort_f, status);
         const uint32_t idesc = idesc_bf16_f32(BM, H2);
-        uint32_t n = 0, g = 0;
+        uint32_t g = 0, ph = 0;
+        int s = 0;
         for (int u = blockIdx.x; ok && u < nunits; u += gridDim.x) {
             const Unit un = unit_of(u, ntiles, nsplit, D);
             for (int d = un.d0; d < un.d1; ++d, ++g) {
@@ -431,9 +442,8 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
                 if (!ok) break;
                 tc_fence_after();
                 const uint32_t dt = tmem + (uint32_t)b * H2;
-                for (int c = 0; c < nch; ++c, ++n) {
-                    const int s = n % NS;
-                    ok = mbar_wait(&full[s], (n / NS) & 1, abort_f, status);
+                for (int c = 0; c < nch; ++c) {
+                    ok = mbar_wait(&full[s], ph, abort_f, status);
                     if (!ok) break;
                     tc_fence_after();
                     const uint64_t ad = sdesc_sw128(smem_u32(ring + s * CHUNK_BYTES));
@@ -442,6 +452,10 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
                     for (int k = 0; k < 4; ++k)
                         mma_bf16(dt, ad + 2 * k, bd + 2 * k, idesc, (c | k) != 0);
                     mma_commit(&empty[s]);
+                    if (++s == NS) {
+                        s = 0;
+                        ph ^= 1;
+                    }
                 }
                 if (!ok) break;
                 mma_commit(&accf[b]);
@@ -584,7 +598,8 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
         }
         const uint32_t one2 = 0x3F803F80u;  // (1.0, 1.0) in bf16
         uint32_t Bq[4][4][4];
-        uint32_t n = 0;
+        uint32_t ph = 0;
+        int s = 0;
         bool ok = true;
         for (int u = blockIdx.x; ok && u < nunits; u += gridDim.x) {
             const Unit un = unit_of(u, ntiles, nsplit, D);
@@ -618,13 +633,12 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
                     const uint4 *An = (const uint4 *)(m.Abf + (size_t)(d + 1) * H1);
 #pragma unroll
                     for (int c = 0; c < 4; ++c)
-                        if (c < nch) an[c] = __ldg(An + c * 8 + gi);
+                        if (c < nch) an[c] = ldg_nc_v4(An + c * 8 + gi);
                 }
 #pragma unroll
                 for (int c = 0; c < 4; ++c) {
                     if (c < nch && ok) {
-                        const int s = n % NS;
-                        ok = mbar_wait(&empty[s], ((n / NS) & 1) ^ 1, abort_f, status);
+                        ok = mbar_wait(&empty[s], ph ^ 1, abort_f, status);
                         if (ok) {
                             const uint32_t st = smem_u32(ring + s * CHUNK_BYTES);
 #pragma unroll
@@ -640,7 +654,10 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
                             }
                             fence_proxy_async_smem();
                             if (!m.test_stall) mbar_arrive(&full[s]);
-                            ++n;
+                            if (++s == NS) {
+                                s = 0;
+                                ph ^= 1;
+                            }
                         }
                     }
                 }
