@@ -635,26 +635,43 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
                     for (int c = 0; c < 4; ++c)
                         if (c < nch) an[c] = ldg_nc_v4(An + c * 8 + gi);
                 }
+                // two chunks per round: one wait / fence / arrive cycle covers
+                // both, halving the serial latency each producer warp pays
 #pragma unroll
-                for (int c = 0; c < 4; ++c) {
+                for (int c = 0; c < 4; c += 2) {
                     if (c < nch && ok) {
+                        const bool two = c + 1 < nch;
+                        const int s1 = s + 1 == NS ? 0 : s + 1;
+                        const uint32_t ph1 = s + 1 == NS ? ph ^ 1 : ph;
                         ok = mbar_wait(&empty[s], ph ^ 1, abort_f, status);
+                        if (ok && two) ok = mbar_wait(&empty[s1], ph1 ^ 1, abort_f, status);
                         if (ok) {
-                            const uint32_t st = smem_u32(ring + s * CHUNK_BYTES);
 #pragma unroll
-                            for (int i = 0; i < 4; ++i) {
-                                const uint32_t h0 = hfma2_relu(Bq[i][c][0], one2, a[c].x);
-                                const uint32_t h1 = hfma2_relu(Bq[i][c][1], one2, a[c].y);
-                                const uint32_t h2 = hfma2_relu(Bq[i][c][2], one2, a[c].z);
-                                const uint32_t h3 = hfma2_relu(Bq[i][c][3], one2, a[c].w);
-                                asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(
-                                                 st + offs[i]),
-                                             "r"(h0), "r"(h1), "r"(h2), "r"(h3)
-                                             : "memory");
+                            for (int cc = 0; cc < 2; ++cc) {
+                                if (cc == 0 || two) {
+                                    const uint4 av = a[c + cc];
+                                    const uint32_t st = smem_u32(ring + (cc ? s1 : s) * CHUNK_BYTES);
+#pragma unroll
+                                    for (int i = 0; i < 4; ++i) {
+                                        const uint32_t h0 = hfma2_relu(Bq[i][c + cc][0], one2, av.x);
+                                        const uint32_t h1 = hfma2_relu(Bq[i][c + cc][1], one2, av.y);
+                                        const uint32_t h2 = hfma2_relu(Bq[i][c + cc][2], one2, av.z);
+                                        const uint32_t h3 = hfma2_relu(Bq[i][c + cc][3], one2, av.w);
+                                        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(
+                                                         st + offs[i]),
+                                                     "r"(h0), "r"(h1), "r"(h2), "r"(h3)
+                                                     : "memory");
+                                    }
+                                }
                             }
                             fence_proxy_async_smem();
-                            if (!m.test_stall) mbar_arrive(&full[s]);
-                            if (++s == NS) {
+                            if (!m.test_stall) {
+                                mbar_arrive(&full[s]);
+                                if (two) mbar_arrive(&full[s1]);
+                            }
+                            s = s1;
+                            ph = ph1;
+                            if (two && ++s == NS) {
                                 s = 0;
                                 ph ^= 1;
                             }
