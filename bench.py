@@ -20,7 +20,11 @@ Printed (one JSON line, rank 0):
             host buffers, at D = 32 (the batch-sweep shape);
   cpu_baseline   the CPU oracle on a bounded sample of the same workload;
   multi_lambda   one hwr_route_batch_multi call for 8 values of lambda on the
-            same batch (the Sec. 5 lambda sweep), next to 8 single routes.
+            same batch (the Sec. 5 lambda sweep), next to 8 single routes;
+  sweep_d32 the batch-size sweep at D = 32 (8 models x 4 GPU types, H = 256,
+            E = 1024): per Q in {1, 16, 256, 4096, 65536, 1048576}, p50 / p99
+            of per-call CUDA-event time with device pointers, queries/s at the
+            median, and the fraction of the bf16 tensor roofline.
 --impl reference times the CPU oracle (the reference arm for this build).
 --online prints the online evaluation metrics of Sec. 4.3 (SLO attainment,
 queue composition, load/running/waiting skew) for the online sequential
@@ -307,6 +311,50 @@ def online_report(args):
                 flush=True)
 
 
+def sweep_d32(H, stream, dev):
+    """Per-call latency and throughput over the batch sizes of the D = 32 sweep."""
+    import torch
+    base = W.make_config(4, Q=65_536)
+    Qmax = max(W.CONFIGS[4]["sweep"])
+    r = H.Router(base, stream=stream.cuda_stream)
+    il0 = torch.from_numpy(base["in_len"]).to(dev)
+    ol0 = torch.from_numpy(base["out_len"]).to(dev)
+    em0 = torch.from_numpy(base["emb"].view(np.int16)).to(dev)
+    reps = Qmax // base["Q"]
+    # the largest batch is the 65,536-query batch repeated (every query is still routed)
+    ilb, olb, emb = il0.repeat(reps), ol0.repeat(reps), em0.repeat(reps, 1)
+    ch = torch.empty(Qmax, dtype=torch.int32, device=dev)
+    lat = torch.empty(Qmax, dtype=torch.float32, device=dev)
+    ut = torch.empty(Qmax, dtype=torch.float32, device=dev)
+    torch.cuda.synchronize()
+    pk, _ = peaks()
+    fq = base["D"] * flops_per_pair(base) + 2 * base["E"] * base["M"]   # flop per query
+    out = []
+    for Q in W.CONFIGS[4]["sweep"]:
+        n = 200 if Q <= 4096 else (50 if Q <= 65_536 else 20)
+        args = (ilb[:Q], olb[:Q], emb[:Q], ch[:Q], lat[:Q], ut[:Q])
+        for _ in range(10):
+            r.route_device(*args, slo=base["slo"], lam=base["lam"])
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(n)]
+        for e0, e1 in ev:
+            e0.record(stream)
+            r.route_device(*args, slo=base["slo"], lam=base["lam"])
+            e1.record(stream)
+        torch.cuda.synchronize()
+        t = np.array([e0.elapsed_time(e1) for e0, e1 in ev]) * 1e3   # us
+        med = float(np.median(t))
+        qps = Q / (med * 1e-6)
+        out.append({"Q": Q, "calls": n, "p50_us": med, "p99_us": float(np.percentile(t, 99)),
+                    "queries_per_s": qps,
+                    "frac_of_tensor_roofline": qps * fq / (pk["bf16_tflops"] * 1e12)})
+    r.close()
+    return {"config": "D=32 (8 models x 4 GPU types), MLP 48->256->256->2, E=1024 bf16; "
+                      "per call, device pointers, CUDA events around each call; "
+                      f"Q={Qmax} is the 65,536-query batch repeated {reps}x",
+            "points": out}
+
+
 def multi_lambda(H, r, p, bufs, flags, stream, steps=10):
     """One 8-lambda call against 8 single-lambda calls on the same device batch."""
     import torch
@@ -359,6 +407,7 @@ def main():
     ap.add_argument("--no-q1", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
     ap.add_argument("--no-multi", action="store_true")
+    ap.add_argument("--no-sweep", action="store_true")
     ap.add_argument("--online", action="store_true",
                     help="print the online evaluation metrics instead of the throughput line")
     args = ap.parse_args()
@@ -503,15 +552,20 @@ def main():
                        "d2h_bytes_per_step": Q * 12, "ms_per_step": dt * 1e3}
     if not args.no_multi:
         line["multi_lambda"] = multi_lambda(H, r, p, bufs, flags, stream)
+    if rank == 0 and not args.no_sweep and p["dtype"] == "bf16":
+        line["sweep_d32"] = sweep_d32(H, stream, dev)
     if rank == 0 and not args.no_q1:
         line["q1_latency_us"] = q1_latency(H)
     if rank == 0 and not args.no_cpu:
         cores = len(os.sched_getaffinity(0))
         v, n, dt = cpu_oracle_rate(p, 10.0, cores)
+        v1, n1, dt1 = cpu_oracle_rate(p, 4.0, 1)
         line["cpu_baseline"] = {"value": v, "unit": "queries/s", "cores": cores,
                                 "kind": "oracle",
                                 "sample": f"first {n} queries of the workload, fp64 oracle, "
-                                          f"{cores} OpenMP threads, {dt:.1f} s"}
+                                          f"{cores} OpenMP threads, {dt:.1f} s",
+                                "single_thread": {"value": v1, "sample": f"first {n1} queries, "
+                                                                         f"1 thread, {dt1:.1f} s"}}
     r.close()
     if rank == 0:
         print(json.dumps(line), flush=True)
