@@ -172,6 +172,9 @@ k_qual_tc(const __grid_constant__ CUtensorMap tmap, TcModel m, int Q, float *qua
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int nch = m.Epad / KCH, ntiles = (Q + BM - 1) / BM, Mpad = m.Mpad;
     const uint32_t membytes = (uint32_t)Mpad * m.Epad * 2;
+    // the predictor kernel that follows may start now: only its epilogue reads
+    // this kernel's output, and it waits for this grid's completion first
+    grid_launch_dependents();
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < QUAL_STAGES; ++s) {
@@ -476,6 +479,9 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
         const int ncol = H2 / 32;
         uint32_t g = 0;
         bool ok = true;
+        // the quality matrix comes from the kernel before (a dependent launch
+        // may start this grid before that one has finished)
+        grid_dependency_wait();
         for (int u = blockIdx.x; ok && u < nunits; u += gridDim.x) {
             const Unit un = unit_of(u, ntiles, nsplit, D);
             const int row = un.tile * BM + r;
@@ -779,19 +785,29 @@ cudaError_t launch_mlp_tc(const TcModel &m, const Queries &q, const float *qual,
     const MlpLayout L = mlp_layout(m.H1, m.H2, m.Mpad, m.D);
     const HeadConsts &hc = *m.head;
     int4 *pt = (int4 *)part;
+    // programmatic dependent launch: the grid may start while the quality
+    // kernel before it on the stream finishes (its epilogue waits for it)
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.gridDim = dim3((unsigned)grid);
+    cfg.blockDim = dim3(MLP_THREADS);
+    cfg.dynamicSmemBytes = L.total;
+    cfg.stream = s;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
 #define HWR_MLP(H2T, NHT) \
-    k_mlp_tc<H2T, NHT><<<grid, MLP_THREADS, L.total, s>>>(m, q, hc, qual, nsplit, pt, count, status)
+    return cudaLaunchKernelEx(&cfg, k_mlp_tc<H2T, NHT>, m, q, hc, qual, nsplit, pt, count, status)
     if (m.NH == 3) {
         if (m.H2 == 256) HWR_MLP(256, 3);
-        else if (m.H2 == 128) HWR_MLP(128, 3);
-        else HWR_MLP(0, 3);
-    } else {
-        if (m.H2 == 256) HWR_MLP(256, 2);
-        else if (m.H2 == 128) HWR_MLP(128, 2);
-        else HWR_MLP(0, 2);
+        if (m.H2 == 128) HWR_MLP(128, 3);
+        HWR_MLP(0, 3);
     }
+    if (m.H2 == 256) HWR_MLP(256, 2);
+    if (m.H2 == 128) HWR_MLP(128, 2);
+    HWR_MLP(0, 2);
 #undef HWR_MLP
-    return cudaGetLastError();
 }
 
 size_t tc_head_consts_bytes() { return sizeof(HeadConsts); }
