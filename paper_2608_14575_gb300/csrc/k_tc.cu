@@ -100,8 +100,10 @@ __host__ __device__ inline QualLayout qual_layout(int Mpad, int Epad) {
     return L;
 }
 
+constexpr int APRE_SLOTS = 4;   // deployment-prefix ring (layer-1 A_d rows)
+
 struct MlpLayout {
-    uint32_t w2, ring, qual, consts, bars, misc, total;
+    uint32_t w2, ring, qual, consts, apre, bars, misc, total;
     int ns;
 };
 
@@ -109,8 +111,9 @@ __host__ __device__ inline MlpLayout mlp_layout(int H1, int H2, int Mpad, int D)
     MlpLayout L;
     uint32_t fixed = (uint32_t)H1 * H2 * 2                  // W2 image
                      + BM * (Mpad + 1) * 4                  // quality rows
-                     + (4 * H2 + 4) * 4 + D * 4             // b2, W3 (<= 3 rows), b3, dep_model
-                     + (2 * MLP_MAX_STAGES + 6) * 8 + 16    // barriers, misc
+                     + (4 * H2 + 4) * 4 + D * 4 + 16        // b2, W3 (<= 3 rows), b3, dep_model
+                     + APRE_SLOTS * H1 * 2                  // deployment-prefix ring
+                     + (2 * MLP_MAX_STAGES + 6 + 2 * APRE_SLOTS) * 8 + 16   // barriers, misc
                      + 1024 + 1024;                         // alignment slack
     int ns = (int)((SMEM_LIMIT - fixed) / CHUNK_BYTES);
     L.ns = ns > MLP_MAX_STAGES ? MLP_MAX_STAGES : ns;
@@ -124,9 +127,11 @@ __host__ __device__ inline MlpLayout mlp_layout(int H1, int H2, int Mpad, int D)
     o += BM * (Mpad + 1) * 4;
     L.consts = o;
     o += (4 * H2 + 4) * 4 + D * 4;
-    o = (o + 7) & ~7u;
+    o = (o + 15) & ~15u;
+    L.apre = o;
+    o += APRE_SLOTS * H1 * 2;
     L.bars = o;
-    o += (2 * MLP_MAX_STAGES + 6) * 8;
+    o += (2 * MLP_MAX_STAGES + 6 + 2 * APRE_SLOTS) * 8;
     L.misc = o;
     o += 16;
     L.total = o + 1024;
@@ -317,16 +322,6 @@ __device__ __forceinline__ Unit unit_of(int u, int ntiles, int nsplit, int D) {
     return x;
 }
 
-// 16-byte read-only load issued where it is written (volatile: not sunk to
-// its first use, so a prefetch stays a prefetch)
-__device__ __forceinline__ uint4 ldg_nc_v4(const uint4 *p) {
-    uint4 v;
-    asm volatile("ld.global.nc.v4.u32 {%0, %1, %2, %3}, [%4];"
-                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
-                 : "l"(p));
-    return v;
-}
-
 // bf16 pairs in 32-bit registers: relu(a * b + c), and float pair -> bf16 pair
 __device__ __forceinline__ uint32_t hfma2_relu(uint32_t a, uint32_t b, uint32_t c) {
     uint32_t d;
@@ -388,6 +383,8 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
     int *dms = (int *)(b3s + 4);
     uint64_t *full = (uint64_t *)(sm + L.bars), *empty = full + MLP_MAX_STAGES;
     uint64_t *accf = empty + MLP_MAX_STAGES, *acce = accf + 2, *wbar = acce + 2, *dbar = wbar + 1;
+    uint64_t *afull = dbar + 1, *afree = afull + APRE_SLOTS;   // prefix ring
+    uint8_t *apre = sm + L.apre;
     uint32_t *tslot = (uint32_t *)(sm + L.misc);
     volatile int *abort_f = (volatile int *)(tslot + 1);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -406,6 +403,10 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
         }
         mbar_init(wbar, 1);
         mbar_init(dbar, 1);
+        for (int j = 0; j < APRE_SLOTS; ++j) {
+            mbar_init(&afull[j], 1);
+            mbar_init(&afree[j], MLP_PRODUCERS);
+        }
         *abort_f = 0;
         fence_mbar_init();
     }
@@ -607,6 +608,34 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
         uint32_t ph = 0;
         int s = 0;
         bool ok = true;
+        // Deployment prefixes A_d come through a 4-slot shared-memory ring:
+        // producer 0 copies the prefix of the deployment two ahead (bulk
+        // copy, completion on afull), every producer frees a slot (afree)
+        // once it has read its granules.  dn counts this CTA's deployments.
+        const uint32_t abytes = (uint32_t)H1 * 2;
+        uint32_t dn = 0, issued = 0;
+        int cu = blockIdx.x, cd = 0;   // issue cursor: unit, deployment
+        Unit cun = cu < nunits ? unit_of(cu, ntiles, nsplit, D) : Unit{0, 0, 0, 0};
+        cd = cun.d0;
+        auto issue_until = [&](uint32_t target) {
+            while (ok && issued <= target && cu < nunits) {
+                const int j = issued & (APRE_SLOTS - 1);
+                if (issued >= APRE_SLOTS)
+                    ok = mbar_wait(&afree[j], ((issued / APRE_SLOTS) & 1) ^ 1, abort_f, status);
+                if (!ok) break;
+                mbar_arrive_expect_tx(&afull[j], abytes);
+                bulk_g2s(apre + j * abytes, (const uint8_t *)m.Abf + (size_t)cd * abytes, abytes,
+                         &afull[j]);
+                ++issued;
+                if (++cd == cun.d1) {
+                    cu += gridDim.x;
+                    if (cu < nunits) {
+                        cun = unit_of(cu, ntiles, nsplit, D);
+                        cd = cun.d0;
+                    }
+                }
+            }
+        };
         for (int u = blockIdx.x; ok && u < nunits; u += gridDim.x) {
             const Unit un = unit_of(u, ntiles, nsplit, D);
 #pragma unroll
@@ -629,18 +658,17 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
                     }
                 }
             }
-            uint4 a[4], an[4];
+            uint4 a[4];
+            for (int d = un.d0; ok && d < un.d1; ++d, ++dn) {
+                if (p == 0) issue_until(dn + 2);
+                const int j = dn & (APRE_SLOTS - 1);
+                ok = ok && mbar_wait(&afull[j], (dn / APRE_SLOTS) & 1, abort_f, status);
+                if (!ok) break;
+                const uint4 *As = (const uint4 *)(apre + j * abytes);
 #pragma unroll
-            for (int c = 0; c < 4; ++c)
-                if (c < nch) a[c] = __ldg((const uint4 *)(m.Abf + (size_t)un.d0 * H1) + c * 8 + gi);
-            for (int d = un.d0; ok && d < un.d1; ++d) {
-                // prefetch the next deployment's prefix while this one is built
-                if (d + 1 < un.d1) {
-                    const uint4 *An = (const uint4 *)(m.Abf + (size_t)(d + 1) * H1);
-#pragma unroll
-                    for (int c = 0; c < 4; ++c)
-                        if (c < nch) an[c] = ldg_nc_v4(An + c * 8 + gi);
-                }
+                for (int c = 0; c < 4; ++c)
+                    if (c < nch) a[c] = As[c * 8 + gi];
+                mbar_arrive(&afree[j]);
                 // two chunks per round: one wait / fence / arrive cycle covers
                 // both, halving the serial latency each producer warp pays
 #pragma unroll
@@ -684,10 +712,12 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
                         }
                     }
                 }
-#pragma unroll
-                for (int c = 0; c < 4; ++c) a[c] = an[c];
             }
         }
+        // copies still in flight must land before the CTA can exit
+        if (p == 0)
+            for (uint32_t k = dn; k < issued; ++k)
+                drain_wait(&afull[k & (APRE_SLOTS - 1)], (k / APRE_SLOTS) & 1);
     }
     tc_fence_before();
     __syncthreads();
