@@ -41,7 +41,7 @@ constexpr int KCH = 64;                         // bf16 K elements per 128-byte 
 constexpr uint32_t CHUNK_BYTES = BM * KCH * 2;  // one A chunk: 16 KB
 constexpr int QUAL_THREADS = 192;               // w0 TMA, w1 MMA, w2-5 epilogue
 constexpr int QUAL_STAGES = 8;
-constexpr int MLP_THREADS = 416;                // w0 MMA, w1-4 epilogue, w5-12 producers
+constexpr int MLP_THREADS = 448;                // w0 MMA, w1-4 epilogue, w5-12 producers, w13 prefix loader
 constexpr int MLP_PRODUCERS = 256;
 constexpr int MLP_MAX_STAGES = 8;
 constexpr uint32_t SMEM_LIMIT = 227 * 1024;
@@ -588,7 +588,7 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
                 count[row] = 0;
             }
         }
-    } else if (warp >= 5) {
+    } else if (warp >= 5 && warp < 13) {
         // ---- producers: layer-1 activations as bf16 UMMA operand tiles ------
         // Thread p owns granule gi = p % 8 (8 consecutive K) of every 64-wide K
         // chunk, for rows rb + 32 i (i < 4).  The query part of layer 1,
@@ -608,34 +608,11 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
         uint32_t ph = 0;
         int s = 0;
         bool ok = true;
-        // Deployment prefixes A_d come through a 4-slot shared-memory ring:
-        // producer 0 copies the prefix of the deployment two ahead (bulk
-        // copy, completion on afull), every producer frees a slot (afree)
-        // once it has read its granules.  dn counts this CTA's deployments.
+        // Deployment prefixes A_d come through the 4-slot shared-memory ring
+        // the loader warp fills; each producer frees a slot (afree) once it has
+        // read its granules.  dn counts this CTA's deployments.
         const uint32_t abytes = (uint32_t)H1 * 2;
-        uint32_t dn = 0, issued = 0;
-        int cu = blockIdx.x, cd = 0;   // issue cursor: unit, deployment
-        Unit cun = cu < nunits ? unit_of(cu, ntiles, nsplit, D) : Unit{0, 0, 0, 0};
-        cd = cun.d0;
-        auto issue_until = [&](uint32_t target) {
-            while (ok && issued <= target && cu < nunits) {
-                const int j = issued & (APRE_SLOTS - 1);
-                if (issued >= APRE_SLOTS)
-                    ok = mbar_wait(&afree[j], ((issued / APRE_SLOTS) & 1) ^ 1, abort_f, status);
-                if (!ok) break;
-                mbar_arrive_expect_tx(&afull[j], abytes);
-                bulk_g2s(apre + j * abytes, (const uint8_t *)m.Abf + (size_t)cd * abytes, abytes,
-                         &afull[j]);
-                ++issued;
-                if (++cd == cun.d1) {
-                    cu += gridDim.x;
-                    if (cu < nunits) {
-                        cun = unit_of(cu, ntiles, nsplit, D);
-                        cd = cun.d0;
-                    }
-                }
-            }
-        };
+        uint32_t dn = 0;
         for (int u = blockIdx.x; ok && u < nunits; u += gridDim.x) {
             const Unit un = unit_of(u, ntiles, nsplit, D);
 #pragma unroll
@@ -660,7 +637,6 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
             }
             uint4 a[4];
             for (int d = un.d0; ok && d < un.d1; ++d, ++dn) {
-                if (p == 0) issue_until(dn + 2);
                 const int j = dn & (APRE_SLOTS - 1);
                 ok = ok && mbar_wait(&afull[j], (dn / APRE_SLOTS) & 1, abort_f, status);
                 if (!ok) break;
@@ -714,10 +690,29 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
                 }
             }
         }
-        // copies still in flight must land before the CTA can exit
-        if (p == 0)
-            for (uint32_t k = dn; k < issued; ++k)
-                drain_wait(&afull[k & (APRE_SLOTS - 1)], (k / APRE_SLOTS) & 1);
+    } else if (warp == 13 && lane == 0) {
+        // ---- prefix loader: the layer-1 deployment prefix of every step of
+        // this CTA's units, in order, into the 4-slot ring (bulk copies,
+        // completion on afull; a slot is reused once afree says all producers
+        // have read it) ------------------------------------------------------
+        const uint32_t abytes = (uint32_t)H1 * 2;
+        uint32_t issued = 0;
+        bool ok = true;
+        for (int u = blockIdx.x; ok && u < nunits; u += gridDim.x) {
+            const Unit un = unit_of(u, ntiles, nsplit, D);
+            for (int d = un.d0; d < un.d1; ++d, ++issued) {
+                const int j = issued & (APRE_SLOTS - 1);
+                if (issued >= APRE_SLOTS)
+                    ok = mbar_wait(&afree[j], ((issued / APRE_SLOTS) & 1) ^ 1, abort_f, status);
+                if (!ok) break;
+                mbar_arrive_expect_tx(&afull[j], abytes);
+                bulk_g2s(apre + j * abytes, (const uint8_t *)m.Abf + (size_t)d * abytes, abytes,
+                         &afull[j]);
+            }
+        }
+        // the last copies may still be in flight: they land before the CTA exits
+        for (uint32_t k = issued > APRE_SLOTS ? issued - APRE_SLOTS : 0; k < issued; ++k)
+            drain_wait(&afull[k & (APRE_SLOTS - 1)], (k / APRE_SLOTS) & 1);
     }
     tc_fence_before();
     __syncthreads();
