@@ -610,7 +610,7 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
         bool ok = true;
         // Deployment prefixes A_d come through the 4-slot shared-memory ring
         // the loader warp fills; each producer frees a slot (afree) once it has
-        // read its granules.  dn counts this CTA's deployments.
+        // built every chunk from its granules.  dn counts this CTA's deployments.
         const uint32_t abytes = (uint32_t)H1 * 2;
         uint32_t dn = 0;
         for (int u = blockIdx.x; ok && u < nunits; u += gridDim.x) {
@@ -644,7 +644,6 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
 #pragma unroll
                 for (int c = 0; c < 4; ++c)
                     if (c < nch) a[c] = As[c * 8 + gi];
-                mbar_arrive(&afree[j]);
                 // two chunks per round: one wait / fence / arrive cycle covers
                 // both, halving the serial latency each producer warp pays
 #pragma unroll
@@ -688,6 +687,10 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
                         }
                     }
                 }
+                // the slot is freed only after the chunks above have used every
+                // granule read from it, so those shared-memory reads are complete
+                // before the loader's next bulk copy can overwrite it
+                mbar_arrive(&afree[j]);
             }
         }
     } else if (warp == 13 && lane == 0) {
