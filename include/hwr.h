@@ -301,7 +301,7 @@ const char *hwr_last_error(const hwr_ctx *ctx);
 enum {
     HWR_K_SNAPSHOT = 0, /* deployment features + first-layer prefix */
     HWR_K_ROUTE_SIMT,   /* fused fp32 gather -> MLP -> mask -> argmax */
-    HWR_K_SEQ_TABLE,    /* sequential mode: score table + serial chain */
+    HWR_K_SEQ_TABLE,    /* sequential mode: feature prep + score table + serial chain */
     HWR_K_QUAL_TC,      /* bf16 quality contraction, TMA + tcgen05 */
     HWR_K_MLP_TC,       /* bf16 predictor + mask + argmax, tcgen05 */
     HWR_K_COUNT

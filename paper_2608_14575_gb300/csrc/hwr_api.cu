@@ -30,11 +30,14 @@ struct AllocHook {
     long fail_at = 0, count = 0;
 };
 
-// Path thresholds, from a sweep of batch sizes on GB300 (defaults;
+// Path thresholds, from sweeps of batch sizes on GB300 (defaults;
 // HWR_TC_MIN_PAIRS and HWR_PAIRS_MAX_PAIRS override them at hwr_create):
 // batches of at most pairs_max pairs (Q * D) take the small-batch SIMT
 // kernel; larger bf16 batches of at least tc_min_pairs pairs take the
-// tensor-core kernels; the rest the fused SIMT kernel.
+// tensor-core kernels; the rest the fused SIMT kernel.  pairs_max is
+// SMALL_MAX_PAIRS where the tensor-core path exists and PAIRS_MAX_PAIRS
+// (the small-batch kernel's limit) otherwise: without tensor cores the
+// small-batch kernel stays ahead of the fused one up to that limit.
 constexpr int TC_MIN_PAIRS = 513;
 constexpr int PIPE_CHUNK_MIN = 8192;   // smallest chunk of a pipelined host batch
 constexpr int SMALL_MAX_PAIRS = 512;
@@ -51,7 +54,7 @@ struct hwr_ctx {
     bool broken = false;
     bool have_snapshot = false;
     int test_stall = 0;          // HWR_TEST_STALL: tensor-path producers never signal
-    int tc_min_pairs = TC_MIN_PAIRS, pairs_max = SMALL_MAX_PAIRS;
+    int tc_min_pairs = TC_MIN_PAIRS, pairs_max = -1;   // -1: by the context's paths
     std::string err;
     AllocHook hook;
     std::vector<void *> allocs;  // device buffers (cudaMalloc)
@@ -401,12 +404,14 @@ static hwr_status build_ctx(hwr_ctx *c, const hwr_deployment_table *t, const hwr
     TRY(dev_alloc(c, &c->pairC, (size_t)PAIRS_MAX_PAIRS));
     TRY(dev_alloc(c, &c->pairQ, (size_t)PAIRS_MAX_PAIRS * M));
     TRY(dev_alloc(c, &c->pairN, (size_t)PAIRS_MAX_PAIRS));
-    TRY(dev_alloc(c, &c->running, D));
-    TRY(dev_alloc(c, &c->waiting, D));
-    TRY(dev_alloc(c, &c->kv, D));
-    TRY(dev_alloc(c, &c->gpu_util, D));
-    TRY(dev_alloc(c, &c->ttft, D));
-    TRY(dev_alloc(c, &c->tpot, D));
+    // the six snapshot arrays, contiguous: an upload lands in them directly
+    TRY(dev_alloc(c, (char **)&c->snap_d, 6 * (size_t)D * 4));
+    c->running = (int32_t *)c->snap_d;
+    c->waiting = c->running + D;
+    c->kv = (float *)(c->waiting + D);
+    c->gpu_util = c->kv + D;
+    c->ttft = c->gpu_util + D;
+    c->tpot = c->ttft + D;
     TRY(dev_alloc(c, &c->X, (size_t)D * F));
     TRY(dev_alloc(c, &c->Spre, (size_t)D * H1));
     TRY(dev_alloc(c, &c->A, (size_t)D * H1));
@@ -473,7 +478,6 @@ static hwr_status build_ctx(hwr_ctx *c, const hwr_deployment_table *t, const hwr
     // snapshot staging: 6 arrays of D 4-byte values
     if (hook_fires(c)) return fail(c, HWR_ERR_OOM, "allocation %ld failed (test hook)", c->hook.count);
     CK(c, cudaHostAlloc(&c->snap_h, 6 * (size_t)D * 4, cudaHostAllocDefault), "alloc snapshot staging");
-    TRY(dev_alloc(c, (char **)&c->snap_d, 6 * (size_t)D * 4));
     CK(c, cudaEventCreateWithFlags(&c->snap_ev, cudaEventDisableTiming), "create event");
     CK(c, cudaEventCreateWithFlags(&c->pin_ev, cudaEventDisableTiming), "create event");
     CK(c, cudaStreamCreateWithFlags(&c->copy_stream, cudaStreamNonBlocking), "create copy stream");
@@ -538,6 +542,7 @@ extern "C" hwr_status hwr_create(const hwr_deployment_table *table, const hwr_pr
         free_ctx(c);
         return s;
     }
+    if (c->pairs_max < 0) c->pairs_max = c->tc_ok ? SMALL_MAX_PAIRS : PAIRS_MAX_PAIRS;
     *out = c;
     return HWR_OK;
 }
@@ -566,15 +571,9 @@ extern "C" hwr_status hwr_update_snapshot(hwr_ctx *c, const hwr_snapshot *s) {
     memcpy(h + 3 * n, s->gpu_util, n);
     memcpy(h + 4 * n, s->ttft_avg, n);
     memcpy(h + 5 * n, s->tpot_avg, n);
+    // one copy straight into the six device arrays (snap_d holds them back to back)
     CK(c, cudaMemcpyAsync(c->snap_d, h, 6 * n, cudaMemcpyHostToDevice, c->stream), "copy snapshot");
     CK(c, cudaEventRecord(c->snap_ev, c->stream), "record");
-    const char *d = (const char *)c->snap_d;
-    CK(c, cudaMemcpyAsync(c->running, d + 0 * n, n, cudaMemcpyDeviceToDevice, c->stream), "snapshot");
-    CK(c, cudaMemcpyAsync(c->waiting, d + 1 * n, n, cudaMemcpyDeviceToDevice, c->stream), "snapshot");
-    CK(c, cudaMemcpyAsync(c->kv, d + 2 * n, n, cudaMemcpyDeviceToDevice, c->stream), "snapshot");
-    CK(c, cudaMemcpyAsync(c->gpu_util, d + 3 * n, n, cudaMemcpyDeviceToDevice, c->stream), "snapshot");
-    CK(c, cudaMemcpyAsync(c->ttft, d + 4 * n, n, cudaMemcpyDeviceToDevice, c->stream), "snapshot");
-    CK(c, cudaMemcpyAsync(c->tpot, d + 5 * n, n, cudaMemcpyDeviceToDevice, c->stream), "snapshot");
     LaunchScope ls(c, HWR_K_SNAPSHOT, false);
     CK(c, launch_snapshot(model_view(c), c->stream), "snapshot kernel");
     ls.done();
@@ -601,7 +600,7 @@ static hwr_status run_kernels(hwr_ctx *c, const Queries &q, uint32_t flags, bool
     if (flags & HWR_SEQUENTIAL) {
         const int Qs = c->seq_qs;
         TRY(grow(c, &c->ctab, &c->ctab_cap, seq_table_floats(c->D, Qs)));
-        TRY(grow(c, &c->qseq, &c->qseq_cap, (size_t)Qs * c->M));
+        TRY(grow(c, &c->qseq, &c->qseq_cap, seq_aux_floats(c->D, c->M, Qs)));
         const size_t es = c->dtype == HWR_BF16 ? 2 : 4;
         for (int lo = 0; lo < q.Q; lo += Qs) {
             Queries k = q;
@@ -618,8 +617,9 @@ static hwr_status run_kernels(hwr_ctx *c, const Queries &q, uint32_t flags, bool
             CK(c, launch_seq_table(m, k, n, c->ctab, c->qseq, c->stream), "sequential table");
             a.done();
             CK(c, launch_seq_chain(m, k, n, c->ctab, c->qseq, c->stream), "sequential chain");
-            c->stats.kernel_launches++;
-            c->stats.launches[HWR_K_SEQ_TABLE]++;
+            // the preparation kernel (inside launch_seq_table) and the chain
+            c->stats.kernel_launches += 2;
+            c->stats.launches[HWR_K_SEQ_TABLE] += 2;
         }
         return HWR_OK;
     }
@@ -727,7 +727,10 @@ static hwr_status route_impl(hwr_ctx *c, int32_t Q, const float *in_len, const f
     const size_t out_total = o_util + outs_b;
     const bool packed = !dev && !(flags & HWR_ASYNC) && in_total <= ((size_t)1 << 20);
     // Large host batches: copy in chunks on the copy stream while the kernels
-    // of the previous chunk run (the link, not the GPU, bounds this path).
+    // of the previous chunk run (the link, not the GPU, bounds this path).  At
+    // most eight chunks: on GB300, 4, 6, 12 and 16 chunks of a 65,536-query
+    // batch were all slower end to end than 8 (fewer leave a longer compute
+    // tail after the last copy, more add per-chunk launch and copy overhead).
     const int nchunk = (!dev && !packed && !seq && Q >= 2 * PIPE_CHUNK_MIN)
                            ? (Q / PIPE_CHUNK_MIN < 8 ? Q / PIPE_CHUNK_MIN : 8) : 1;
     const bool pipelined = nchunk > 1;
@@ -827,20 +830,21 @@ static hwr_status route_impl(hwr_ctx *c, int32_t Q, const float *in_len, const f
         CK(c, cudaEventRecord(c->io_free_ev, c->stream), "record");
         CK(c, cudaStreamWaitEvent(c->copy_stream, c->io_free_ev, 0), "order copies");
         const int per = ((Q + nchunk - 1) / nchunk + 127) / 128 * 128;
+        // the lengths (and budgets) of the whole batch in one copy each, ahead
+        // of the embedding chunks: small copies per chunk cost more than they move
+        CK(c, cudaMemcpyAsync(c->io_d + off_in, in_len, len_b, cudaMemcpyHostToDevice,
+                              c->copy_stream), "copy in_len");
+        CK(c, cudaMemcpyAsync(c->io_d + off_out, out_len, len_b, cudaMemcpyHostToDevice,
+                              c->copy_stream), "copy out_len");
+        if (budgets)
+            CK(c, cudaMemcpyAsync(c->io_d + off_slo, spec->budget, len_b, cudaMemcpyHostToDevice,
+                                  c->copy_stream), "copy budgets");
         int k = 0;
         for (int lo = 0; lo < Q; lo += per, ++k) {
             const int n = Q - lo < per ? Q - lo : per;
             const size_t eo = (size_t)lo * c->E * es, eb = (size_t)n * c->E * es;
             CK(c, cudaMemcpyAsync(c->io_d + eo, (const char *)q_emb + eo, eb, cudaMemcpyHostToDevice,
                                   c->copy_stream), "copy emb");
-            CK(c, cudaMemcpyAsync(c->io_d + off_in + (size_t)lo * 4, in_len + lo, (size_t)n * 4,
-                                  cudaMemcpyHostToDevice, c->copy_stream), "copy in_len");
-            CK(c, cudaMemcpyAsync(c->io_d + off_out + (size_t)lo * 4, out_len + lo, (size_t)n * 4,
-                                  cudaMemcpyHostToDevice, c->copy_stream), "copy out_len");
-            if (budgets)
-                CK(c, cudaMemcpyAsync(c->io_d + off_slo + (size_t)lo * 4, spec->budget + lo,
-                                      (size_t)n * 4, cudaMemcpyHostToDevice, c->copy_stream),
-                   "copy budgets");
             CK(c, cudaEventRecord(c->chunk_ev[k], c->copy_stream), "record");
             CK(c, cudaStreamWaitEvent(c->stream, c->chunk_ev[k], 0), "order kernels");
             Queries qc = q;

@@ -96,13 +96,16 @@ constexpr int PAIRS_MAX_PAIRS = 2048;   // default upper bound on Q * D for this
 cudaError_t launch_route_pairs(const Model &m, const Queries &q, const float *W2T, float *pairC,
                                float *qualS, int32_t *count, cudaStream_t s);
 size_t route_pairs_smem(const Model &m);
-// Sequential mode over one chunk of Qs <= seq_chunk(m) queries: the score
-// table (every (picks c, deployment d, query i >= c)), then the serial chain.
-//   ctab: scratch of seq_table_floats(D, Qs) floats; qual: Qs * M floats.
+// Sequential mode over one chunk of Qs <= seq_chunk(m) queries: the chunk's
+// standardised features and the score table (every (picks c, deployment d,
+// query i >= c)) in launch_seq_table (two kernels), then the serial chain.
+//   ctab: scratch of seq_table_floats(D, Qs) floats;
+//   aux: scratch of seq_aux_floats(D, M, Qs) floats.
 cudaError_t launch_seq_table(const Model &m, const Queries &q, int Qs,
-                             float *ctab, float *qual, cudaStream_t s);
+                             float *ctab, float *aux, cudaStream_t s);
 cudaError_t launch_seq_chain(const Model &m, const Queries &q, int Qs,
-                             const float *ctab, const float *qual, cudaStream_t s);
+                             const float *ctab, float *aux, cudaStream_t s);
+size_t seq_aux_floats(int D, int M, int Qs);
 // Decision maker for K lambdas from stored scores: C [Q][D], quality
 // qual[q * qstride + model]; outputs [K][ostride] starting at query 0.
 cudaError_t launch_select_multi(const Model &m, const Queries &q, const float *C,

@@ -70,6 +70,41 @@ __device__ __forceinline__ float emb_at(const void *emb, int bf16, size_t i) {
     return ((const float *)emb)[i];
 }
 
+// Quality score (Sec. 3.2, hardware-independent term) of queries
+// [q0, q0 + nq): one serial chain per (query, model) from 0 with k ascending,
+// then the sigmoid.  The embedding rows and the model columns are staged
+// through `stage` (stage_floats >= 2 nq + M + 1) in chunks of the embedding
+// dimension; the chains read shared memory only.  Every thread of the block
+// calls this; thread t < nq * M returns the score of query t / M, model t % M
+// (rows at or past q.Q give sigmoid(0)), the others return 0.  Ends with the
+// stage free for reuse after a barrier.
+__device__ float quality_staged(const Model &m, const Queries &q, int q0, int nq, float *stage,
+                                int stage_floats) {
+    const int tid = threadIdx.x, M = m.M, E = m.E;
+    int ek = (stage_floats - nq) / (nq + M);
+    if (ek > E) ek = E;
+    const int ld = ek + 1;
+    float *er = stage, *mb = stage + (size_t)nq * ld;
+    const int qi = tid / M, mi = tid - qi * M;
+    float s = 0.f;
+    for (int k0 = 0; k0 < E; k0 += ek) {
+        const int kc = min(ek, E - k0);
+        __syncthreads();
+        for (int t = tid; t < nq * kc; t += SIMT_THREADS) {
+            const int i = t / kc, k = t - i * kc, qq = q0 + i;
+            er[i * ld + k] = qq < q.Q ? emb_at(q.emb, q.emb_bf16, (size_t)qq * E + k0 + k) : 0.f;
+        }
+        for (int t = tid; t < kc * M; t += SIMT_THREADS) mb[t] = m.memb[(size_t)k0 * M + t];
+        __syncthreads();
+        if (tid < nq * M) {
+            const float *a = er + qi * ld, *b = mb + mi;
+#pragma unroll 8
+            for (int k = 0; k < kc; ++k) s = __fmaf_rn(a[k], b[k * M], s);
+        }
+    }
+    return tid < nq * M ? sigmoid_c(s) : 0.f;
+}
+
 // ---------------------------------------------------------------------------
 // K_snap: standardised deployment features and the deployment prefix of
 // layer 1 (the part of W1 x + b1 that does not depend on the query).
@@ -105,7 +140,8 @@ __global__ void __launch_bounds__(SIMT_THREADS) k_snapshot(Model m) {
 //
 // Thread map: warp w owns rows w + 8 i (i < RPT); lane l owns columns
 // l + 32 j (j < CPT).  Shared memory: h1 [8 RPT][KC + 1] and W2 chunk
-// [KC][H2 + 1] during the K loop, then h2 [8 RPT][H2 + 1] in the same space.
+// [KC][H2 + 1] during the K loop, then h2 [8 RPT][H2 + 1] in the same space;
+// W3 [NH][H2] staged in w3s for the head chains.
 
 template <int RPT>
 __host__ __device__ constexpr size_t tile_floats_for(int H2) {
@@ -117,13 +153,15 @@ __host__ __device__ constexpr size_t tile_floats_for(int H2) {
 
 template <int RPT, int CPT, class Rows>
 __device__ void pair_mlp(const Model &m, int R, const Rows &rows, const float *us,
-                         const float *vs, float *tile, float *sp) {
+                         const float *vs, float *tile, float *w3s, float *sp) {
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int H1 = m.H1, H2 = m.H2, F = m.F;
     float *h1s = tile;
     float *w2s = tile + 8 * RPT * (SIMT_KC + 1);
     const int w2ld = H2 + 1;
 
+    // W3 for the head chains (visible after the first barrier of the K loop)
+    for (int i = tid; i < m.NH * H2; i += SIMT_THREADS) w3s[i] = m.W3[i];
     float acc[RPT][CPT];
 #pragma unroll
     for (int j = 0; j < CPT; ++j) {
@@ -185,7 +223,7 @@ __device__ void pair_mlp(const Model &m, int R, const Rows &rows, const float *u
     __syncthreads();
     for (int e = tid; e < m.NH * R; e += SIMT_THREADS) {
         const int r = e / m.NH, o = e - r * m.NH;
-        const float *w3 = m.W3 + (size_t)o * H2;
+        const float *w3 = w3s + (size_t)o * H2;
         float z = m.b3[o];
         for (int n = 0; n < H2; ++n) z = __fmaf_rn(w3[n], h2s[r * w2ld + n], z);
         sp[e] = softplus_c(z);
@@ -207,7 +245,7 @@ __host__ __device__ inline int route_qb(int D) { return D >= 64 ? 1 : 64 / D; }
 
 struct RouteLayout {
     int QB, R;
-    size_t us, vs, ol, qual, sp, C, U, tile, total;  // float offsets
+    size_t us, vs, ol, qual, sp, C, U, w3, tile, total;  // float offsets
 };
 
 __host__ __device__ inline RouteLayout route_layout(int D, int M, int H2) {
@@ -222,6 +260,7 @@ __host__ __device__ inline RouteLayout route_layout(int D, int M, int H2) {
     L.sp = o; o += 3 * 64;
     L.C = o; o += 64;
     L.U = o; o += 64;
+    L.w3 = o; o += 3 * (size_t)H2;
     o = (o + 3) & ~(size_t)3;
     L.tile = o;
     o += tile_floats_for<ROUTE_RPT>(H2);
@@ -251,21 +290,14 @@ __global__ void __launch_bounds__(SIMT_THREADS) k_route_simt(Model m, Queries q)
         vs[qi] = v;
         ol[qi] = o;
     }
-    // quality: one serial chain per (query, model), from 0, k ascending
-    for (int e = tid; e < QB * M; e += SIMT_THREADS) {
-        const int qi = e / M, mi = e - qi * M, qq = q0 + qi;
-        float s = 0.f;
-        if (qq < q.Q) {
-            const size_t row = (size_t)qq * m.E;
-            for (int k = 0; k < m.E; ++k)
-                s = __fmaf_rn(emb_at(q.emb, q.emb_bf16, row + k), m.memb[(size_t)k * M + mi], s);
-        }
-        qual[e] = sigmoid_c(s);
-    }
+    // quality, staged through the (not yet used) tile space
+    const float qv = quality_staged(m, q, q0, QB, sm + L.tile,
+                                    (int)tile_floats_for<ROUTE_RPT>(m.H2));
+    if (tid < QB * M) qual[tid] = qv;
     __syncthreads();
 
     RouteRows rows{m.A, D, m.H1};
-    pair_mlp<ROUTE_RPT, CPT>(m, R, rows, us, vs, sm + L.tile, sp);
+    pair_mlp<ROUTE_RPT, CPT>(m, R, rows, us, vs, sm + L.tile, sm + L.w3, sp);
 
     for (int r = tid; r < R; r += SIMT_THREADS) {
         const int qi = r / D, d = r - qi * D;
@@ -324,8 +356,47 @@ struct SeqRows {
     __device__ int query(int r) const { return r < n1 ? c1 + r : c2 + (r - n1); }
 };
 
+// Per-chunk auxiliary arrays (one scratch buffer, seq_aux_floats floats):
+// quality [Qs][M], standardised query slots u [Qs] and v [Qs], and the
+// standardised running count of every deployment after c more picks,
+// xr [D][Qs + 1] (c = 0 .. Qs).
+struct SeqAux {
+    float *qual, *us, *vs, *xr;
+};
+
+__host__ __device__ inline SeqAux seq_aux(float *aux, int D, int M, int Qs) {
+    SeqAux a;
+    a.qual = aux;
+    a.us = aux + (size_t)Qs * M;
+    a.vs = a.us + Qs;
+    a.xr = a.vs + Qs;
+    (void)D;
+    return a;
+}
+
+size_t seq_aux_floats(int D, int M, int Qs) {
+    return (size_t)Qs * M + 2 * (size_t)Qs + (size_t)D * (Qs + 1);
+}
+
+// K_seq_prep: the chunk's standardised features, each computed once (double
+// arithmetic is scarce on this GPU; the table blocks would otherwise repeat it).
+__global__ void __launch_bounds__(32) k_seq_prep(Model m, Queries q, int Qs, float *aux) {
+    const SeqAux a = seq_aux(aux, m.D, m.M, Qs);
+    const int t = blockIdx.x * 32 + threadIdx.x, F = m.F, P = m.P;
+    if (t < Qs) {
+        a.us[t] = standardise(m.xform[F - 2], (double)q.in_len[t], m.mu[F - 2], m.sd[F - 2]);
+    } else if (t < 2 * Qs) {
+        const int i = t - Qs;
+        a.vs[i] = standardise(m.xform[F - 1], (double)q.out_len[i], m.mu[F - 1], m.sd[F - 1]);
+    } else if (t < 2 * Qs + m.D * (Qs + 1)) {
+        const int e = t - 2 * Qs, d = e / (Qs + 1), c = e - d * (Qs + 1);
+        a.xr[e] = standardise(m.xform[P + 1], (double)(m.running[d] + c), m.mu[P + 1],
+                              m.sd[P + 1]);
+    }
+}
+
 struct SeqLayout {
-    size_t us, vs, ol, pre, sp, tile, total;
+    size_t us, vs, pre, sp, w3, tile, total;
 };
 
 __host__ __device__ inline SeqLayout seq_layout(int H1, int H2) {
@@ -333,9 +404,9 @@ __host__ __device__ inline SeqLayout seq_layout(int H1, int H2) {
     size_t o = 0;
     L.us = o; o += SEQ_MAX_CHUNK;
     L.vs = o; o += SEQ_MAX_CHUNK;
-    L.ol = o; o += SEQ_MAX_CHUNK;
     L.pre = o; o += 2 * (size_t)H1;
     L.sp = o; o += 3 * 8 * SEQ_RPT;
+    L.w3 = o; o += 3 * (size_t)H2;
     o = (o + 3) & ~(size_t)3;
     L.tile = o;
     o += tile_floats_for<SEQ_RPT>(H2);
@@ -343,127 +414,218 @@ __host__ __device__ inline SeqLayout seq_layout(int H1, int H2) {
     return L;
 }
 
+// Queries per quality block of the sequential table (at most 256 chains).
+__host__ __device__ inline int seq_qual_rows(int M) {
+    const int n = SIMT_THREADS / M;
+    return n < 1 ? 1 : (n > 8 ? 8 : n);
+}
+
 template <int CPT>
-__global__ void __launch_bounds__(SIMT_THREADS)
-k_seq_table(Model m, Queries q, int Qs, int nb_table, float *ctab, float *qualS) {
+__global__ void __launch_bounds__(SIMT_THREADS, CPT <= 4 ? 4 : 2)
+k_seq_table(Model m, Queries q, int Qs, int nb_table, float *ctab, float *aux) {
     extern __shared__ float sm[];
     const int tid = threadIdx.x;
     const int D = m.D, F = m.F, H1 = m.H1, M = m.M, P = m.P;
+    const SeqLayout L = seq_layout(H1, m.H2);
+    const SeqAux A = seq_aux(aux, D, M, Qs);
     if ((int)blockIdx.x >= nb_table) {
-        // quality of the chunk's queries: one serial chain per (query, model)
-        const int e = ((int)blockIdx.x - nb_table) * SIMT_THREADS + tid;
-        if (e < Qs * M) {
-            const int i = e / M, mi = e - i * M;
-            const size_t row = (size_t)i * m.E;
-            float s = 0.f;
-            for (int k = 0; k < m.E; ++k)
-                s = __fmaf_rn(emb_at(q.emb, q.emb_bf16, row + k), m.memb[(size_t)k * M + mi], s);
-            qualS[e] = sigmoid_c(s);
-        }
+        // quality of the chunk's queries [q0, q0 + nq), staged through the whole
+        // shared space
+        const int nq = seq_qual_rows(M), q0 = ((int)blockIdx.x - nb_table) * nq;
+        const float v = quality_staged(m, q, q0, nq, sm, (int)L.total);
+        if (tid < nq * M && q0 + tid / M < Qs) A.qual[(size_t)q0 * M + tid] = v;
         return;
     }
-    const SeqLayout L = seq_layout(H1, m.H2);
-    float *us = sm + L.us, *vs = sm + L.vs, *ol = sm + L.ol, *pre = sm + L.pre;
-    float *sp = sm + L.sp;
+    float *us = sm + L.us, *vs = sm + L.vs, *pre = sm + L.pre, *sp = sm + L.sp;
     const int d = blockIdx.x % D, c1 = blockIdx.x / D, c2 = Qs - 1 - c1;
     const bool two = c2 != c1;
     const int n1 = Qs - c1, R = n1 + (two ? c1 + 1 : 0);
 
-    for (int i = tid; i < Qs; i += SIMT_THREADS) {
-        const float o = q.out_len[i];
-        us[i] = standardise(m.xform[F - 2], (double)q.in_len[i], m.mu[F - 2], m.sd[F - 2]);
-        vs[i] = standardise(m.xform[F - 1], (double)o, m.mu[F - 1], m.sd[F - 1]);
-        ol[i] = o;
+    // standardised query slots of the rows of this block (queries c1 .. Qs - 1)
+    for (int i = c1 + tid; i < Qs; i += SIMT_THREADS) {
+        us[i] = A.us[i];
+        vs[i] = A.vs[i];
     }
     // layer-1 prefixes for running counts r_d + c1 and r_d + c2: continue the
-    // chain from slot P + 1 (running) with the deployment's other features
-    const int32_t run = m.running[d];
-    for (int e = tid; e < 2 * H1; e += SIMT_THREADS) {
-        const int g = e / H1, j = e - g * H1;
-        if (g == 1 && !two) continue;
-        const int c = g ? c2 : c1;
-        const float xr = standardise(m.xform[P + 1], (double)(run + c), m.mu[P + 1], m.sd[P + 1]);
+    // chain from slot P + 1 (running) with the deployment's other features;
+    // the two chains share their operands
+    const float xa = A.xr[(size_t)d * (Qs + 1) + c1], xb = A.xr[(size_t)d * (Qs + 1) + c2];
+    for (int j = tid; j < H1; j += SIMT_THREADS) {
         const float *w = m.W1 + (size_t)j * F;
         const float *x = m.X + (size_t)d * F;
-        float acc = m.Spre[(size_t)d * H1 + j];
-        acc = __fmaf_rn(w[P + 1], xr, acc);
-        for (int k = P + 2; k < F - 2; ++k) acc = __fmaf_rn(w[k], x[k], acc);
-        pre[e] = acc;
+        const float s0 = m.Spre[(size_t)d * H1 + j], wr = w[P + 1];
+        float a1 = __fmaf_rn(wr, xa, s0);
+        float a2 = __fmaf_rn(wr, xb, s0);
+#pragma unroll 8
+        for (int k = P + 2; k < F - 2; ++k) {
+            const float wk = w[k], xk = x[k];
+            a1 = __fmaf_rn(wk, xk, a1);
+            a2 = __fmaf_rn(wk, xk, a2);
+        }
+        pre[j] = a1;
+        if (two) pre[H1 + j] = a2;
     }
     __syncthreads();
 
     SeqRows rows{pre, H1, n1, c1, c2};
-    pair_mlp<SEQ_RPT, CPT>(m, R, rows, us, vs, sm + L.tile, sp);
+    pair_mlp<SEQ_RPT, CPT>(m, R, rows, us, vs, sm + L.tile, sm + L.w3, sp);
 
     for (int r = tid; r < R; r += SIMT_THREADS) {
         const int c = r < n1 ? c1 : c2, i = rows.query(r);
         const float *h = sp + m.NH * r;
-        const float C = __fmaf_rn(m.NH == 3 ? h[2] : ol[i], h[1], h[0]);
+        const float C = __fmaf_rn(m.NH == 3 ? h[2] : q.out_len[i], h[1], h[0]);
         ctab[tri_off(D, Qs, c) + (size_t)d * (Qs - c) + (i - c)] = C;
     }
 }
 
+// Chain shared memory (4-byte words): dep_model and picks [MAX_D] ints each,
+// the table [T rounded up to 4] (16-byte aligned), the chunk's quality
+// [Qs][M] and budgets [Qs].  After the walk the refresh reuses the space
+// from the table on: standardised running counts [MAX_D], deployment slots
+// P + 2 .. F - 3 [D][F - P - 4], W1 columns P + 1 .. F - 3 [H1][odd stride].
+__host__ __device__ inline size_t chain_tab_floats(int D, int Qs) {
+    return (tri_off(D, Qs, Qs) + 3) & ~(size_t)3;
+}
+
+__host__ __device__ inline int refresh_ld(int F, int P) { return (F - P - 3) | 1; }
+
+// Offset of the table entry (picks c, deployment d, query 0) (only i >= c is stored).
+__device__ __forceinline__ int tab_row(int D, int Qs, int c, int d) {
+    return D * (c * Qs - (c * (c - 1)) / 2) + d * (Qs - c) - c;
+}
+
 __global__ void __launch_bounds__(SIMT_THREADS)
-k_seq_chain(Model m, Queries q, int Qs, const float *ctab, const float *qualS) {
-    extern __shared__ float sm[];
+k_seq_chain(Model m, Queries q, int Qs, const float *ctab, float *aux) {
+    extern __shared__ float4 sm4[];
+    float *sm = reinterpret_cast<float *>(sm4);
     const int tid = threadIdx.x, lane = tid & 31;
     const int D = m.D, M = m.M, F = m.F, H1 = m.H1, P = m.P;
+    const SeqAux A = seq_aux(aux, D, M, Qs);
     const size_t T = tri_off(D, Qs, Qs);
-    float *tab = sm;
-    float *qs = sm + T;
-    int *dm = (int *)(qs + (size_t)Qs * M);
-    int *cnt = dm + MAX_D;
-    for (size_t e = tid; e < T; e += SIMT_THREADS) tab[e] = ctab[e];
-    for (int e = tid; e < Qs * M; e += SIMT_THREADS) qs[e] = qualS[e];
+    int *dm = reinterpret_cast<int *>(sm), *cnt = dm + MAX_D;
+    float *tab = sm + 2 * MAX_D;
+    float *qs = tab + chain_tab_floats(D, Qs), *slo = qs + (size_t)Qs * M;
+
+    // the table, by 16-byte asynchronous copies (both sides 16-byte aligned)
+    const uint32_t tab_s = (uint32_t)__cvta_generic_to_shared(tab);
+    for (size_t e = tid; e < T / 4; e += SIMT_THREADS)
+        asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(tab_s + (uint32_t)(16 * e)),
+                     "l"(__cvta_generic_to_global(ctab + 4 * e))
+                     : "memory");
+    asm volatile("cp.async.commit_group;" ::: "memory");
+    for (size_t e = T / 4 * 4 + tid; e < T; e += SIMT_THREADS) tab[e] = __ldcg(ctab + e);
+    for (int e = tid; e < Qs * M; e += SIMT_THREADS) qs[e] = __ldcg(A.qual + e);
+    for (int i = tid; i < Qs; i += SIMT_THREADS) slo[i] = query_budget(q, i);
     for (int e = tid; e < D; e += SIMT_THREADS) dm[e] = m.dep_model[e];
+    asm volatile("cp.async.wait_all;" ::: "memory");
     __syncthreads();
 
     if (tid < 32) {
-        int cA = 0, cB = 0;  // picks so far of deployments lane and lane + 32
+        // The walk.  Lane l holds deployments d0 = l and d1 = l + 32 with their
+        // picks so far (c0, c1); entry (c, d, i) is tab[tab_row(c, d) + i].
+        // Step i + 1's operands are loaded while step i is decided: for each
+        // deployment both the entry at the current count and the one after a
+        // further pick.  The winner is the decision maker's candidate order:
+        // best class, then best key, then the lowest deployment.
+        const unsigned full = 0xffffffffu;
+        const int d0 = lane, d1 = lane + 32;
+        const bool h0 = d0 < D, h1 = d1 < D;
+        const int m0 = h0 ? dm[d0] : 0, m1 = h1 ? dm[d1] : 0;
+        const float lam = q.lam, wq = q.wq;
+        int c0 = 0, c1 = 0;
+        int r0 = h0 ? tab_row(D, Qs, 0, d0) : 0, r1 = h1 ? tab_row(D, Qs, 0, d1) : 0;
+        float C0 = h0 ? tab[r0] : 0.f, C1 = h1 ? tab[r1] : 0.f;
+        float Q0 = qs[m0], Q1 = qs[m1], b = slo[0];
         for (int i = 0; i < Qs; ++i) {
-            Cand best = no_cand();
-            const float slo = query_budget(q, i);
-#pragma unroll
-            for (int t = 0; t < 2; ++t) {
-                const int d = lane + 32 * t;
-                if (d < D) {
-                    const int c = t ? cB : cA;
-                    const float C = tab[tri_off(D, Qs, c) + (size_t)d * (Qs - c) + (i - c)];
-                    const float U = __fmaf_rn(-q.lam, C, __fmul_rn(q.wq, qs[i * M + dm[d]]));
-                    Cand cd = make_cand(C, U, d, slo);
-                    if (better(cd, best)) best = cd;
+            // prefetch step i + 1 (entries exist: c <= i + 1 and c < Qs)
+            float C0s = 0.f, C0p = 0.f, C1s = 0.f, C1p = 0.f, Q0n = 0.f, Q1n = 0.f, bn = 0.f;
+            int r0p = 0, r1p = 0;
+            if (i + 1 < Qs) {
+                if (h0) {
+                    r0p = tab_row(D, Qs, c0 + 1, d0);
+                    C0s = tab[r0 + i + 1];
+                    C0p = tab[r0p + i + 1];
                 }
+                if (h1) {
+                    r1p = tab_row(D, Qs, c1 + 1, d1);
+                    C1s = tab[r1 + i + 1];
+                    C1p = tab[r1p + i + 1];
+                }
+                Q0n = qs[(i + 1) * M + m0];
+                Q1n = qs[(i + 1) * M + m1];
+                bn = slo[i + 1];
             }
-            best = warp_best(best);
-            const bool ok = best.cls > 0;
-            if (lane == 0) {
+            Cand best = no_cand();
+            if (h0) best = make_cand(C0, __fmaf_rn(-lam, C0, __fmul_rn(wq, Q0)), d0, b);
+            if (h1) {
+                Cand cd = make_cand(C1, __fmaf_rn(-lam, C1, __fmul_rn(wq, Q1)), d1, b);
+                if (better(cd, best)) best = cd;
+            }
+            const unsigned b2 = __ballot_sync(full, best.cls == 2);
+            const unsigned b1 = __ballot_sync(full, best.cls == 1);
+            const int cls = b2 ? 2 : (b1 ? 1 : 0);
+            uint32_t key = 0u;
+            if (best.cls == cls)
+                key = cls == 2 ? order_key(best.U) : cls == 1 ? ~order_key(best.C) : 1u;
+            const uint32_t kmax = __reduce_max_sync(full, key);
+            const bool tied = best.cls == cls && key == kmax;
+            const unsigned tlo = __ballot_sync(full, tied && best.d < 32);
+            const unsigned tall = __ballot_sync(full, tied);
+            const int wl = __ffs(tlo ? tlo : tall) - 1;
+            const bool ok = cls > 0;
+            if (lane == wl) {
                 q.chosen[i] = ok ? best.d : -1;
                 q.lat[i] = ok ? best.C : __int_as_float(0x7fc00000);
                 q.util[i] = ok ? best.U : __int_as_float(0x7fc00000);
             }
-            if (ok) {
-                if (best.d == lane) ++cA;
-                else if (best.d == lane + 32) ++cB;
+            const bool p0 = ok && lane == wl && best.d == d0;
+            const bool p1 = ok && lane == wl && best.d == d1;
+            if (p0) {
+                ++c0;
+                r0 = r0p;
             }
+            if (p1) {
+                ++c1;
+                r1 = r1p;
+            }
+            C0 = p0 ? C0p : C0s;
+            C1 = p1 ? C1p : C1s;
+            Q0 = Q0n;
+            Q1 = Q1n;
+            b = bn;
         }
-        if (lane < D) cnt[lane] = cA;
-        if (lane + 32 < D) cnt[lane + 32] = cB;
+        if (h0) cnt[d0] = c0;
+        if (h1) cnt[d1] = c1;
     }
     __syncthreads();
-    // persist the increments and refresh the deployment state they touch
-    for (int d = tid; d < D; d += SIMT_THREADS) m.running[d] += cnt[d];
+
+    // persist the picks and refresh the state they touch (standardised running
+    // count, layer-1 prefix): the snapshot kernel's chains, operands staged
+    const int nk = F - P - 3, wld = refresh_ld(F, P);
+    float *xr = tab, *xs = xr + MAX_D, *w1s = xs + (size_t)D * (nk - 1);
+    for (int d = tid; d < D; d += SIMT_THREADS) {
+        const float x = A.xr[(size_t)d * (Qs + 1) + cnt[d]];
+        m.running[d] += cnt[d];
+        xr[d] = x;
+        m.X[(size_t)d * F + P + 1] = x;
+    }
+    for (int e = tid; e < D * (nk - 1); e += SIMT_THREADS) {
+        const int d = e / (nk - 1), k = e - d * (nk - 1);
+        xs[e] = m.X[(size_t)d * F + P + 2 + k];
+    }
+    for (int e = tid; e < H1 * nk; e += SIMT_THREADS) {
+        const int j = e / nk, k = e - j * nk;
+        w1s[j * wld + k] = m.W1[(size_t)j * F + P + 1 + k];
+    }
     __syncthreads();
     for (int e = tid; e < D * H1; e += SIMT_THREADS) {
         const int d = e / H1, j = e - d * H1;
-        const float xr = standardise(m.xform[P + 1], (double)m.running[d], m.mu[P + 1], m.sd[P + 1]);
-        const float *w = m.W1 + (size_t)j * F;
-        const float *x = m.X + (size_t)d * F;
-        float acc = m.Spre[(size_t)d * H1 + j];
-        acc = __fmaf_rn(w[P + 1], xr, acc);
-        for (int k = P + 2; k < F - 2; ++k) acc = __fmaf_rn(w[k], x[k], acc);
-        m.A[(size_t)d * H1 + j] = acc;
-        m.Abf[(size_t)d * H1 + j] = __bfloat16_as_ushort(__float2bfloat16_rn(acc));
-        if (j == 0) m.X[(size_t)d * F + P + 1] = xr;
+        const float *w = w1s + j * wld, *x = xs + (size_t)d * (nk - 1);
+        float acc = m.Spre[e];
+        acc = __fmaf_rn(w[0], xr[d], acc);
+        for (int k = 1; k < nk; ++k) acc = __fmaf_rn(w[k], x[k - 1], acc);
+        m.A[e] = acc;
+        m.Abf[e] = __bfloat16_as_ushort(__float2bfloat16_rn(acc));
     }
 }
 
@@ -645,7 +807,12 @@ size_t seq_table_smem(const Model &m) {
 }
 
 static size_t chain_smem(int D, int M, int Qs) {
-    return (tri_off(D, Qs, Qs) + (size_t)Qs * M) * sizeof(float) + 2 * MAX_D * sizeof(int);
+    return (2 * MAX_D + chain_tab_floats(D, Qs) + (size_t)Qs * M + Qs) * sizeof(float);
+}
+
+static size_t refresh_smem(const Model &m) {
+    return (2 * MAX_D + MAX_D + (size_t)m.D * (m.F - m.P - 4) +
+            (size_t)m.H1 * refresh_ld(m.F, m.P)) * sizeof(float);
 }
 
 int seq_chunk(const Model &m) {
@@ -725,23 +892,26 @@ cudaError_t launch_select_multi(const Model &m, const Queries &q, const float *C
 }
 
 cudaError_t launch_seq_table(const Model &m, const Queries &q, int Qs, float *ctab,
-                             float *qual, cudaStream_t s) {
+                             float *aux, cudaStream_t s) {
+    const int np = 2 * Qs + m.D * (Qs + 1);
+    k_seq_prep<<<(np + 31) / 32, 32, 0, s>>>(m, q, Qs, aux);
     const int nb_table = m.D * ((Qs + 1) / 2);
-    const int nb_qual = (Qs * m.M + SIMT_THREADS - 1) / SIMT_THREADS;
+    const int nb_qual = (Qs + seq_qual_rows(m.M) - 1) / seq_qual_rows(m.M);
     const size_t smem = seq_layout(m.H1, m.H2).total * sizeof(float);
     const int blocks = nb_table + nb_qual;
     switch (cpt_for(m.H2)) {
-        case 1: k_seq_table<1><<<blocks, SIMT_THREADS, smem, s>>>(m, q, Qs, nb_table, ctab, qual); break;
-        case 2: k_seq_table<2><<<blocks, SIMT_THREADS, smem, s>>>(m, q, Qs, nb_table, ctab, qual); break;
-        case 4: k_seq_table<4><<<blocks, SIMT_THREADS, smem, s>>>(m, q, Qs, nb_table, ctab, qual); break;
-        default: k_seq_table<8><<<blocks, SIMT_THREADS, smem, s>>>(m, q, Qs, nb_table, ctab, qual); break;
+        case 1: k_seq_table<1><<<blocks, SIMT_THREADS, smem, s>>>(m, q, Qs, nb_table, ctab, aux); break;
+        case 2: k_seq_table<2><<<blocks, SIMT_THREADS, smem, s>>>(m, q, Qs, nb_table, ctab, aux); break;
+        case 4: k_seq_table<4><<<blocks, SIMT_THREADS, smem, s>>>(m, q, Qs, nb_table, ctab, aux); break;
+        default: k_seq_table<8><<<blocks, SIMT_THREADS, smem, s>>>(m, q, Qs, nb_table, ctab, aux); break;
     }
     return cudaGetLastError();
 }
 
 cudaError_t launch_seq_chain(const Model &m, const Queries &q, int Qs, const float *ctab,
-                             const float *qual, cudaStream_t s) {
-    k_seq_chain<<<1, SIMT_THREADS, chain_smem(m.D, m.M, Qs), s>>>(m, q, Qs, ctab, qual);
+                             float *aux, cudaStream_t s) {
+    const size_t a = chain_smem(m.D, m.M, Qs), b = refresh_smem(m);
+    k_seq_chain<<<1, SIMT_THREADS, a > b ? a : b, s>>>(m, q, Qs, ctab, aux);
     return cudaGetLastError();
 }
 

@@ -38,17 +38,35 @@ __device__ __forceinline__ bool better(const Cand &a, const Cand &b) {
     return a.d < b.d;
 }
 
+// 32-bit key that orders non-NaN floats as the floats compare (+0 and -0
+// map to the same key).
+__device__ __forceinline__ uint32_t order_key(float x) {
+    uint32_t u = __float_as_uint(x);
+    if ((u << 1) == 0u) u = 0u;
+    return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+
+// Best candidate of a full warp under `better`, on every lane.  Three warp
+// reductions: the best class, then within it the best key (larger U for
+// class 2, smaller C for class 1), then the lowest deployment among the
+// lanes holding that key; C and U come from the lane that holds the winner.
+// Keys of participating lanes are never 0 (a NaN would be needed), so the 0
+// of the other lanes never wins.
 __device__ __forceinline__ Cand warp_best(Cand c) {
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) {
-        Cand o;
-        o.cls = __shfl_xor_sync(0xffffffffu, c.cls, off);
-        o.d = __shfl_xor_sync(0xffffffffu, c.d, off);
-        o.C = __shfl_xor_sync(0xffffffffu, c.C, off);
-        o.U = __shfl_xor_sync(0xffffffffu, c.U, off);
-        if (better(o, c)) c = o;
-    }
-    return c;
+    const unsigned full = 0xffffffffu;
+    const int cls = (int)__reduce_max_sync(full, (unsigned)(c.cls + 1)) - 1;
+    uint32_t key = 0u;
+    if (c.cls == cls) key = cls == 2 ? order_key(c.U) : cls == 1 ? ~order_key(c.C) : 1u;
+    const uint32_t kmax = __reduce_max_sync(full, key);
+    const bool tied = c.cls == cls && key == kmax;
+    const uint32_t dmin = __reduce_min_sync(full, tied ? (uint32_t)c.d : 0xffffffffu);
+    const int src = __ffs(__ballot_sync(full, tied && (uint32_t)c.d == dmin)) - 1;
+    Cand b;
+    b.cls = cls;
+    b.d = (int)dmin;
+    b.C = __shfl_sync(full, c.C, src);
+    b.U = __shfl_sync(full, c.U, src);
+    return b;
 }
 
 __device__ __forceinline__ Cand no_cand() {

@@ -222,3 +222,95 @@ def test_three_heads_simt_exact(c, Q, flags):
                               nthreads=8)
     assert_exact(got, want, f"three heads cfg{c}")
     r.close()
+
+
+# ---------------------------------------------------------------------------
+# both small-batch kernels (pair-parallel and fused) at the same sizes: the
+# threshold between them is a tuning choice, so each must be exact on its own
+
+@pytest.mark.parametrize("pairs_max", ["0", "2048"])
+@pytest.mark.parametrize("c,Q", [(0, 1), (0, 100), (0, 511), (2, 7), (2, 64), (2, 170)])
+def test_small_batch_kernels_both_exact(monkeypatch, pairs_max, c, Q):
+    monkeypatch.setenv("HWR_PAIRS_MAX_PAIRS", pairs_max)
+    p = W.make_config(c, Q=Q)
+    r = H.Router(p)
+    got = r.route()
+    C, qual = r.score()
+    r.close()
+    orc = O.Problem(p)
+    assert_exact(got, orc.route(mode=O.F32, nthreads=8), f"cfg{c} Q={Q} pairs_max={pairs_max}")
+    Cw, _ = orc.score_all(mode=O.F32, nthreads=8)
+    assert np.array_equal(C, Cw.astype(np.float32))
+    qw = np.array([orc.quality(p["emb"][i], mode=O.F32) for i in range(Q)])
+    assert np.array_equal(qual, qw.astype(np.float32))
+
+
+# ---------------------------------------------------------------------------
+# sequential mode on more shapes: D > 32 (two deployments per lane of the
+# chain's warp), odd D, D = 1, a bf16 context, several chunks each
+
+@pytest.mark.parametrize("shape,Q", [
+    (dict(M=16, G=4, F=48, H1=32, H2=32, E=16), 100),    # D = 64: chunks of 39
+    (dict(M=5, G=3, F=24, H1=96, H2=200, E=40), 150),    # D = 15
+    (dict(M=1, G=1, F=12, H1=8, H2=8, E=8), 70),         # D = 1
+])
+def test_sequential_shapes_exact(shape, Q):
+    p = W.make_problem(Q=Q, dtype="f32", lam=0.3, slo=3.0, seed=41, bias_std=0.2, **shape)
+    r = H.Router(p)
+    got = r.route(flags=H.HWR_SEQUENTIAL)
+    want = O.Problem(p).route(mode=O.F32, sequential=True, nthreads=8)
+    assert_exact(got, want, str(shape))
+    assert np.array_equal(r.get_snapshot(), want[3])
+    r.close()
+
+
+def test_sequential_bf16_context_exact():
+    p = W.make_config(4, Q=90)      # D = 32, H = 256, bf16 inputs
+    r = H.Router(p)
+    got = r.route(flags=H.HWR_SEQUENTIAL)
+    want = O.Problem(p).route(mode=O.F32, sequential=True, nthreads=8)
+    assert_exact(got, want, "cfg4 sequential")
+    r.close()
+
+
+@pytest.mark.parametrize("slo", [0.0, float("-inf"), float("inf")])
+def test_sequential_degenerate_budgets_exact(slo):
+    p = W.make_config(2, Q=80)
+    r = H.Router(p)
+    got = r.route(slo=slo, flags=H.HWR_SEQUENTIAL)
+    want = O.Problem(p).route(slo=slo, mode=O.F32, sequential=True, nthreads=8)
+    assert_exact(got, want, f"slo={slo}")
+    r.close()
+
+
+# ---------------------------------------------------------------------------
+# exact ties: only the GPU-type columns of W1 (and the query slots) carry
+# weight and the model embeddings are zero, so deployments of one GPU type
+# have bit-identical costs and utilities; the lowest index must win (that is
+# d = g* for the best type g*, d = m G + g), on every path
+
+def _tied_problem(Q):
+    M, G, F = 16, 4, 48
+    p = W.make_problem(Q=Q, dtype="f32", M=M, G=G, F=F, H1=32, H2=32, E=16, seed=9,
+                       lam=0.4, slo=2.0, bias_std=0.3)
+    keep = np.zeros(F, bool)
+    keep[M:M + G] = True
+    keep[F - 2:] = True
+    p["W1"] = np.where(keep[None, :], p["W1"], 0.0).astype(p["W1"].dtype)
+    p["memb"] = np.zeros_like(p["memb"])
+    return p
+
+
+@pytest.mark.parametrize("slo", [float("inf"), float("-inf")])
+@pytest.mark.parametrize("mode", ["pairs", "fused", "sequential"])
+def test_exact_ties_go_to_lowest_index(monkeypatch, slo, mode):
+    Q = 40
+    p = _tied_problem(Q)
+    monkeypatch.setenv("HWR_PAIRS_MAX_PAIRS", "0" if mode == "fused" else "2048")
+    flags = H.HWR_SEQUENTIAL if mode == "sequential" else 0
+    r = H.Router(p)
+    got = r.route(slo=slo, flags=flags)
+    r.close()
+    want = O.Problem(p).route(slo=slo, mode=O.F32, sequential=bool(flags), nthreads=8)
+    assert_exact(got, want, f"ties {mode} slo={slo}")
+    assert np.all((got[0] >= 0) & (got[0] < p["G"]))
