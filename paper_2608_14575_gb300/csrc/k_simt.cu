@@ -480,9 +480,12 @@ k_seq_table(Model m, Queries q, int Qs, int nb_table, float *ctab, float *aux) {
 
 // Chain shared memory (4-byte words): dep_model and picks [MAX_D] ints each,
 // the table [T rounded up to 4] (16-byte aligned), the chunk's quality
-// [Qs][M] and budgets [Qs].  After the walk the refresh reuses the space
-// from the table on: standardised running counts [MAX_D], deployment slots
-// P + 2 .. F - 3 [D][F - P - 4], W1 columns P + 1 .. F - 3 [H1][odd stride].
+// [Qs][M], budgets [Qs] and the walk's outputs (chosen, latency, utility)
+// [3][Qs].  After the walk the refresh reuses the space from the table on:
+// standardised running counts [MAX_D], deployment slots P + 2 .. F - 3
+// [D][F - P - 4], W1 columns P + 1 .. F - 3 [H1][odd stride].
+constexpr int CHAIN_THREADS = 1024;
+
 __host__ __device__ inline size_t chain_tab_floats(int D, int Qs) {
     return (tri_off(D, Qs, Qs) + 3) & ~(size_t)3;
 }
@@ -494,7 +497,27 @@ __device__ __forceinline__ int tab_row(int D, int Qs, int c, int d) {
     return D * (c * Qs - (c * (c - 1)) / 2) + d * (Qs - c) - c;
 }
 
-__global__ void __launch_bounds__(SIMT_THREADS)
+// The decision maker's candidate order as one 40-bit integer: class + 1
+// (bits 38-39), the key within the class (bits 6-37: larger U for a
+// feasible candidate, smaller C for an infeasible one, as order-preserving
+// integers) and 63 - d (bits 0-5), so that the largest value is the best
+// candidate and ties go to the lowest deployment.  Same classes as make_cand.
+__device__ __forceinline__ uint64_t cand_key(float C, float U, int d, float slo) {
+    uint32_t cls, key;
+    if (C != C) {
+        cls = 1u;
+        key = 1u;
+    } else if (C <= slo && U == U) {
+        cls = 3u;
+        key = order_key(U);
+    } else {
+        cls = 2u;
+        key = ~order_key(C);
+    }
+    return ((uint64_t)cls << 38) | ((uint64_t)key << 6) | (uint64_t)(63 - d);
+}
+
+__global__ void __launch_bounds__(CHAIN_THREADS)
 k_seq_chain(Model m, Queries q, int Qs, const float *ctab, float *aux) {
     extern __shared__ float4 sm4[];
     float *sm = reinterpret_cast<float *>(sm4);
@@ -505,28 +528,30 @@ k_seq_chain(Model m, Queries q, int Qs, const float *ctab, float *aux) {
     int *dm = reinterpret_cast<int *>(sm), *cnt = dm + MAX_D;
     float *tab = sm + 2 * MAX_D;
     float *qs = tab + chain_tab_floats(D, Qs), *slo = qs + (size_t)Qs * M;
+    float *o_lat = slo + Qs, *o_util = o_lat + Qs;
+    int *o_ch = reinterpret_cast<int *>(o_util + Qs);
 
     // the table, by 16-byte asynchronous copies (both sides 16-byte aligned)
     const uint32_t tab_s = (uint32_t)__cvta_generic_to_shared(tab);
-    for (size_t e = tid; e < T / 4; e += SIMT_THREADS)
+    for (size_t e = tid; e < T / 4; e += CHAIN_THREADS)
         asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(tab_s + (uint32_t)(16 * e)),
                      "l"(__cvta_generic_to_global(ctab + 4 * e))
                      : "memory");
     asm volatile("cp.async.commit_group;" ::: "memory");
-    for (size_t e = T / 4 * 4 + tid; e < T; e += SIMT_THREADS) tab[e] = __ldcg(ctab + e);
-    for (int e = tid; e < Qs * M; e += SIMT_THREADS) qs[e] = __ldcg(A.qual + e);
-    for (int i = tid; i < Qs; i += SIMT_THREADS) slo[i] = query_budget(q, i);
-    for (int e = tid; e < D; e += SIMT_THREADS) dm[e] = m.dep_model[e];
+    for (size_t e = T / 4 * 4 + tid; e < T; e += CHAIN_THREADS) tab[e] = __ldcg(ctab + e);
+    for (int e = tid; e < Qs * M; e += CHAIN_THREADS) qs[e] = __ldcg(A.qual + e);
+    for (int i = tid; i < Qs; i += CHAIN_THREADS) slo[i] = query_budget(q, i);
+    for (int e = tid; e < D; e += CHAIN_THREADS) dm[e] = m.dep_model[e];
     asm volatile("cp.async.wait_all;" ::: "memory");
     __syncthreads();
 
     if (tid < 32) {
         // The walk.  Lane l holds deployments d0 = l and d1 = l + 32 with their
         // picks so far (c0, c1); entry (c, d, i) is tab[tab_row(c, d) + i].
-        // Step i + 1's operands are loaded while step i is decided: for each
-        // deployment both the entry at the current count and the one after a
-        // further pick.  The winner is the decision maker's candidate order:
-        // best class, then best key, then the lowest deployment.
+        // While step i is decided, step i + 1's entries at the current count
+        // and at one more pick are loaded and turned into candidate keys, so a
+        // step is a choice between two ready keys, a 64-bit max over the warp
+        // (two reductions) and the winner's index from the low bits.
         const unsigned full = 0xffffffffu;
         const int d0 = lane, d1 = lane + 32;
         const bool h0 = d0 < D, h1 = d1 < D;
@@ -534,52 +559,68 @@ k_seq_chain(Model m, Queries q, int Qs, const float *ctab, float *aux) {
         const float lam = q.lam, wq = q.wq;
         int c0 = 0, c1 = 0;
         int r0 = h0 ? tab_row(D, Qs, 0, d0) : 0, r1 = h1 ? tab_row(D, Qs, 0, d1) : 0;
-        float C0 = h0 ? tab[r0] : 0.f, C1 = h1 ? tab[r1] : 0.f;
-        float Q0 = qs[m0], Q1 = qs[m1], b = slo[0];
+        // this step's candidate of each deployment: cost, utility, key
+        float C0 = 0.f, U0 = 0.f, C1 = 0.f, U1 = 0.f;
+        uint64_t K0 = 0, K1 = 0;
+        {
+            const float b = slo[0];
+            if (h0) {
+                C0 = tab[r0];
+                U0 = __fmaf_rn(-lam, C0, __fmul_rn(wq, qs[m0]));
+                K0 = cand_key(C0, U0, d0, b);
+            }
+            if (h1) {
+                C1 = tab[r1];
+                U1 = __fmaf_rn(-lam, C1, __fmul_rn(wq, qs[m1]));
+                K1 = cand_key(C1, U1, d1, b);
+            }
+        }
         for (int i = 0; i < Qs; ++i) {
-            // prefetch step i + 1 (entries exist: c <= i + 1 and c < Qs)
-            float C0s = 0.f, C0p = 0.f, C1s = 0.f, C1p = 0.f, Q0n = 0.f, Q1n = 0.f, bn = 0.f;
+            // step i + 1's candidates: s = same count, p = after one more pick
+            float C0s = 0.f, U0s = 0.f, C0p = 0.f, U0p = 0.f;
+            float C1s = 0.f, U1s = 0.f, C1p = 0.f, U1p = 0.f;
+            uint64_t K0s = 0, K0p = 0, K1s = 0, K1p = 0;
             int r0p = 0, r1p = 0;
             if (i + 1 < Qs) {
+                const float b = slo[i + 1];
                 if (h0) {
+                    const float wQ = __fmul_rn(wq, qs[(i + 1) * M + m0]);
                     r0p = tab_row(D, Qs, c0 + 1, d0);
                     C0s = tab[r0 + i + 1];
                     C0p = tab[r0p + i + 1];
+                    U0s = __fmaf_rn(-lam, C0s, wQ);
+                    U0p = __fmaf_rn(-lam, C0p, wQ);
+                    K0s = cand_key(C0s, U0s, d0, b);
+                    K0p = cand_key(C0p, U0p, d0, b);
                 }
                 if (h1) {
+                    const float wQ = __fmul_rn(wq, qs[(i + 1) * M + m1]);
                     r1p = tab_row(D, Qs, c1 + 1, d1);
                     C1s = tab[r1 + i + 1];
                     C1p = tab[r1p + i + 1];
+                    U1s = __fmaf_rn(-lam, C1s, wQ);
+                    U1p = __fmaf_rn(-lam, C1p, wQ);
+                    K1s = cand_key(C1s, U1s, d1, b);
+                    K1p = cand_key(C1p, U1p, d1, b);
                 }
-                Q0n = qs[(i + 1) * M + m0];
-                Q1n = qs[(i + 1) * M + m1];
-                bn = slo[i + 1];
             }
-            Cand best = no_cand();
-            if (h0) best = make_cand(C0, __fmaf_rn(-lam, C0, __fmul_rn(wq, Q0)), d0, b);
-            if (h1) {
-                Cand cd = make_cand(C1, __fmaf_rn(-lam, C1, __fmul_rn(wq, Q1)), d1, b);
-                if (better(cd, best)) best = cd;
+            // step i: the warp's largest key
+            const uint64_t kl = K0 > K1 ? K0 : K1;
+            const uint32_t hi = __reduce_max_sync(full, (uint32_t)(kl >> 32));
+            const uint32_t lo =
+                __reduce_max_sync(full, (uint32_t)(kl >> 32) == hi ? (uint32_t)kl : 0u);
+            const int wd = 63 - (int)(lo & 63u);
+            const bool ok = (hi >> 6) >= 2u;    // class feasible or infeasible, not NaN
+            const bool p0 = ok && wd == d0, p1 = ok && wd == d1;
+            if (p0 || p1) {
+                o_ch[i] = wd;
+                o_lat[i] = p0 ? C0 : C1;
+                o_util[i] = p0 ? U0 : U1;
+            } else if (!ok && lane == 0) {
+                o_ch[i] = -1;
+                o_lat[i] = __int_as_float(0x7fc00000);
+                o_util[i] = __int_as_float(0x7fc00000);
             }
-            const unsigned b2 = __ballot_sync(full, best.cls == 2);
-            const unsigned b1 = __ballot_sync(full, best.cls == 1);
-            const int cls = b2 ? 2 : (b1 ? 1 : 0);
-            uint32_t key = 0u;
-            if (best.cls == cls)
-                key = cls == 2 ? order_key(best.U) : cls == 1 ? ~order_key(best.C) : 1u;
-            const uint32_t kmax = __reduce_max_sync(full, key);
-            const bool tied = best.cls == cls && key == kmax;
-            const unsigned tlo = __ballot_sync(full, tied && best.d < 32);
-            const unsigned tall = __ballot_sync(full, tied);
-            const int wl = __ffs(tlo ? tlo : tall) - 1;
-            const bool ok = cls > 0;
-            if (lane == wl) {
-                q.chosen[i] = ok ? best.d : -1;
-                q.lat[i] = ok ? best.C : __int_as_float(0x7fc00000);
-                q.util[i] = ok ? best.U : __int_as_float(0x7fc00000);
-            }
-            const bool p0 = ok && lane == wl && best.d == d0;
-            const bool p1 = ok && lane == wl && best.d == d1;
             if (p0) {
                 ++c0;
                 r0 = r0p;
@@ -589,13 +630,20 @@ k_seq_chain(Model m, Queries q, int Qs, const float *ctab, float *aux) {
                 r1 = r1p;
             }
             C0 = p0 ? C0p : C0s;
+            U0 = p0 ? U0p : U0s;
+            K0 = p0 ? K0p : K0s;
             C1 = p1 ? C1p : C1s;
-            Q0 = Q0n;
-            Q1 = Q1n;
-            b = bn;
+            U1 = p1 ? U1p : U1s;
+            K1 = p1 ? K1p : K1s;
         }
         if (h0) cnt[d0] = c0;
         if (h1) cnt[d1] = c1;
+    }
+    __syncthreads();
+    for (int i = tid; i < Qs; i += CHAIN_THREADS) {
+        q.chosen[i] = o_ch[i];
+        q.lat[i] = o_lat[i];
+        q.util[i] = o_util[i];
     }
     __syncthreads();
 
@@ -603,22 +651,22 @@ k_seq_chain(Model m, Queries q, int Qs, const float *ctab, float *aux) {
     // count, layer-1 prefix): the snapshot kernel's chains, operands staged
     const int nk = F - P - 3, wld = refresh_ld(F, P);
     float *xr = tab, *xs = xr + MAX_D, *w1s = xs + (size_t)D * (nk - 1);
-    for (int d = tid; d < D; d += SIMT_THREADS) {
+    for (int d = tid; d < D; d += CHAIN_THREADS) {
         const float x = A.xr[(size_t)d * (Qs + 1) + cnt[d]];
         m.running[d] += cnt[d];
         xr[d] = x;
         m.X[(size_t)d * F + P + 1] = x;
     }
-    for (int e = tid; e < D * (nk - 1); e += SIMT_THREADS) {
+    for (int e = tid; e < D * (nk - 1); e += CHAIN_THREADS) {
         const int d = e / (nk - 1), k = e - d * (nk - 1);
         xs[e] = m.X[(size_t)d * F + P + 2 + k];
     }
-    for (int e = tid; e < H1 * nk; e += SIMT_THREADS) {
+    for (int e = tid; e < H1 * nk; e += CHAIN_THREADS) {
         const int j = e / nk, k = e - j * nk;
         w1s[j * wld + k] = m.W1[(size_t)j * F + P + 1 + k];
     }
     __syncthreads();
-    for (int e = tid; e < D * H1; e += SIMT_THREADS) {
+    for (int e = tid; e < D * H1; e += CHAIN_THREADS) {
         const int d = e / H1, j = e - d * H1;
         const float *w = w1s + j * wld, *x = xs + (size_t)d * (nk - 1);
         float acc = m.Spre[e];
@@ -807,7 +855,7 @@ size_t seq_table_smem(const Model &m) {
 }
 
 static size_t chain_smem(int D, int M, int Qs) {
-    return (2 * MAX_D + chain_tab_floats(D, Qs) + (size_t)Qs * M + Qs) * sizeof(float);
+    return (2 * MAX_D + chain_tab_floats(D, Qs) + (size_t)Qs * M + 4 * (size_t)Qs) * sizeof(float);
 }
 
 static size_t refresh_smem(const Model &m) {
@@ -911,7 +959,7 @@ cudaError_t launch_seq_table(const Model &m, const Queries &q, int Qs, float *ct
 cudaError_t launch_seq_chain(const Model &m, const Queries &q, int Qs, const float *ctab,
                              float *aux, cudaStream_t s) {
     const size_t a = chain_smem(m.D, m.M, Qs), b = refresh_smem(m);
-    k_seq_chain<<<1, SIMT_THREADS, a > b ? a : b, s>>>(m, q, Qs, ctab, aux);
+    k_seq_chain<<<1, CHAIN_THREADS, a > b ? a : b, s>>>(m, q, Qs, ctab, aux);
     return cudaGetLastError();
 }
 
