@@ -70,7 +70,7 @@ struct hwr_ctx {
     uint8_t *xform = nullptr;
     float *memb = nullptr;
     float *W1q = nullptr;            // [2][H1]
-    float *W2T = nullptr;            // [H1][H2] fp32, for the small-batch kernel
+    float *W2T = nullptr;            // [H1][H2p] fp32 (rows zero-padded), for the SIMT tiles
     uint16_t *W2img = nullptr, *membimg = nullptr;
     std::vector<char> head_consts;   // output-layer constants for the tensor path
     int32_t *running = nullptr, *waiting = nullptr;
@@ -99,6 +99,7 @@ struct hwr_ctx {
     float *ctab = nullptr;   size_t ctab_cap = 0;
     float *qseq = nullptr;   size_t qseq_cap = 0;
     int seq_qs = 0;
+    int seq_slots = 0;       // sequential-table blocks resident at once
 
     // I/O staging for host pointers: device [emb | in | out] and [chosen | lat | util]
     char *io_d = nullptr;    size_t io_cap = 0;
@@ -227,6 +228,7 @@ static Model model_view(const hwr_ctx *c) {
     m.E = c->E; m.P = c->P; m.NH = c->NH;
     m.dep_model = c->dep_model; m.dep_gpu = c->dep_gpu; m.log10p = c->log10p;
     m.W1 = c->W1; m.b1 = c->b1; m.W2 = c->W2; m.b2 = c->b2; m.W3 = c->W3; m.b3 = c->b3;
+    m.W2T = c->W2T; m.H2p = (c->H2 + 3) & ~3;
     m.mu = c->mu; m.sd = c->sd; m.xform = c->xform; m.memb = c->memb;
     m.running = c->running; m.waiting = c->waiting; m.kv = c->kv;
     m.gpu_util = c->gpu_util; m.ttft = c->ttft; m.tpot = c->tpot;
@@ -403,7 +405,8 @@ static hwr_status build_ctx(hwr_ctx *c, const hwr_deployment_table *t, const hwr
     TRY(dev_alloc(c, &c->xform, F));
     TRY(dev_alloc(c, &c->memb, me.size()));
     TRY(dev_alloc(c, &c->W1q, 2 * (size_t)H1));
-    TRY(dev_alloc(c, &c->W2T, (size_t)H1 * H2));
+    const int H2p = (H2 + 3) & ~3;
+    TRY(dev_alloc(c, &c->W2T, (size_t)H1 * H2p));
     TRY(dev_alloc(c, &c->pairC, (size_t)PAIRS_MAX_PAIRS));
     TRY(dev_alloc(c, &c->pairQ, (size_t)PAIRS_MAX_PAIRS * M));
     TRY(dev_alloc(c, &c->pairN, (size_t)PAIRS_MAX_PAIRS));
@@ -439,9 +442,9 @@ static hwr_status build_ctx(hwr_ctx *c, const hwr_deployment_table *t, const hwr
         w1q[H1 + j] = w1[(size_t)j * F + F - 1];
     }
     TRY(upload(c, c->W1q, w1q.data(), w1q.size() * 4, "upload W1 query columns"));
-    std::vector<float> w2t((size_t)H1 * H2);
+    std::vector<float> w2t((size_t)H1 * H2p, 0.0f);
     for (int n = 0; n < H2; ++n)
-        for (int k = 0; k < H1; ++k) w2t[(size_t)k * H2 + n] = w2[(size_t)n * H1 + k];
+        for (int k = 0; k < H1; ++k) w2t[(size_t)k * H2p + n] = w2[(size_t)n * H1 + k];
     TRY(upload(c, c->W2T, w2t.data(), w2t.size() * 4, "upload W2 transposed"));
     CK(c, cudaMemset(c->pairN, 0, PAIRS_MAX_PAIRS * sizeof(int32_t)), "zero counters");
     c->mu_in = p->feat_mean[F - 2]; c->sd_in = p->feat_std[F - 2]; c->xf_in = p->feat_xform[F - 2];
@@ -489,6 +492,7 @@ static hwr_status build_ctx(hwr_ctx *c, const hwr_deployment_table *t, const hwr
     CK(c, cudaEventCreateWithFlags(&c->io_free_ev, cudaEventDisableTiming), "create event");
 
     c->seq_qs = seq_chunk(model_view(c));
+    c->seq_slots = seq_table_slots(model_view(c));
     CK(c, cudaDeviceSynchronize(), "create");
     return HWR_OK;
 }
@@ -603,7 +607,7 @@ static hwr_status run_kernels(hwr_ctx *c, const Queries &q, uint32_t flags, bool
     if (flags & HWR_SEQUENTIAL) {
         const int Qs = c->seq_qs;
         TRY(grow(c, &c->ctab, &c->ctab_cap, seq_table_floats(c->D, Qs)));
-        TRY(grow(c, &c->qseq, &c->qseq_cap, seq_aux_floats(c->D, c->M, Qs)));
+        TRY(grow(c, &c->qseq, &c->qseq_cap, seq_aux_floats(c->D, c->M, c->H1, Qs)));
         const size_t es = c->dtype == HWR_BF16 ? 2 : 4;
         for (int lo = 0; lo < q.Q; lo += Qs) {
             Queries k = q;
@@ -617,7 +621,8 @@ static hwr_status run_kernels(hwr_ctx *c, const Queries &q, uint32_t flags, bool
             k.util = q.util + lo;
             if (q.slo_q) k.slo_q = q.slo_q + lo;
             LaunchScope a(c, HWR_K_SEQ_TABLE, prof);
-            CK(c, launch_seq_table(m, k, n, c->ctab, c->qseq, c->stream), "sequential table");
+            CK(c, launch_seq_table(m, k, n, c->seq_slots, c->ctab, c->qseq, c->stream),
+               "sequential table");
             a.done();
             CK(c, launch_seq_chain(m, k, n, c->ctab, c->qseq, c->stream), "sequential chain");
             // the preparation kernel (inside launch_seq_table) and the chain
@@ -648,7 +653,7 @@ static hwr_status run_kernels(hwr_ctx *c, const Queries &q, uint32_t flags, bool
     }
     LaunchScope a(c, HWR_K_ROUTE_SIMT, prof);
     if ((long)q.Q * c->D <= c->pairs_max)
-        CK(c, launch_route_pairs(m, q, c->W2T, c->pairC, c->pairQ, c->pairN, c->stream),
+        CK(c, launch_route_pairs(m, q, c->pairC, c->pairQ, c->pairN, c->stream),
            "route kernel");
     else
         CK(c, launch_route_simt(m, q, c->stream), "route kernel");

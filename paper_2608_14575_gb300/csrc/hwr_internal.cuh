@@ -12,12 +12,8 @@ namespace hwr {
 // Device status word, written by kernels whose waits are bounded.
 enum : int32_t { ST_OK = 0, ST_TIMEOUT = 1, ST_BAD_LAUNCH = 2 };
 
-// Largest number of (query, deployment) rows one SIMT tile holds:
-// 8 row groups (one per warp) x RPT rows each.
 constexpr int SIMT_THREADS = 256;
-constexpr int SIMT_KC = 32;          // K chunk of the layer-2 tile
-constexpr int ROUTE_RPT = 8;         // route kernel: rows <= 64
-constexpr int SEQ_RPT = 9;           // sequential table: rows <= 72 (Qs + 1)
+constexpr int SIMT_KC = 32;          // K chunk of the layer-2 tile (64 rows: 8 warps x 8)
 constexpr int MAX_D = 64;
 constexpr int MAX_H = 256;
 constexpr int SEQ_MAX_CHUNK = 64;    // queries per sequential table
@@ -32,6 +28,8 @@ struct Model {
     const float *log10p;        // [M]
     const float *W1, *b1;       // [H1][F], [H1]   fp32 (bf16 widened)
     const float *W2, *b2;       // [H2][H1], [H2]
+    const float *W2T;           // [H1][H2p]: W2 transposed, rows zero-padded to H2p
+    int H2p;                    // H2 rounded up to a multiple of 4 (16-byte rows)
     const float *W3, *b3;       // [NH][H2], [NH]
     const float *mu, *sd;       // [F]
     const uint8_t *xform;       // [F]
@@ -91,21 +89,24 @@ cudaError_t launch_snapshot(const Model &m, cudaStream_t s);
 cudaError_t launch_route_simt(const Model &m, const Queries &q, cudaStream_t s);
 // Small-batch (latency) variant: one block per (query, deployment) pair plus
 // quality blocks; scratch pairC [Q][D], qualS [Q][M], count [Q] (zeroed once,
-// self-resetting).  W2T is W2 transposed ([H1][H2], fp32).
+// self-resetting).  Reads W2 through m.W2T.
 constexpr int PAIRS_MAX_PAIRS = 2048;   // default upper bound on Q * D for this kernel
-cudaError_t launch_route_pairs(const Model &m, const Queries &q, const float *W2T, float *pairC,
-                               float *qualS, int32_t *count, cudaStream_t s);
+cudaError_t launch_route_pairs(const Model &m, const Queries &q, float *pairC, float *qualS,
+                               int32_t *count, cudaStream_t s);
 size_t route_pairs_smem(const Model &m);
 // Sequential mode over one chunk of Qs <= seq_chunk(m) queries: the chunk's
-// standardised features and the score table (every (picks c, deployment d,
-// query i >= c)) in launch_seq_table (two kernels), then the serial chain.
+// standardised features and layer-1 prefixes, and the score table (every
+// (picks c, deployment d, query i >= c)) in launch_seq_table (two kernels),
+// then the serial chain.
 //   ctab: scratch of seq_table_floats(D, Qs) floats;
-//   aux: scratch of seq_aux_floats(D, M, Qs) floats.
-cudaError_t launch_seq_table(const Model &m, const Queries &q, int Qs,
+//   aux: scratch of seq_aux_floats(D, M, H1, Qs) floats;
+//   slots: table blocks resident on the whole GPU at once (seq_table_slots).
+cudaError_t launch_seq_table(const Model &m, const Queries &q, int Qs, int slots,
                              float *ctab, float *aux, cudaStream_t s);
 cudaError_t launch_seq_chain(const Model &m, const Queries &q, int Qs,
                              const float *ctab, float *aux, cudaStream_t s);
-size_t seq_aux_floats(int D, int M, int Qs);
+size_t seq_aux_floats(int D, int M, int H1, int Qs);
+int seq_table_slots(const Model &m);
 // Decision maker for K lambdas from stored scores: C [Q][D], quality
 // qual[q * qstride + model]; outputs [K][ostride] starting at query 0.
 cudaError_t launch_select_multi(const Model &m, const Queries &q, const float *C,

@@ -72,34 +72,75 @@ __device__ __forceinline__ float emb_at(const void *emb, int bf16, size_t i) {
 
 // Quality score (Sec. 3.2, hardware-independent term) of queries
 // [q0, q0 + nq): one serial chain per (query, model) from 0 with k ascending,
-// then the sigmoid.  The embedding rows and the model columns are staged
-// through `stage` (stage_floats >= 2 nq + M + 1) in chunks of the embedding
-// dimension; the chains read shared memory only.  Every thread of the block
-// calls this; thread t < nq * M returns the score of query t / M, model t % M
-// (rows at or past q.Q give sigmoid(0)), the others return 0.  Ends with the
-// stage free for reuse after a barrier.
+// then the sigmoid.  The embedding rows (as stored, fp32 or bf16) and the
+// model columns are staged through `stage` (at least (nq + M) * 8 + 64
+// floats) in chunks of the embedding dimension by 16-byte asynchronous copies
+// when the embeddings are 16-byte aligned (plain loads otherwise); the
+// chains read shared memory only.  Every thread of the block calls this;
+// thread t < nq * M returns the score of query t / M, model t % M (rows at or
+// past q.Q give sigmoid(0)), the others return 0.  Ends with the stage free
+// for reuse after a barrier.
 __device__ float quality_staged(const Model &m, const Queries &q, int q0, int nq, float *stage,
                                 int stage_floats) {
     const int tid = threadIdx.x, M = m.M, E = m.E;
-    int ek = (stage_floats - nq) / (nq + M);
-    if (ek > E) ek = E;
-    const int ld = ek + 1;
-    float *er = stage, *mb = stage + (size_t)nq * ld;
+    const int es = q.emb_bf16 ? 2 : 4;
+    const bool async = ((uintptr_t)q.emb & 15) == 0;
+    // row stride ld (elements): 16-byte rows whose 4-byte word stride is 4
+    // mod 32, so the chains of one warp (up to 8 rows) read distinct banks
+    auto stride = [&](int ek) {
+        return es == 4 ? ((ek - 4 + 31) / 32) * 32 + 4 : ((ek - 8 + 63) / 64) * 64 + 8;
+    };
+    int ek = E;
+    while (ek > 8 && ((size_t)nq * stride(ek) * es + 16 + (size_t)ek * M * 4) > 4 * (size_t)stage_floats)
+        ek -= 8;
+    const int ld = stride(ek);
+    char *er = reinterpret_cast<char *>(stage);
+    float *mb = reinterpret_cast<float *>(er + (((size_t)nq * ld * es + 15) & ~(size_t)15));
     const int qi = tid / M, mi = tid - qi * M;
     float s = 0.f;
     for (int k0 = 0; k0 < E; k0 += ek) {
         const int kc = min(ek, E - k0);
         __syncthreads();
-        for (int t = tid; t < nq * kc; t += SIMT_THREADS) {
-            const int i = t / kc, k = t - i * kc, qq = q0 + i;
-            er[i * ld + k] = qq < q.Q ? emb_at(q.emb, q.emb_bf16, (size_t)qq * E + k0 + k) : 0.f;
+        if (async) {
+            const int gpr = kc * es / 16;     // granules per row (kc is a multiple of 8)
+            const uint32_t eb = (uint32_t)__cvta_generic_to_shared(er);
+            for (int g = tid; g < nq * gpr; g += SIMT_THREADS) {
+                const int i = g / gpr, c = g - i * gpr, qq = q0 + i;
+                const char *src = (const char *)q.emb + ((size_t)(qq < q.Q ? qq : 0) * E + k0) * es + 16 * c;
+                asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(
+                                 eb + (uint32_t)(i * ld * es + 16 * c)),
+                             "l"(__cvta_generic_to_global(src)), "r"(qq < q.Q ? 16 : 0)
+                             : "memory");
+            }
+            const uint32_t mbs = (uint32_t)__cvta_generic_to_shared(mb);
+            for (int g = tid; g < kc * M / 4; g += SIMT_THREADS)
+                asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(mbs + 16u * g),
+                             "l"(__cvta_generic_to_global(m.memb + (size_t)k0 * M + 4 * g))
+                             : "memory");
+            asm volatile("cp.async.commit_group;" ::: "memory");
+            asm volatile("cp.async.wait_group 0;" ::: "memory");
+        } else {
+            for (int t = tid; t < nq * kc; t += SIMT_THREADS) {
+                const int i = t / kc, k = t - i * kc, qq = q0 + i;
+                const size_t src = (size_t)(qq < q.Q ? qq : 0) * E + k0 + k;
+                if (es == 4) reinterpret_cast<float *>(er)[i * ld + k] = qq < q.Q ? ((const float *)q.emb)[src] : 0.f;
+                else reinterpret_cast<uint16_t *>(er)[i * ld + k] = qq < q.Q ? ((const uint16_t *)q.emb)[src] : 0;
+            }
+            for (int t = tid; t < kc * M; t += SIMT_THREADS) mb[t] = m.memb[(size_t)k0 * M + t];
         }
-        for (int t = tid; t < kc * M; t += SIMT_THREADS) mb[t] = m.memb[(size_t)k0 * M + t];
         __syncthreads();
         if (tid < nq * M) {
-            const float *a = er + qi * ld, *b = mb + mi;
+            const float *b = mb + mi;
+            if (es == 4) {
+                const float *a = reinterpret_cast<const float *>(er) + qi * ld;
 #pragma unroll 8
-            for (int k = 0; k < kc; ++k) s = __fmaf_rn(a[k], b[k * M], s);
+                for (int k = 0; k < kc; ++k) s = __fmaf_rn(a[k], b[k * M], s);
+            } else {
+                const uint16_t *a = reinterpret_cast<const uint16_t *>(er) + qi * ld;
+#pragma unroll 8
+                for (int k = 0; k < kc; ++k)
+                    s = __fmaf_rn(__uint_as_float((uint32_t)a[k] << 16), b[k * M], s);
+            }
         }
     }
     return tid < nq * M ? sigmoid_c(s) : 0.f;
@@ -132,91 +173,159 @@ __global__ void __launch_bounds__(SIMT_THREADS) k_snapshot(Model m) {
 }
 
 // ---------------------------------------------------------------------------
-// The shared SIMT tile: rows are (query, deployment) pairs.  For every row it
-// completes layer 1 from a deployment prefix and the two query features,
-// runs layer 2 (register-tiled, K ascending in chunks of SIMT_KC), layer 3
-// and the softplus heads.  Output: sp[NH r + 0] = TTFT, sp[NH r + 1] = TPOT
-// and, with three heads, sp[NH r + 2] = N_out.
+// The shared SIMT tile: up to TILE_ROWS rows, each a (query, deployment) pair
+// or a sequential-table entry.  For every row it completes layer 1 from a
+// deployment prefix and the two query features, runs layer 2 (register-tiled,
+// K ascending in chunks of SIMT_KC), layer 3 and the softplus heads.  Output:
+// sp[NH r + 0] = TTFT, sp[NH r + 1] = TPOT and, with three heads,
+// sp[NH r + 2] = N_out.
 //
-// Thread map: warp w owns rows w + 8 i (i < RPT); lane l owns columns
-// l + 32 j (j < CPT).  Shared memory: h1 [8 RPT][KC + 1] and W2 chunk
-// [KC][H2 + 1] during the K loop, then h2 [8 RPT][H2 + 1] in the same space;
-// W3 [NH][H2] staged in w3s for the head chains.
+// Thread map: warp w owns rows 8w .. 8w + 7 and lane l owns columns
+// 128 j + VW l + v (v < VW = min(CPT, 4), j < CPT / VW): a lane reads its
+// rows' layer-1 values as two 16-byte broadcasts and its W2 columns as
+// vectors that are contiguous across the warp.  Shared memory: the layer-1
+// chunk [KC][TILE_ROWS] (k-major) and two W2 chunks [KC][32 CPT] (rows of W2
+// transposed; the next chunk's cp.async copies run while this one is used),
+// then h2 [TILE_ROWS][H2 + 1] in the same space; W3 [NH][H2] in w3s.
 
-template <int RPT>
-__host__ __device__ constexpr size_t tile_floats_for(int H2) {
-    return (size_t)8 * RPT * (SIMT_KC + 1) + (size_t)SIMT_KC * (H2 + 1) >
-                   (size_t)8 * RPT * (H2 + 1)
-               ? (size_t)8 * RPT * (SIMT_KC + 1) + (size_t)SIMT_KC * (H2 + 1)
-               : (size_t)8 * RPT * (H2 + 1);
+constexpr int TILE_ROWS = 64;
+
+__host__ __device__ constexpr int tile_width(int H2) {
+    return H2 <= 32 ? 32 : H2 <= 64 ? 64 : H2 <= 128 ? 128 : 256;
 }
 
-template <int RPT, int CPT, class Rows>
+__host__ __device__ constexpr size_t tile_floats_for(int H2) {
+    return (size_t)SIMT_KC * TILE_ROWS + 2 * (size_t)SIMT_KC * tile_width(H2) >
+                   (size_t)TILE_ROWS * (H2 + 1)
+               ? (size_t)SIMT_KC * TILE_ROWS + 2 * (size_t)SIMT_KC * tile_width(H2)
+               : (size_t)TILE_ROWS * (H2 + 1);
+}
+
+// Rows k0 .. k0 + kc - 1 of W2 transposed into dst [kc][W] by 16-byte
+// asynchronous copies (W2T rows are H2p floats, 16-byte aligned); one group.
+__device__ __forceinline__ void w2_chunk_async(const Model &m, int k0, int kc, float *dst, int W) {
+    const int gpr = m.H2p >> 2;
+    const uint32_t base = (uint32_t)__cvta_generic_to_shared(dst);
+    for (int g = threadIdx.x; g < kc * gpr; g += SIMT_THREADS) {
+        const int kk = g / gpr, c4 = g - kk * gpr;
+        const float *src = m.W2T + (size_t)(k0 + kk) * m.H2p + 4 * c4;
+        asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(
+                         base + (uint32_t)(4 * (kk * W + 4 * c4))),
+                     "l"(__cvta_generic_to_global(src))
+                     : "memory");
+    }
+    asm volatile("cp.async.commit_group;" ::: "memory");
+}
+
+template <int CPT, class Rows>
 __device__ void pair_mlp(const Model &m, int R, const Rows &rows, const float *us,
-                         const float *vs, float *tile, float *w3s, float *sp) {
+                         const float *vs, float *tile, float *w3s, float *w1q, float *sp) {
+    constexpr int VW = CPT < 4 ? CPT : 4, W = 32 * CPT;
+    static_assert(SIMT_THREADS == 4 * TILE_ROWS, "layer-1 map: 4 threads per row");
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int H1 = m.H1, H2 = m.H2, F = m.F;
-    float *h1s = tile;
-    float *w2s = tile + 8 * RPT * (SIMT_KC + 1);
-    const int w2ld = H2 + 1;
+    float *h1T = tile;
+    float *w2b = tile + SIMT_KC * TILE_ROWS;
 
-    // W3 for the head chains (visible after the first barrier of the K loop)
+    // W3 for the head chains and the two query columns of W1 (visible after
+    // the first barrier of the K loop)
     for (int i = tid; i < m.NH * H2; i += SIMT_THREADS) w3s[i] = m.W3[i];
-    float acc[RPT][CPT];
+    for (int k = tid; k < H1; k += SIMT_THREADS) {
+        w1q[k] = m.W1[(size_t)k * F + F - 2];
+        w1q[H1 + k] = m.W1[(size_t)k * F + F - 1];
+    }
+    w2_chunk_async(m, 0, min(SIMT_KC, H1), w2b, W);
+    // layer-1 map: thread t fills row t % 64 at k offsets t / 64 + 4 j of a chunk
+    const int r1 = tid % TILE_ROWS, kq = tid / TILE_ROWS;
+    const bool rv = r1 < R;
+    const float *pr = rv ? rows.prefix(r1) : m.W1;
+    const float uq = rv ? us[rows.query(r1)] : 0.f, vq = rv ? vs[rows.query(r1)] : 0.f;
+    __syncthreads();
+    float acc[8][CPT];
 #pragma unroll
     for (int j = 0; j < CPT; ++j) {
-        const int n = lane + 32 * j;
+        const int n = 128 * (j / VW) + VW * lane + j % VW;
         const float b = n < H2 ? m.b2[n] : 0.f;
 #pragma unroll
-        for (int i = 0; i < RPT; ++i) acc[i][j] = b;
+        for (int i = 0; i < 8; ++i) acc[i][j] = b;
     }
+    const bool active = 8 * warp < R;
 
-    for (int k0 = 0; k0 < H1; k0 += SIMT_KC) {
+    for (int k0 = 0, it = 0; k0 < H1; k0 += SIMT_KC, ++it) {
         const int kc = min(SIMT_KC, H1 - k0);
-        // layer 1, query suffix: h1 = relu(fma(w_out, v, fma(w_in, u, prefix)))
-        for (int e = tid; e < R * SIMT_KC; e += SIMT_THREADS) {
-            const int r = e / SIMT_KC, kk = e - r * SIMT_KC;
-            if (kk < kc) {
-                const int k = k0 + kk;
-                const float *w = m.W1 + (size_t)k * F;
-                float a = rows.prefix(r)[k];
-                a = __fmaf_rn(w[F - 2], us[rows.query(r)], a);
-                a = __fmaf_rn(w[F - 1], vs[rows.query(r)], a);
-                h1s[r * (SIMT_KC + 1) + kk] = a > 0.f ? a : 0.f;
-            }
+        // layer 1, query suffix: h1 = relu(fma(w_out, v, fma(w_in, u, prefix)));
+        // rows at or past R hold 0; a thread's prefix loads are issued together
+        float pv[SIMT_KC / 4];
+#pragma unroll
+        for (int j = 0; j < SIMT_KC / 4; ++j) {
+            const int kk = kq + 4 * j;
+            pv[j] = rv && kk < kc ? pr[k0 + kk] : 0.f;
         }
-        for (int e = tid; e < H2 * SIMT_KC; e += SIMT_THREADS) {
-            const int n = e / SIMT_KC, kk = e - n * SIMT_KC;
-            if (kk < kc) w2s[kk * w2ld + n] = m.W2[(size_t)n * H1 + k0 + kk];
+#pragma unroll
+        for (int j = 0; j < SIMT_KC / 4; ++j) {
+            const int kk = kq + 4 * j;
+            float a = 0.f;
+            if (rv && kk < kc) {
+                a = __fmaf_rn(w1q[k0 + kk], uq, pv[j]);
+                a = __fmaf_rn(w1q[H1 + k0 + kk], vq, a);
+                a = a > 0.f ? a : 0.f;
+            }
+            h1T[kk * TILE_ROWS + r1] = a;
+        }
+        // the next W2 chunk goes into the other buffer; this one must be complete
+        if (k0 + SIMT_KC < H1) {
+            w2_chunk_async(m, k0 + SIMT_KC, min(SIMT_KC, H1 - k0 - SIMT_KC),
+                           w2b + ((it + 1) & 1) * SIMT_KC * W, W);
+            asm volatile("cp.async.wait_group 1;" ::: "memory");
+        } else {
+            asm volatile("cp.async.wait_group 0;" ::: "memory");
         }
         __syncthreads();
-        for (int kk = 0; kk < kc; ++kk) {
-            float b[CPT];
+        if (active) {
+            const float *wb = w2b + (it & 1) * SIMT_KC * W;
+            for (int kk = 0; kk < kc; ++kk) {
+                const float4 a0 = *reinterpret_cast<const float4 *>(h1T + kk * TILE_ROWS + 8 * warp);
+                const float4 a1 =
+                    *reinterpret_cast<const float4 *>(h1T + kk * TILE_ROWS + 8 * warp + 4);
+                const float a[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
+                float b[CPT];
+                const float *wr = wb + kk * W + VW * lane;
 #pragma unroll
-            for (int j = 0; j < CPT; ++j) {
-                const int n = lane + 32 * j;
-                b[j] = n < H2 ? w2s[kk * w2ld + n] : 0.f;
-            }
+                for (int v = 0; v < CPT / VW; ++v) {
+                    if constexpr (VW == 4) {
+                        const float4 t = *reinterpret_cast<const float4 *>(wr + 128 * v);
+                        b[4 * v] = t.x;
+                        b[4 * v + 1] = t.y;
+                        b[4 * v + 2] = t.z;
+                        b[4 * v + 3] = t.w;
+                    } else if constexpr (VW == 2) {
+                        const float2 t = *reinterpret_cast<const float2 *>(wr);
+                        b[0] = t.x;
+                        b[1] = t.y;
+                    } else {
+                        b[0] = wr[0];
+                    }
+                }
 #pragma unroll
-            for (int i = 0; i < RPT; ++i) {
-                const float a = h1s[(warp + 8 * i) * (SIMT_KC + 1) + kk];
+                for (int i = 0; i < 8; ++i)
 #pragma unroll
-                for (int j = 0; j < CPT; ++j) acc[i][j] = __fmaf_rn(b[j], a, acc[i][j]);
+                    for (int j = 0; j < CPT; ++j) acc[i][j] = __fmaf_rn(b[j], a[i], acc[i][j]);
             }
         }
         __syncthreads();
     }
 
     float *h2s = tile;
+    const int ld = H2 + 1;
 #pragma unroll
-    for (int i = 0; i < RPT; ++i) {
-        const int r = warp + 8 * i;
+    for (int i = 0; i < 8; ++i) {
+        const int r = 8 * warp + i;
 #pragma unroll
         for (int j = 0; j < CPT; ++j) {
-            const int n = lane + 32 * j;
+            const int n = 128 * (j / VW) + VW * lane + j % VW;
             if (r < R && n < H2) {
                 const float v = acc[i][j];
-                h2s[r * w2ld + n] = v > 0.f ? v : 0.f;
+                h2s[r * ld + n] = v > 0.f ? v : 0.f;
             }
         }
     }
@@ -225,7 +334,7 @@ __device__ void pair_mlp(const Model &m, int R, const Rows &rows, const float *u
         const int r = e / m.NH, o = e - r * m.NH;
         const float *w3 = w3s + (size_t)o * H2;
         float z = m.b3[o];
-        for (int n = 0; n < H2; ++n) z = __fmaf_rn(w3[n], h2s[r * w2ld + n], z);
+        for (int n = 0; n < H2; ++n) z = __fmaf_rn(w3[n], h2s[r * ld + n], z);
         sp[e] = softplus_c(z);
     }
     __syncthreads();
@@ -245,7 +354,7 @@ __host__ __device__ inline int route_qb(int D) { return D >= 64 ? 1 : 64 / D; }
 
 struct RouteLayout {
     int QB, R;
-    size_t us, vs, ol, qual, sp, C, U, w3, tile, total;  // float offsets
+    size_t us, vs, ol, qual, sp, C, U, w3, w1q, tile, total;  // float offsets
 };
 
 __host__ __device__ inline RouteLayout route_layout(int D, int M, int H2) {
@@ -261,16 +370,18 @@ __host__ __device__ inline RouteLayout route_layout(int D, int M, int H2) {
     L.C = o; o += 64;
     L.U = o; o += 64;
     L.w3 = o; o += 3 * (size_t)H2;
+    L.w1q = o; o += 2 * (size_t)MAX_H;
     o = (o + 3) & ~(size_t)3;
     L.tile = o;
-    o += tile_floats_for<ROUTE_RPT>(H2);
+    o += tile_floats_for(H2);
     L.total = o;
     return L;
 }
 
 template <int CPT>
-__global__ void __launch_bounds__(SIMT_THREADS) k_route_simt(Model m, Queries q) {
-    extern __shared__ float sm[];
+__global__ void __launch_bounds__(SIMT_THREADS, CPT <= 4 ? 3 : 2) k_route_simt(Model m, Queries q) {
+    extern __shared__ float4 sm4[];
+    float *sm = reinterpret_cast<float *>(sm4);
     const RouteLayout L = route_layout(m.D, m.M, m.H2);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int D = m.D, M = m.M, F = m.F, QB = L.QB, R = L.R;
@@ -278,26 +389,24 @@ __global__ void __launch_bounds__(SIMT_THREADS) k_route_simt(Model m, Queries q)
     float *us = sm + L.us, *vs = sm + L.vs, *ol = sm + L.ol, *qual = sm + L.qual;
     float *sp = sm + L.sp, *Cs = sm + L.C, *Us = sm + L.U;
 
-    for (int qi = tid; qi < QB; qi += SIMT_THREADS) {
-        const int qq = q0 + qi;
-        float u = 0.f, v = 0.f, o = 0.f;
-        if (qq < q.Q) {
-            o = q.out_len[qq];
-            u = standardise(m.xform[F - 2], (double)q.in_len[qq], m.mu[F - 2], m.sd[F - 2]);
-            v = standardise(m.xform[F - 1], (double)o, m.mu[F - 1], m.sd[F - 1]);
-        }
-        us[qi] = u;
-        vs[qi] = v;
+    // the two query slots on two warps (their fp64 chains run side by side)
+    if (tid < QB) {
+        const int qq = q0 + tid;
+        us[tid] = qq < q.Q ? standardise(m.xform[F - 2], (double)q.in_len[qq], m.mu[F - 2], m.sd[F - 2])
+                           : 0.f;
+    } else if (tid >= 64 && tid < 64 + QB) {
+        const int qi = tid - 64, qq = q0 + qi;
+        const float o = qq < q.Q ? q.out_len[qq] : 0.f;
+        vs[qi] = qq < q.Q ? standardise(m.xform[F - 1], (double)o, m.mu[F - 1], m.sd[F - 1]) : 0.f;
         ol[qi] = o;
     }
     // quality, staged through the (not yet used) tile space
-    const float qv = quality_staged(m, q, q0, QB, sm + L.tile,
-                                    (int)tile_floats_for<ROUTE_RPT>(m.H2));
+    const float qv = quality_staged(m, q, q0, QB, sm + L.tile, (int)tile_floats_for(m.H2));
     if (tid < QB * M) qual[tid] = qv;
     __syncthreads();
 
     RouteRows rows{m.A, D, m.H1};
-    pair_mlp<ROUTE_RPT, CPT>(m, R, rows, us, vs, sm + L.tile, sm + L.w3, sp);
+    pair_mlp<CPT>(m, R, rows, us, vs, sm + L.tile, sm + L.w3, sm + L.w1q, sp);
 
     for (int r = tid; r < R; r += SIMT_THREADS) {
         const int qi = r / D, d = r - qi * D;
@@ -349,19 +458,13 @@ __host__ __device__ inline size_t tri_off(int D, int Qs, int c) {
 
 size_t seq_table_floats(int D, int Qs) { return tri_off(D, Qs, Qs); }
 
-struct SeqRows {
-    const float *pre;  // [2][H1] in shared memory
-    int H1, n1, c1, c2;
-    __device__ const float *prefix(int r) const { return r < n1 ? pre : pre + H1; }
-    __device__ int query(int r) const { return r < n1 ? c1 + r : c2 + (r - n1); }
-};
-
 // Per-chunk auxiliary arrays (one scratch buffer, seq_aux_floats floats):
-// quality [Qs][M], standardised query slots u [Qs] and v [Qs], and the
-// standardised running count of every deployment after c more picks,
-// xr [D][Qs + 1] (c = 0 .. Qs).
+// quality [Qs][M], standardised query slots u [Qs] and v [Qs], and, for every
+// deployment d and count c = 0 .. Qs of further picks, the standardised
+// running count xr [D][Qs + 1] and the layer-1 prefix through slot F - 3
+// pre [D][Qs + 1][H1] (the snapshot kernel's chain with running r_d + c).
 struct SeqAux {
-    float *qual, *us, *vs, *xr;
+    float *qual, *us, *vs, *xr, *pre;
 };
 
 __host__ __device__ inline SeqAux seq_aux(float *aux, int D, int M, int Qs) {
@@ -370,46 +473,80 @@ __host__ __device__ inline SeqAux seq_aux(float *aux, int D, int M, int Qs) {
     a.us = aux + (size_t)Qs * M;
     a.vs = a.us + Qs;
     a.xr = a.vs + Qs;
-    (void)D;
+    a.pre = a.xr + (((size_t)D * (Qs + 1) + 3) & ~(size_t)3);
     return a;
 }
 
-size_t seq_aux_floats(int D, int M, int Qs) {
-    return (size_t)Qs * M + 2 * (size_t)Qs + (size_t)D * (Qs + 1);
+size_t seq_aux_floats(int D, int M, int H1, int Qs) {
+    return (size_t)Qs * M + 2 * (size_t)Qs + (((size_t)D * (Qs + 1) + 3) & ~(size_t)3) +
+           (size_t)D * (Qs + 1) * H1;
 }
 
-// K_seq_prep: the chunk's standardised features, each computed once (double
-// arithmetic is scarce on this GPU; the table blocks would otherwise repeat it).
-__global__ void __launch_bounds__(32) k_seq_prep(Model m, Queries q, int Qs, float *aux) {
+// K_seq_prep: the chunk's standardised features and layer-1 prefixes, each
+// computed once (double arithmetic is scarce on this GPU, and every table
+// block would otherwise repeat it).  Blocks [0, nuv): the query slots; then
+// one block per (d, c).
+constexpr int PREP_THREADS = 128;
+
+__global__ void __launch_bounds__(PREP_THREADS) k_seq_prep(Model m, Queries q, int Qs, float *aux) {
     const SeqAux a = seq_aux(aux, m.D, m.M, Qs);
-    const int t = blockIdx.x * 32 + threadIdx.x, F = m.F, P = m.P;
-    if (t < Qs) {
-        a.us[t] = standardise(m.xform[F - 2], (double)q.in_len[t], m.mu[F - 2], m.sd[F - 2]);
-    } else if (t < 2 * Qs) {
-        const int i = t - Qs;
-        a.vs[i] = standardise(m.xform[F - 1], (double)q.out_len[i], m.mu[F - 1], m.sd[F - 1]);
-    } else if (t < 2 * Qs + m.D * (Qs + 1)) {
-        const int e = t - 2 * Qs, d = e / (Qs + 1), c = e - d * (Qs + 1);
-        a.xr[e] = standardise(m.xform[P + 1], (double)(m.running[d] + c), m.mu[P + 1],
-                              m.sd[P + 1]);
+    const int tid = threadIdx.x, F = m.F, P = m.P, H1 = m.H1;
+    const int nuv = (2 * Qs + PREP_THREADS - 1) / PREP_THREADS;
+    if ((int)blockIdx.x < nuv) {
+        const int t = blockIdx.x * PREP_THREADS + tid;
+        if (t < Qs) {
+            a.us[t] = standardise(m.xform[F - 2], (double)q.in_len[t], m.mu[F - 2], m.sd[F - 2]);
+        } else if (t < 2 * Qs) {
+            const int i = t - Qs;
+            a.vs[i] = standardise(m.xform[F - 1], (double)q.out_len[i], m.mu[F - 1], m.sd[F - 1]);
+        }
+        return;
+    }
+    const int g = blockIdx.x - nuv, d = g / (Qs + 1), c = g - d * (Qs + 1);
+    __shared__ float xr;
+    if (tid == 0) {
+        xr = standardise(m.xform[P + 1], (double)(m.running[d] + c), m.mu[P + 1], m.sd[P + 1]);
+        a.xr[g] = xr;
+    }
+    __syncthreads();
+    // continue the chain from slot P + 1 (running) with the deployment's other features
+    for (int j = tid; j < H1; j += PREP_THREADS) {
+        const float *w = m.W1 + (size_t)j * F;
+        const float *x = m.X + (size_t)d * F;
+        float acc = m.Spre[(size_t)d * H1 + j];
+        acc = __fmaf_rn(w[P + 1], xr, acc);
+        for (int k = P + 2; k < F - 2; ++k) acc = __fmaf_rn(w[k], x[k], acc);
+        a.pre[(size_t)g * H1 + j] = acc;
     }
 }
 
-struct SeqLayout {
-    size_t us, vs, pre, sp, w3, tile, total;
+// Table rows of one block: row r is table entry t0 + r, i.e. (c, d, i) with
+// prefix pre[d][c] and query slot i (decoded into shared memory).
+struct FlatRows {
+    const float *pre;
+    const int *gi, *qi;
+    int H1;
+    __device__ const float *prefix(int r) const { return pre + (size_t)gi[r] * H1; }
+    __device__ int query(int r) const { return qi[r]; }
 };
 
-__host__ __device__ inline SeqLayout seq_layout(int H1, int H2) {
+struct SeqLayout {
+    size_t us, vs, gi, qi, sp, w3, w1q, tile, total;
+};
+
+__host__ __device__ inline SeqLayout seq_layout(int H2) {
     SeqLayout L;
     size_t o = 0;
     L.us = o; o += SEQ_MAX_CHUNK;
     L.vs = o; o += SEQ_MAX_CHUNK;
-    L.pre = o; o += 2 * (size_t)H1;
-    L.sp = o; o += 3 * 8 * SEQ_RPT;
+    L.gi = o; o += TILE_ROWS;
+    L.qi = o; o += TILE_ROWS;
+    L.sp = o; o += 3 * TILE_ROWS;
     L.w3 = o; o += 3 * (size_t)H2;
+    L.w1q = o; o += 2 * (size_t)MAX_H;
     o = (o + 3) & ~(size_t)3;
     L.tile = o;
-    o += tile_floats_for<SEQ_RPT>(H2);
+    o += tile_floats_for(H2);
     L.total = o;
     return L;
 }
@@ -420,77 +557,69 @@ __host__ __device__ inline int seq_qual_rows(int M) {
     return n < 1 ? 1 : (n > 8 ? 8 : n);
 }
 
+// K_seq_table: blocks [0, nb_qual) compute the chunk's quality; the others
+// take rows_per_block consecutive table entries each (the last block fewer),
+// so that every SM gets the same number of rows.
 template <int CPT>
-__global__ void __launch_bounds__(SIMT_THREADS, CPT <= 4 ? 4 : 2)
-k_seq_table(Model m, Queries q, int Qs, int nb_table, float *ctab, float *aux) {
-    extern __shared__ float sm[];
+__global__ void __launch_bounds__(SIMT_THREADS, CPT <= 4 ? 3 : 2)
+k_seq_table(Model m, Queries q, int Qs, int nb_qual, int rows_per_block, float *ctab,
+            float *aux) {
+    extern __shared__ float4 sm4[];
+    float *sm = reinterpret_cast<float *>(sm4);
     const int tid = threadIdx.x;
-    const int D = m.D, F = m.F, H1 = m.H1, M = m.M, P = m.P;
-    const SeqLayout L = seq_layout(H1, m.H2);
+    const int D = m.D, M = m.M;
+    const SeqLayout L = seq_layout(m.H2);
     const SeqAux A = seq_aux(aux, D, M, Qs);
-    if ((int)blockIdx.x >= nb_table) {
+    if ((int)blockIdx.x < nb_qual) {
         // quality of the chunk's queries [q0, q0 + nq), staged through the whole
         // shared space
-        const int nq = seq_qual_rows(M), q0 = ((int)blockIdx.x - nb_table) * nq;
+        const int nq = seq_qual_rows(M), q0 = (int)blockIdx.x * nq;
         const float v = quality_staged(m, q, q0, nq, sm, (int)L.total);
         if (tid < nq * M && q0 + tid / M < Qs) A.qual[(size_t)q0 * M + tid] = v;
         return;
     }
-    float *us = sm + L.us, *vs = sm + L.vs, *pre = sm + L.pre, *sp = sm + L.sp;
-    const int d = blockIdx.x % D, c1 = blockIdx.x / D, c2 = Qs - 1 - c1;
-    const bool two = c2 != c1;
-    const int n1 = Qs - c1, R = n1 + (two ? c1 + 1 : 0);
-
-    // standardised query slots of the rows of this block (queries c1 .. Qs - 1)
-    for (int i = c1 + tid; i < Qs; i += SIMT_THREADS) {
+    const int T = (int)tri_off(D, Qs, Qs);
+    const int t0 = ((int)blockIdx.x - nb_qual) * rows_per_block;
+    const int R = min(rows_per_block, T - t0);
+    float *us = sm + L.us, *vs = sm + L.vs, *sp = sm + L.sp;
+    int *gi = reinterpret_cast<int *>(sm + L.gi), *qi = reinterpret_cast<int *>(sm + L.qi);
+    for (int i = tid; i < Qs; i += SIMT_THREADS) {
         us[i] = A.us[i];
         vs[i] = A.vs[i];
     }
-    // layer-1 prefixes for running counts r_d + c1 and r_d + c2: continue the
-    // chain from slot P + 1 (running) with the deployment's other features;
-    // the two chains share their operands
-    const float xa = A.xr[(size_t)d * (Qs + 1) + c1], xb = A.xr[(size_t)d * (Qs + 1) + c2];
-    for (int j = tid; j < H1; j += SIMT_THREADS) {
-        const float *w = m.W1 + (size_t)j * F;
-        const float *x = m.X + (size_t)d * F;
-        const float s0 = m.Spre[(size_t)d * H1 + j], wr = w[P + 1];
-        float a1 = __fmaf_rn(wr, xa, s0);
-        float a2 = __fmaf_rn(wr, xb, s0);
-#pragma unroll 8
-        for (int k = P + 2; k < F - 2; ++k) {
-            const float wk = w[k], xk = x[k];
-            a1 = __fmaf_rn(wk, xk, a1);
-            a2 = __fmaf_rn(wk, xk, a2);
+    for (int r = tid; r < R; r += SIMT_THREADS) {
+        // entry t: the count c with tri_off(c) <= t < tri_off(c + 1), then d and i
+        const int t = t0 + r;
+        int lo = 0, hi = Qs - 1;
+        while (lo < hi) {
+            const int mid = (lo + hi + 1) >> 1;
+            if ((int)tri_off(D, Qs, mid) <= t) lo = mid;
+            else hi = mid - 1;
         }
-        pre[j] = a1;
-        if (two) pre[H1 + j] = a2;
+        const int off = t - (int)tri_off(D, Qs, lo), len = Qs - lo, d = off / len;
+        gi[r] = d * (Qs + 1) + lo;
+        qi[r] = lo + off - d * len;
     }
     __syncthreads();
 
-    SeqRows rows{pre, H1, n1, c1, c2};
-    pair_mlp<SEQ_RPT, CPT>(m, R, rows, us, vs, sm + L.tile, sm + L.w3, sp);
+    FlatRows rows{A.pre, gi, qi, m.H1};
+    pair_mlp<CPT>(m, R, rows, us, vs, sm + L.tile, sm + L.w3, sm + L.w1q, sp);
 
     for (int r = tid; r < R; r += SIMT_THREADS) {
-        const int c = r < n1 ? c1 : c2, i = rows.query(r);
         const float *h = sp + m.NH * r;
-        const float C = __fmaf_rn(m.NH == 3 ? h[2] : q.out_len[i], h[1], h[0]);
-        ctab[tri_off(D, Qs, c) + (size_t)d * (Qs - c) + (i - c)] = C;
+        ctab[t0 + r] = __fmaf_rn(m.NH == 3 ? h[2] : q.out_len[qi[r]], h[1], h[0]);
     }
 }
 
 // Chain shared memory (4-byte words): dep_model and picks [MAX_D] ints each,
 // the table [T rounded up to 4] (16-byte aligned), the chunk's quality
 // [Qs][M], budgets [Qs] and the walk's outputs (chosen, latency, utility)
-// [3][Qs].  After the walk the refresh reuses the space from the table on:
-// standardised running counts [MAX_D], deployment slots P + 2 .. F - 3
-// [D][F - P - 4], W1 columns P + 1 .. F - 3 [H1][odd stride].
+// [3][Qs].
 constexpr int CHAIN_THREADS = 1024;
 
 __host__ __device__ inline size_t chain_tab_floats(int D, int Qs) {
     return (tri_off(D, Qs, Qs) + 3) & ~(size_t)3;
 }
-
-__host__ __device__ inline int refresh_ld(int F, int P) { return (F - P - 3) | 1; }
 
 // Offset of the table entry (picks c, deployment d, query 0) (only i >= c is stored).
 __device__ __forceinline__ int tab_row(int D, int Qs, int c, int d) {
@@ -647,33 +776,18 @@ k_seq_chain(Model m, Queries q, int Qs, const float *ctab, float *aux) {
     }
     __syncthreads();
 
-    // persist the picks and refresh the state they touch (standardised running
-    // count, layer-1 prefix): the snapshot kernel's chains, operands staged
-    const int nk = F - P - 3, wld = refresh_ld(F, P);
-    float *xr = tab, *xs = xr + MAX_D, *w1s = xs + (size_t)D * (nk - 1);
+    // persist the picks and refresh the state they touch: the standardised
+    // running count and the layer-1 prefix are the preparation kernel's values
+    // for the final count
     for (int d = tid; d < D; d += CHAIN_THREADS) {
-        const float x = A.xr[(size_t)d * (Qs + 1) + cnt[d]];
         m.running[d] += cnt[d];
-        xr[d] = x;
-        m.X[(size_t)d * F + P + 1] = x;
+        m.X[(size_t)d * F + P + 1] = A.xr[(size_t)d * (Qs + 1) + cnt[d]];
     }
-    for (int e = tid; e < D * (nk - 1); e += CHAIN_THREADS) {
-        const int d = e / (nk - 1), k = e - d * (nk - 1);
-        xs[e] = m.X[(size_t)d * F + P + 2 + k];
-    }
-    for (int e = tid; e < H1 * nk; e += CHAIN_THREADS) {
-        const int j = e / nk, k = e - j * nk;
-        w1s[j * wld + k] = m.W1[(size_t)j * F + P + 1 + k];
-    }
-    __syncthreads();
     for (int e = tid; e < D * H1; e += CHAIN_THREADS) {
         const int d = e / H1, j = e - d * H1;
-        const float *w = w1s + j * wld, *x = xs + (size_t)d * (nk - 1);
-        float acc = m.Spre[e];
-        acc = __fmaf_rn(w[0], xr[d], acc);
-        for (int k = 1; k < nk; ++k) acc = __fmaf_rn(w[k], x[k - 1], acc);
-        m.A[e] = acc;
-        m.Abf[e] = __bfloat16_as_ushort(__float2bfloat16_rn(acc));
+        const float v = A.pre[((size_t)d * (Qs + 1) + cnt[d]) * H1 + j];
+        m.A[e] = v;
+        m.Abf[e] = __bfloat16_as_ushort(__float2bfloat16_rn(v));
     }
 }
 
@@ -686,7 +800,6 @@ k_seq_chain(Model m, Queries q, int Qs, const float *ctab, float *aux) {
 // decision maker.  Same canonical order as the kernels above.
 
 struct PairArgs {
-    const float *W2T;   // [H1][H2]: W2 transposed
     float *pairC;       // [Q][D] scratch
     float *qualS;       // [Q][M] scratch
     int32_t *count;     // [Q] arrivals, zero between calls
@@ -751,11 +864,11 @@ __global__ void __launch_bounds__(SIMT_THREADS) k_route_pairs(Model m, Queries q
             float acc = m.b2[n];
             float w[32], wn[32];
 #pragma unroll
-            for (int j = 0; j < 32; ++j) w[j] = j < H1 ? a.W2T[(size_t)j * H2 + n] : 0.f;
+            for (int j = 0; j < 32; ++j) w[j] = j < H1 ? m.W2T[(size_t)j * m.H2p + n] : 0.f;
             for (int k0 = 0; k0 < H1; k0 += 32) {
 #pragma unroll
                 for (int j = 0; j < 32; ++j)
-                    wn[j] = k0 + 32 + j < H1 ? a.W2T[(size_t)(k0 + 32 + j) * H2 + n] : 0.f;
+                    wn[j] = k0 + 32 + j < H1 ? m.W2T[(size_t)(k0 + 32 + j) * m.H2p + n] : 0.f;
 #pragma unroll
                 for (int j = 0; j < 32; ++j)
                     if (k0 + j < H1) acc = __fmaf_rn(w[j], h1[k0 + j], acc);
@@ -851,17 +964,13 @@ size_t route_simt_smem(const Model &m) {
 }
 
 size_t seq_table_smem(const Model &m) {
-    return seq_layout(m.H1, m.H2).total * sizeof(float);
+    return seq_layout(m.H2).total * sizeof(float);
 }
 
 static size_t chain_smem(int D, int M, int Qs) {
     return (2 * MAX_D + chain_tab_floats(D, Qs) + (size_t)Qs * M + 4 * (size_t)Qs) * sizeof(float);
 }
 
-static size_t refresh_smem(const Model &m) {
-    return (2 * MAX_D + MAX_D + (size_t)m.D * (m.F - m.P - 4) +
-            (size_t)m.H1 * refresh_ld(m.F, m.P)) * sizeof(float);
-}
 
 int seq_chunk(const Model &m) {
     int Qs = SEQ_MAX_CHUNK;
@@ -915,11 +1024,10 @@ size_t route_pairs_smem(const Model &m) {
     return pair > qual ? pair : qual;
 }
 
-cudaError_t launch_route_pairs(const Model &m, const Queries &q, const float *W2T, float *pairC,
+cudaError_t launch_route_pairs(const Model &m, const Queries &q, float *pairC,
                                float *qualS, int32_t *count, cudaStream_t s) {
     if (q.Q <= 0) return cudaSuccess;
     PairArgs a;
-    a.W2T = W2T;
     a.pairC = pairC;
     a.qualS = qualS;
     a.count = count;
@@ -939,27 +1047,48 @@ cudaError_t launch_select_multi(const Model &m, const Queries &q, const float *C
     return cudaGetLastError();
 }
 
-cudaError_t launch_seq_table(const Model &m, const Queries &q, int Qs, float *ctab,
+cudaError_t launch_seq_table(const Model &m, const Queries &q, int Qs, int slots, float *ctab,
                              float *aux, cudaStream_t s) {
-    const int np = 2 * Qs + m.D * (Qs + 1);
-    k_seq_prep<<<(np + 31) / 32, 32, 0, s>>>(m, q, Qs, aux);
-    const int nb_table = m.D * ((Qs + 1) / 2);
+    const int nuv = (2 * Qs + PREP_THREADS - 1) / PREP_THREADS;
+    k_seq_prep<<<nuv + m.D * (Qs + 1), PREP_THREADS, 0, s>>>(m, q, Qs, aux);
+    // rows per table block: a multiple of 8 (whole warps of the tile) that
+    // spreads the table evenly over the blocks resident at once
+    const int T = (int)tri_off(m.D, Qs, Qs);
     const int nb_qual = (Qs + seq_qual_rows(m.M) - 1) / seq_qual_rows(m.M);
-    const size_t smem = seq_layout(m.H1, m.H2).total * sizeof(float);
-    const int blocks = nb_table + nb_qual;
+    const int want = slots - nb_qual > 1 ? slots - nb_qual : 1;
+    int rpb = ((T + want - 1) / want + 7) / 8 * 8;
+    rpb = rpb < 8 ? 8 : (rpb > TILE_ROWS ? TILE_ROWS : rpb);
+    const int blocks = nb_qual + (T + rpb - 1) / rpb;
+    const size_t smem = seq_layout(m.H2).total * sizeof(float);
     switch (cpt_for(m.H2)) {
-        case 1: k_seq_table<1><<<blocks, SIMT_THREADS, smem, s>>>(m, q, Qs, nb_table, ctab, aux); break;
-        case 2: k_seq_table<2><<<blocks, SIMT_THREADS, smem, s>>>(m, q, Qs, nb_table, ctab, aux); break;
-        case 4: k_seq_table<4><<<blocks, SIMT_THREADS, smem, s>>>(m, q, Qs, nb_table, ctab, aux); break;
-        default: k_seq_table<8><<<blocks, SIMT_THREADS, smem, s>>>(m, q, Qs, nb_table, ctab, aux); break;
+        case 1: k_seq_table<1><<<blocks, SIMT_THREADS, smem, s>>>(m, q, Qs, nb_qual, rpb, ctab, aux); break;
+        case 2: k_seq_table<2><<<blocks, SIMT_THREADS, smem, s>>>(m, q, Qs, nb_qual, rpb, ctab, aux); break;
+        case 4: k_seq_table<4><<<blocks, SIMT_THREADS, smem, s>>>(m, q, Qs, nb_qual, rpb, ctab, aux); break;
+        default: k_seq_table<8><<<blocks, SIMT_THREADS, smem, s>>>(m, q, Qs, nb_qual, rpb, ctab, aux); break;
     }
     return cudaGetLastError();
 }
 
+int seq_table_slots(const Model &m) {
+    int dev = 0, nsm = 0, per = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+        return 1;
+    const size_t smem = seq_layout(m.H2).total * sizeof(float);
+    cudaError_t e;
+    switch (cpt_for(m.H2)) {
+        case 1: e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per, k_seq_table<1>, SIMT_THREADS, smem); break;
+        case 2: e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per, k_seq_table<2>, SIMT_THREADS, smem); break;
+        case 4: e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per, k_seq_table<4>, SIMT_THREADS, smem); break;
+        default: e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per, k_seq_table<8>, SIMT_THREADS, smem); break;
+    }
+    if (e != cudaSuccess || per < 1) per = 1;
+    return nsm * per;
+}
+
 cudaError_t launch_seq_chain(const Model &m, const Queries &q, int Qs, const float *ctab,
                              float *aux, cudaStream_t s) {
-    const size_t a = chain_smem(m.D, m.M, Qs), b = refresh_smem(m);
-    k_seq_chain<<<1, CHAIN_THREADS, a > b ? a : b, s>>>(m, q, Qs, ctab, aux);
+    k_seq_chain<<<1, CHAIN_THREADS, chain_smem(m.D, m.M, Qs), s>>>(m, q, Qs, ctab, aux);
     return cudaGetLastError();
 }
 
