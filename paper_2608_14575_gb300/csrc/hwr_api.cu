@@ -71,6 +71,7 @@ struct hwr_ctx {
     float *memb = nullptr;
     float *W1q = nullptr;            // [2][H1]
     float *W2T = nullptr;            // [H1][H2p] fp32 (rows zero-padded), for the SIMT tiles
+    float *W1T = nullptr;            // [F][H1] fp32, W1 slot-major
     uint16_t *W2img = nullptr, *membimg = nullptr;
     std::vector<char> head_consts;   // output-layer constants for the tensor path
     int32_t *running = nullptr, *waiting = nullptr;
@@ -228,7 +229,7 @@ static Model model_view(const hwr_ctx *c) {
     m.E = c->E; m.P = c->P; m.NH = c->NH;
     m.dep_model = c->dep_model; m.dep_gpu = c->dep_gpu; m.log10p = c->log10p;
     m.W1 = c->W1; m.b1 = c->b1; m.W2 = c->W2; m.b2 = c->b2; m.W3 = c->W3; m.b3 = c->b3;
-    m.W2T = c->W2T; m.H2p = (c->H2 + 3) & ~3;
+    m.W2T = c->W2T; m.H2p = (c->H2 + 3) & ~3; m.W1T = c->W1T;
     m.mu = c->mu; m.sd = c->sd; m.xform = c->xform; m.memb = c->memb;
     m.running = c->running; m.waiting = c->waiting; m.kv = c->kv;
     m.gpu_util = c->gpu_util; m.ttft = c->ttft; m.tpot = c->tpot;
@@ -407,6 +408,7 @@ static hwr_status build_ctx(hwr_ctx *c, const hwr_deployment_table *t, const hwr
     TRY(dev_alloc(c, &c->W1q, 2 * (size_t)H1));
     const int H2p = (H2 + 3) & ~3;
     TRY(dev_alloc(c, &c->W2T, (size_t)H1 * H2p));
+    TRY(dev_alloc(c, &c->W1T, (size_t)F * H1));
     TRY(dev_alloc(c, &c->pairC, (size_t)PAIRS_MAX_PAIRS));
     TRY(dev_alloc(c, &c->pairQ, (size_t)PAIRS_MAX_PAIRS * M));
     TRY(dev_alloc(c, &c->pairN, (size_t)PAIRS_MAX_PAIRS));
@@ -446,6 +448,10 @@ static hwr_status build_ctx(hwr_ctx *c, const hwr_deployment_table *t, const hwr
     for (int n = 0; n < H2; ++n)
         for (int k = 0; k < H1; ++k) w2t[(size_t)k * H2p + n] = w2[(size_t)n * H1 + k];
     TRY(upload(c, c->W2T, w2t.data(), w2t.size() * 4, "upload W2 transposed"));
+    std::vector<float> w1t((size_t)F * H1);
+    for (int j = 0; j < H1; ++j)
+        for (int k = 0; k < F; ++k) w1t[(size_t)k * H1 + j] = w1[(size_t)j * F + k];
+    TRY(upload(c, c->W1T, w1t.data(), w1t.size() * 4, "upload W1 transposed"));
     CK(c, cudaMemset(c->pairN, 0, PAIRS_MAX_PAIRS * sizeof(int32_t)), "zero counters");
     c->mu_in = p->feat_mean[F - 2]; c->sd_in = p->feat_std[F - 2]; c->xf_in = p->feat_xform[F - 2];
     c->mu_out = p->feat_mean[F - 1]; c->sd_out = p->feat_std[F - 1]; c->xf_out = p->feat_xform[F - 1];

@@ -27,6 +27,7 @@ struct Model {
     const int32_t *dep_gpu;     // [D]
     const float *log10p;        // [M]
     const float *W1, *b1;       // [H1][F], [H1]   fp32 (bf16 widened)
+    const float *W1T;           // [F][H1]: W1 transposed (slot-major, coalesced per slot)
     const float *W2, *b2;       // [H2][H1], [H2]
     const float *W2T;           // [H1][H2p]: W2 transposed, rows zero-padded to H2p
     int H2p;                    // H2 rounded up to a multiple of 4 (16-byte rows)

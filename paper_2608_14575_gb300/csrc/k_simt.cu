@@ -161,12 +161,12 @@ __global__ void __launch_bounds__(SIMT_THREADS) k_snapshot(Model m) {
     }
     __syncthreads();
     for (int j = threadIdx.x; j < m.H1; j += blockDim.x) {
-        const float *w = m.W1 + (size_t)j * m.F;
+        const float *w = m.W1T + j;   // slot k at w[k * H1]
         float acc = m.b1[j];
         int k = 0;
-        for (; k <= m.P; ++k) acc = __fmaf_rn(w[k], xs[k], acc);
+        for (; k <= m.P; ++k) acc = __fmaf_rn(w[(size_t)k * m.H1], xs[k], acc);
         m.Spre[(size_t)d * m.H1 + j] = acc;
-        for (; k < m.F - 2; ++k) acc = __fmaf_rn(w[k], xs[k], acc);
+        for (; k < m.F - 2; ++k) acc = __fmaf_rn(w[(size_t)k * m.H1], xs[k], acc);
         m.A[(size_t)d * m.H1 + j] = acc;
         m.Abf[(size_t)d * m.H1 + j] = __bfloat16_as_ushort(__float2bfloat16_rn(acc));
     }
@@ -510,12 +510,12 @@ __global__ void __launch_bounds__(PREP_THREADS) k_seq_prep(Model m, Queries q, i
     }
     __syncthreads();
     // continue the chain from slot P + 1 (running) with the deployment's other features
+    // (W1 read slot-major: a warp's loads of one slot are contiguous)
     for (int j = tid; j < H1; j += PREP_THREADS) {
-        const float *w = m.W1 + (size_t)j * F;
         const float *x = m.X + (size_t)d * F;
         float acc = m.Spre[(size_t)d * H1 + j];
-        acc = __fmaf_rn(w[P + 1], xr, acc);
-        for (int k = P + 2; k < F - 2; ++k) acc = __fmaf_rn(w[k], x[k], acc);
+        acc = __fmaf_rn(m.W1T[(size_t)(P + 1) * H1 + j], xr, acc);
+        for (int k = P + 2; k < F - 2; ++k) acc = __fmaf_rn(m.W1T[(size_t)k * H1 + j], x[k], acc);
         a.pre[(size_t)g * H1 + j] = acc;
     }
 }
