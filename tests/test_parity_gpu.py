@@ -314,3 +314,26 @@ def test_exact_ties_go_to_lowest_index(monkeypatch, slo, mode):
     want = O.Problem(p).route(slo=slo, mode=O.F32, sequential=bool(flags), nthreads=8)
     assert_exact(got, want, f"ties {mode} slo={slo}")
     assert np.all((got[0] >= 0) & (got[0] < p["G"]))
+
+
+# ---------------------------------------------------------------------------
+# widths the SIMT tile pads: H2 not a multiple of 4 (padded rows of W2
+# transposed), H1 not a multiple of the 32-wide K chunk, width 1, the widest
+# columns, on the pair-parallel, fused and sequential paths
+
+@pytest.mark.parametrize("shape", [
+    dict(M=2, G=2, F=13, H1=37, H2=30, E=24),
+    dict(M=3, G=2, F=16, H1=1, H2=1, E=8),
+    dict(M=2, G=3, F=20, H1=250, H2=253, E=16),
+])
+@pytest.mark.parametrize("mode", ["pairs", "fused", "sequential"])
+def test_odd_widths_exact(monkeypatch, shape, mode):
+    Q = 45
+    p = W.make_problem(Q=Q, dtype="f32", lam=0.35, slo=2.5, seed=77, bias_std=0.25, **shape)
+    monkeypatch.setenv("HWR_PAIRS_MAX_PAIRS", "0" if mode == "fused" else "2048")
+    flags = H.HWR_SEQUENTIAL if mode == "sequential" else 0
+    r = H.Router(p)
+    got = r.route(flags=flags)
+    r.close()
+    want = O.Problem(p).route(mode=O.F32, sequential=bool(flags), nthreads=8)
+    assert_exact(got, want, f"{shape} {mode}")
