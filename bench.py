@@ -241,7 +241,7 @@ def run_reference(args, p):
     print(json.dumps(line), flush=True)
 
 
-def q1_latency(H, iters=2000):
+def q1_latency(H, iters=10_000):
     """p50/p99 of one-query routes through the C ABI with pinned host buffers."""
     import torch
     p = W.make_config(4, Q=1024)
@@ -268,6 +268,57 @@ def q1_latency(H, iters=2000):
             "calls": iters, "config": "D=32 (8 models x 4 GPU types), MLP 48->256->256->2, "
                                       "E=1024 bf16, host buffers, end to end",
             "paper_routing_overhead_us": 200.0}
+
+
+def config_latencies(H, stream, dev, calls=300):
+    """Per-call latency of the other workloads: the small fp32 batch and the mid
+    bf16 batch (device pointers, isolated calls, CUDA events) and a 64-request
+    micro-batch of the online sequential workload (snapshot upload + sequential
+    route through the C ABI with host buffers, wall clock)."""
+    import torch
+    out = {}
+    for c in (0, 1):
+        p = W.make_config(c)
+        r = H.Router(p, stream=stream.cuda_stream)
+        emb = p["emb"].view(np.int16) if p["dtype"] == "bf16" else p["emb"]
+        args = (torch.from_numpy(p["in_len"]).to(dev), torch.from_numpy(p["out_len"]).to(dev),
+                torch.from_numpy(emb).to(dev), torch.empty(p["Q"], dtype=torch.int32, device=dev),
+                torch.empty(p["Q"], dtype=torch.float32, device=dev),
+                torch.empty(p["Q"], dtype=torch.float32, device=dev))
+        for _ in range(20):
+            r.route_device(*args, slo=p["slo"], lam=p["lam"])
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(calls)]
+        for e0, e1 in ev:
+            e0.record(stream)
+            r.route_device(*args, slo=p["slo"], lam=p["lam"])
+            e1.record(stream)
+        torch.cuda.synchronize()
+        t = np.array([a.elapsed_time(b) for a, b in ev]) * 1e3
+        r.close()
+        out[f"config{c}"] = {"workload": workload_name(p), "calls": calls,
+                             "p50_us": float(np.median(t)), "p99_us": float(np.percentile(t, 99)),
+                             "queries_per_s": float(p["Q"] / (np.median(t) * 1e-6))}
+    p = W.make_config(2, Q=64 * 200)
+    r = H.Router(p)
+    n, times = 64, []
+    for k in range(220):
+        lo = (k % 200) * n
+        t = time.perf_counter()
+        r.update_snapshot(p["snap"])
+        r.route(p["in_len"][lo:lo + n], p["out_len"][lo:lo + n], p["emb"][lo:lo + n],
+                flags=H.HWR_SEQUENTIAL)
+        if k >= 20:
+            times.append(time.perf_counter() - t)
+    r.close()
+    a = np.array(times) * 1e6
+    out["config2"] = {"workload": workload_name(p) + ", micro-batches of 64, sequential",
+                      "calls": len(a), "p50_us": float(np.median(a)),
+                      "p99_us": float(np.percentile(a, 99)),
+                      "requests_per_s": float(n / (np.median(a) * 1e-6)),
+                      "note": "snapshot upload + sequential route of one micro-batch, "
+                              "host buffers, wall clock"}
+    return out
 
 
 # Online scenarios on the online sequential workload's shapes (D = 12).  The
@@ -311,6 +362,7 @@ def online_report(args):
                 "route_call_us": {"p50": float(np.percentile(us, 50)),
                                   "p99": float(np.percentile(us, 99)),
                                   "mean_batch": float(sizes[sizes > 0].mean()),
+                                  "requests_per_s": float(sizes.sum() / (us.sum() * 1e-6)),
                                   "note": "snapshot upload + sequential route of one "
                                           "micro-batch, host buffers, wall clock"}}),
                 flush=True)
@@ -421,6 +473,7 @@ def main():
     ap.add_argument("--no-clocks", action="store_true")
     ap.add_argument("--no-multi", action="store_true")
     ap.add_argument("--no-sweep", action="store_true")
+    ap.add_argument("--no-configs", action="store_true")
     ap.add_argument("--online", action="store_true",
                     help="print the online evaluation metrics instead of the throughput line")
     args = ap.parse_args()
@@ -581,6 +634,8 @@ def main():
         line["sweep_d32"] = sweep_d32(H, stream, dev)
     if rank == 0 and not args.no_q1:
         line["q1_latency_us"] = q1_latency(H)
+    if rank == 0 and not args.no_configs:
+        line["configs"] = config_latencies(H, stream, dev)
     if rank == 0 and not args.no_cpu:
         cores = len(os.sched_getaffinity(0))
         v, n, dt = cpu_oracle_rate(p, 10.0, cores)

@@ -35,15 +35,16 @@ struct AllocHook {
 // batches of at most pairs_max pairs (Q * D) take the small-batch SIMT
 // kernel; larger bf16 batches of at least tc_min_pairs pairs take the
 // tensor-core kernels; the rest the fused SIMT kernel.  pairs_max is
-// SMALL_MAX_PAIRS where the tensor-core path exists and PAIRS_MAX_PAIRS
-// (the small-batch kernel's limit) otherwise: without tensor cores the
-// small-batch kernel stays ahead of the fused one up to that limit.
-// (bf16, device pointers, isolated calls: the tensor path costs 31-33 us at
-// D = 32 and 38-40 us at D = 64 for 1 to 64 queries; the small-batch kernel
-// is ahead up to 256 pairs and behind from 512 on.)
+// SMALL_MAX_PAIRS where the tensor-core path exists and FP32_MAX_PAIRS
+// otherwise.  (Device pointers, isolated calls.  bf16: the tensor path costs
+// 31-33 us at D = 32 and 38-40 us at D = 64 for 1 to 64 queries; the
+// small-batch kernel is ahead up to 256 pairs and behind from 512 on.  fp32:
+// the fused kernel costs ~23.5 us at H = 32 and ~38 us at H = 128 from 1 to
+// 512 queries; the small-batch kernel is ahead up to 384-512 pairs.)
 constexpr int TC_MIN_PAIRS = 257;
 constexpr int PIPE_CHUNK_MIN = 8192;   // smallest chunk of a pipelined host batch
 constexpr int SMALL_MAX_PAIRS = 256;
+constexpr int FP32_MAX_PAIRS = 512;
 
 }  // namespace
 
@@ -555,7 +556,7 @@ extern "C" hwr_status hwr_create(const hwr_deployment_table *table, const hwr_pr
         free_ctx(c);
         return s;
     }
-    if (c->pairs_max < 0) c->pairs_max = c->tc_ok ? SMALL_MAX_PAIRS : PAIRS_MAX_PAIRS;
+    if (c->pairs_max < 0) c->pairs_max = c->tc_ok ? SMALL_MAX_PAIRS : FP32_MAX_PAIRS;
     *out = c;
     return HWR_OK;
 }
