@@ -79,10 +79,21 @@ __device__ __forceinline__ float emb_at(const void *emb, int bf16, size_t i) {
 // chains read shared memory only.  Every thread of the block calls this;
 // thread t < nq * M returns the score of query t / M, model t % M (rows at or
 // past q.Q give sigmoid(0)), the others return 0.  Ends with the stage free
-// for reuse after a barrier.
-__device__ float quality_staged(const Model &m, const Queries &q, int q0, int nq, float *stage,
-                                int stage_floats) {
-    const int tid = threadIdx.x, M = m.M, E = m.E;
+// for reuse after a barrier.  NT threads take part: the whole block
+// (NT = SIMT_THREADS, block barriers, thread index t = threadIdx.x) or one
+// warp (NT = 32, warp barriers, t = lane), which then runs the chains
+// t, t + 32 (CH = 2: at most 64 (query, model) pairs) and returns the score of
+// chain t + 32 j in res[j].
+template <int NT>
+__device__ __forceinline__ void group_sync() {
+    if constexpr (NT == 32) __syncwarp();
+    else __syncthreads();
+}
+
+template <int NT, int CH>
+__device__ void quality_group(const Model &m, const Queries &q, int q0, int nq, float *stage,
+                              int stage_floats, int t, float (&res)[CH]) {
+    const int tid = t, M = m.M, E = m.E;
     const int es = q.emb_bf16 ? 2 : 4;
     const bool async = ((uintptr_t)q.emb & 15) == 0;
     // row stride ld (elements): 16-byte rows whose 4-byte word stride is 4
@@ -96,15 +107,16 @@ __device__ float quality_staged(const Model &m, const Queries &q, int q0, int nq
     const int ld = stride(ek);
     char *er = reinterpret_cast<char *>(stage);
     float *mb = reinterpret_cast<float *>(er + (((size_t)nq * ld * es + 15) & ~(size_t)15));
-    const int qi = tid / M, mi = tid - qi * M;
-    float s = 0.f;
+    float s[CH];
+#pragma unroll
+    for (int j = 0; j < CH; ++j) s[j] = 0.f;
     for (int k0 = 0; k0 < E; k0 += ek) {
         const int kc = min(ek, E - k0);
-        __syncthreads();
+        group_sync<NT>();
         if (async) {
             const int gpr = kc * es / 16;     // granules per row (kc is a multiple of 8)
             const uint32_t eb = (uint32_t)__cvta_generic_to_shared(er);
-            for (int g = tid; g < nq * gpr; g += SIMT_THREADS) {
+            for (int g = tid; g < nq * gpr; g += NT) {
                 const int i = g / gpr, c = g - i * gpr, qq = q0 + i;
                 const char *src = (const char *)q.emb + ((size_t)(qq < q.Q ? qq : 0) * E + k0) * es + 16 * c;
                 asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(
@@ -113,37 +125,51 @@ __device__ float quality_staged(const Model &m, const Queries &q, int q0, int nq
                              : "memory");
             }
             const uint32_t mbs = (uint32_t)__cvta_generic_to_shared(mb);
-            for (int g = tid; g < kc * M / 4; g += SIMT_THREADS)
+            for (int g = tid; g < kc * M / 4; g += NT)
                 asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(mbs + 16u * g),
                              "l"(__cvta_generic_to_global(m.memb + (size_t)k0 * M + 4 * g))
                              : "memory");
             asm volatile("cp.async.commit_group;" ::: "memory");
             asm volatile("cp.async.wait_group 0;" ::: "memory");
         } else {
-            for (int t = tid; t < nq * kc; t += SIMT_THREADS) {
+            for (int t = tid; t < nq * kc; t += NT) {
                 const int i = t / kc, k = t - i * kc, qq = q0 + i;
                 const size_t src = (size_t)(qq < q.Q ? qq : 0) * E + k0 + k;
                 if (es == 4) reinterpret_cast<float *>(er)[i * ld + k] = qq < q.Q ? ((const float *)q.emb)[src] : 0.f;
                 else reinterpret_cast<uint16_t *>(er)[i * ld + k] = qq < q.Q ? ((const uint16_t *)q.emb)[src] : 0;
             }
-            for (int t = tid; t < kc * M; t += SIMT_THREADS) mb[t] = m.memb[(size_t)k0 * M + t];
+            for (int t = tid; t < kc * M; t += NT) mb[t] = m.memb[(size_t)k0 * M + t];
         }
-        __syncthreads();
-        if (tid < nq * M) {
-            const float *b = mb + mi;
-            if (es == 4) {
-                const float *a = reinterpret_cast<const float *>(er) + qi * ld;
+        group_sync<NT>();
+#pragma unroll
+        for (int j = 0; j < CH; ++j) {
+            const int e = tid + NT * j, qi = e / M, mi = e - qi * M;
+            if (e < nq * M) {
+                const float *b = mb + mi;
+                float acc = s[j];
+                if (es == 4) {
+                    const float *a = reinterpret_cast<const float *>(er) + qi * ld;
 #pragma unroll 8
-                for (int k = 0; k < kc; ++k) s = __fmaf_rn(a[k], b[k * M], s);
-            } else {
-                const uint16_t *a = reinterpret_cast<const uint16_t *>(er) + qi * ld;
+                    for (int k = 0; k < kc; ++k) acc = __fmaf_rn(a[k], b[k * M], acc);
+                } else {
+                    const uint16_t *a = reinterpret_cast<const uint16_t *>(er) + qi * ld;
 #pragma unroll 8
-                for (int k = 0; k < kc; ++k)
-                    s = __fmaf_rn(__uint_as_float((uint32_t)a[k] << 16), b[k * M], s);
+                    for (int k = 0; k < kc; ++k)
+                        acc = __fmaf_rn(__uint_as_float((uint32_t)a[k] << 16), b[k * M], acc);
+                }
+                s[j] = acc;
             }
         }
     }
-    return tid < nq * M ? sigmoid_c(s) : 0.f;
+#pragma unroll
+    for (int j = 0; j < CH; ++j) res[j] = tid + NT * j < nq * M ? sigmoid_c(s[j]) : 0.f;
+}
+
+__device__ __forceinline__ float quality_staged(const Model &m, const Queries &q, int q0, int nq,
+                                                float *stage, int stage_floats) {
+    float r[1];
+    quality_group<SIMT_THREADS, 1>(m, q, q0, nq, stage, stage_floats, threadIdx.x, r);
+    return r[0];
 }
 
 // ---------------------------------------------------------------------------
@@ -189,6 +215,12 @@ __global__ void __launch_bounds__(SIMT_THREADS) k_snapshot(Model m) {
 // then h2 [TILE_ROWS][H2 + 1] in the same space; W3 [NH][H2] in w3s.
 
 constexpr int TILE_ROWS = 64;
+
+// Barrier of the tile's SIMT_THREADS threads only (named barrier 1), so a
+// block may run other warps beside the tile.
+__device__ __forceinline__ void tile_sync() {
+    asm volatile("bar.sync 1, %0;" ::"n"(SIMT_THREADS) : "memory");
+}
 
 __host__ __device__ constexpr int tile_width(int H2) {
     return H2 <= 32 ? 32 : H2 <= 64 ? 64 : H2 <= 128 ? 128 : 256;
@@ -240,7 +272,7 @@ __device__ void pair_mlp(const Model &m, int R, const Rows &rows, const float *u
     const bool rv = r1 < R;
     const float *pr = rv ? rows.prefix(r1) : m.W1;
     const float uq = rv ? us[rows.query(r1)] : 0.f, vq = rv ? vs[rows.query(r1)] : 0.f;
-    __syncthreads();
+    tile_sync();
     float acc[8][CPT];
 #pragma unroll
     for (int j = 0; j < CPT; ++j) {
@@ -280,7 +312,7 @@ __device__ void pair_mlp(const Model &m, int R, const Rows &rows, const float *u
         } else {
             asm volatile("cp.async.wait_group 0;" ::: "memory");
         }
-        __syncthreads();
+        tile_sync();
         if (active) {
             const float *wb = w2b + (it & 1) * SIMT_KC * W;
             for (int kk = 0; kk < kc; ++kk) {
@@ -312,7 +344,7 @@ __device__ void pair_mlp(const Model &m, int R, const Rows &rows, const float *u
                     for (int j = 0; j < CPT; ++j) acc[i][j] = __fmaf_rn(b[j], a[i], acc[i][j]);
             }
         }
-        __syncthreads();
+        tile_sync();
     }
 
     float *h2s = tile;
@@ -329,7 +361,7 @@ __device__ void pair_mlp(const Model &m, int R, const Rows &rows, const float *u
             }
         }
     }
-    __syncthreads();
+    tile_sync();
     for (int e = tid; e < m.NH * R; e += SIMT_THREADS) {
         const int r = e / m.NH, o = e - r * m.NH;
         const float *w3 = w3s + (size_t)o * H2;
@@ -337,7 +369,7 @@ __device__ void pair_mlp(const Model &m, int R, const Rows &rows, const float *u
         for (int n = 0; n < H2; ++n) z = __fmaf_rn(w3[n], h2s[r * ld + n], z);
         sp[e] = softplus_c(z);
     }
-    __syncthreads();
+    tile_sync();
 }
 
 // ---------------------------------------------------------------------------
@@ -352,9 +384,11 @@ struct RouteRows {
 
 __host__ __device__ inline int route_qb(int D) { return D >= 64 ? 1 : 64 / D; }
 
+constexpr int ROUTE_QSTAGE = 4096;   // floats of the quality warp's staging space
+
 struct RouteLayout {
     int QB, R;
-    size_t us, vs, ol, qual, sp, C, U, w3, w1q, tile, total;  // float offsets
+    size_t us, vs, ol, qual, sp, C, U, w3, w1q, qstage, tile, total;  // float offsets
 };
 
 __host__ __device__ inline RouteLayout route_layout(int D, int M, int H2) {
@@ -372,14 +406,19 @@ __host__ __device__ inline RouteLayout route_layout(int D, int M, int H2) {
     L.w3 = o; o += 3 * (size_t)H2;
     L.w1q = o; o += 2 * (size_t)MAX_H;
     o = (o + 3) & ~(size_t)3;
+    L.qstage = o; o += ROUTE_QSTAGE;
     L.tile = o;
     o += tile_floats_for(H2);
     L.total = o;
     return L;
 }
 
+// K_route_simt runs the tile on warps 0-7 and the quality chains on warp 8,
+// side by side.
+constexpr int ROUTE_THREADS = SIMT_THREADS + 32;
+
 template <int CPT>
-__global__ void __launch_bounds__(SIMT_THREADS, CPT <= 4 ? 3 : 2) k_route_simt(Model m, Queries q) {
+__global__ void __launch_bounds__(ROUTE_THREADS, CPT <= 4 ? 3 : 2) k_route_simt(Model m, Queries q) {
     extern __shared__ float4 sm4[];
     float *sm = reinterpret_cast<float *>(sm4);
     const RouteLayout L = route_layout(m.D, m.M, m.H2);
@@ -389,26 +428,33 @@ __global__ void __launch_bounds__(SIMT_THREADS, CPT <= 4 ? 3 : 2) k_route_simt(M
     float *us = sm + L.us, *vs = sm + L.vs, *ol = sm + L.ol, *qual = sm + L.qual;
     float *sp = sm + L.sp, *Cs = sm + L.C, *Us = sm + L.U;
 
-    // the two query slots on two warps (their fp64 chains run side by side)
-    if (tid < QB) {
-        const int qq = q0 + tid;
-        us[tid] = qq < q.Q ? standardise(m.xform[F - 2], (double)q.in_len[qq], m.mu[F - 2], m.sd[F - 2])
-                           : 0.f;
-    } else if (tid >= 64 && tid < 64 + QB) {
-        const int qi = tid - 64, qq = q0 + qi;
-        const float o = qq < q.Q ? q.out_len[qq] : 0.f;
-        vs[qi] = qq < q.Q ? standardise(m.xform[F - 1], (double)o, m.mu[F - 1], m.sd[F - 1]) : 0.f;
-        ol[qi] = o;
+    if (warp < SIMT_THREADS / 32) {
+        // the two query slots on two warps (their fp64 chains run side by side)
+        if (tid < QB) {
+            const int qq = q0 + tid;
+            us[tid] = qq < q.Q ? standardise(m.xform[F - 2], (double)q.in_len[qq], m.mu[F - 2],
+                                             m.sd[F - 2])
+                               : 0.f;
+        } else if (tid >= 64 && tid < 64 + QB) {
+            const int qi = tid - 64, qq = q0 + qi;
+            const float o = qq < q.Q ? q.out_len[qq] : 0.f;
+            vs[qi] = qq < q.Q ? standardise(m.xform[F - 1], (double)o, m.mu[F - 1], m.sd[F - 1])
+                              : 0.f;
+            ol[qi] = o;
+        }
+        tile_sync();
+        RouteRows rows{m.A, D, m.H1};
+        pair_mlp<CPT>(m, R, rows, us, vs, sm + L.tile, sm + L.w3, sm + L.w1q, sp);
+    } else {
+        // quality (QB M <= 64 chains) on the last warp, while the tile runs
+        float qv[2];
+        quality_group<32, 2>(m, q, q0, QB, sm + L.qstage, ROUTE_QSTAGE, lane, qv);
+        if (lane < QB * M) qual[lane] = qv[0];
+        if (lane + 32 < QB * M) qual[lane + 32] = qv[1];
     }
-    // quality, staged through the (not yet used) tile space
-    const float qv = quality_staged(m, q, q0, QB, sm + L.tile, (int)tile_floats_for(m.H2));
-    if (tid < QB * M) qual[tid] = qv;
     __syncthreads();
 
-    RouteRows rows{m.A, D, m.H1};
-    pair_mlp<CPT>(m, R, rows, us, vs, sm + L.tile, sm + L.w3, sm + L.w1q, sp);
-
-    for (int r = tid; r < R; r += SIMT_THREADS) {
+    for (int r = tid; r < R; r += ROUTE_THREADS) {
         const int qi = r / D, d = r - qi * D;
         const float *h = sp + m.NH * r;   // TTFT, TPOT (, N_out)
         const float C = __fmaf_rn(m.NH == 3 ? h[2] : ol[qi], h[1], h[0]);
@@ -418,11 +464,11 @@ __global__ void __launch_bounds__(SIMT_THREADS, CPT <= 4 ? 3 : 2) k_route_simt(M
         if (q.pair_C && q0 + qi < q.Q) q.pair_C[(size_t)(q0 + qi) * D + d] = C;
     }
     if (q.qual_out)
-        for (int e = tid; e < QB * M; e += SIMT_THREADS)
+        for (int e = tid; e < QB * M; e += ROUTE_THREADS)
             if (q0 + e / M < q.Q) q.qual_out[(size_t)q0 * M + e] = qual[e];
     __syncthreads();
 
-    for (int qi = warp; qi < QB; qi += SIMT_THREADS / 32) {
+    for (int qi = warp; qi < QB; qi += ROUTE_THREADS / 32) {
         const int qq = q0 + qi;
         if (qq >= q.Q) continue;
         Cand best = no_cand();
@@ -1010,10 +1056,10 @@ cudaError_t launch_route_simt(const Model &m, const Queries &q, cudaStream_t s) 
     const int blocks = (q.Q + L.QB - 1) / L.QB;
     const size_t smem = L.total * sizeof(float);
     switch (cpt_for(m.H2)) {
-        case 1: k_route_simt<1><<<blocks, SIMT_THREADS, smem, s>>>(m, q); break;
-        case 2: k_route_simt<2><<<blocks, SIMT_THREADS, smem, s>>>(m, q); break;
-        case 4: k_route_simt<4><<<blocks, SIMT_THREADS, smem, s>>>(m, q); break;
-        default: k_route_simt<8><<<blocks, SIMT_THREADS, smem, s>>>(m, q); break;
+        case 1: k_route_simt<1><<<blocks, ROUTE_THREADS, smem, s>>>(m, q); break;
+        case 2: k_route_simt<2><<<blocks, ROUTE_THREADS, smem, s>>>(m, q); break;
+        case 4: k_route_simt<4><<<blocks, ROUTE_THREADS, smem, s>>>(m, q); break;
+        default: k_route_simt<8><<<blocks, ROUTE_THREADS, smem, s>>>(m, q); break;
     }
     return cudaGetLastError();
 }

@@ -32,7 +32,7 @@ def _exact_row(got, k, want, what):
     assert np.array_equal(util, want[2].astype(np.float32), equal_nan=True), what
 
 
-# (config, Q, flags): small pair-parallel batches, the fused SIMT kernel, bf16
+# (config, Q, flags): small batches, the fused SIMT kernel, bf16
 # contexts on the SIMT kernels, and the score-convex utility
 @pytest.mark.parametrize("c,Q,flags", [
     (0, 1, 0), (0, 97, 0), (0, 256, 0), (0, 1000, 0),
@@ -132,3 +132,19 @@ def test_argument_errors():
     assert e.value.status == 7
     assert r.route_multi(LAMS[:2])[0].shape == (2, 8)     # still usable
     r.close()
+
+
+@pytest.mark.parametrize("c,Q", [(0, 97), (2, 40)])
+def test_pair_kernel_rows_equal_oracle(monkeypatch, c, Q):
+    """The pair-parallel kernel's stored scores feed the multi-lambda selection."""
+    monkeypatch.setenv("HWR_PAIRS_MAX_PAIRS", "2048")
+    p = W.make_config(c, Q=Q)
+    r = H.Router(p)
+    got = r.route_multi(LAMS)
+    C, qual = r.score()
+    r.close()
+    orc = O.Problem(p)
+    for k, lam in enumerate(LAMS):
+        _exact_row(got, k, orc.route(lam=float(lam), mode=O.F32, nthreads=8), f"cfg{c} lambda={lam}")
+    Cw, _ = orc.score_all(mode=O.F32, nthreads=8)
+    assert np.array_equal(C, Cw.astype(np.float32))
