@@ -36,13 +36,13 @@ struct AllocHook {
 // kernel; larger bf16 batches of at least tc_min_pairs pairs take the
 // tensor-core kernels; the rest the fused SIMT kernel.  pairs_max is
 // SMALL_MAX_PAIRS where the tensor-core path exists; otherwise FP32_MAX_PAIRS
-// for hidden layers wider than 64 x 64 and 0 (always the fused kernel) for
-// narrower ones.  (Device pointers, isolated calls.  bf16: the tensor path
-// costs 31-33 us at D = 32 and 38-40 us at D = 64 for 1 to 64 queries; the
-// small-batch kernel is ahead up to 256 pairs and behind from 512 on.  fp32:
-// the fused kernel costs ~21 us at H = 32 and ~33.5 us at H = 128 from 1 to
-// 512 queries; the small-batch kernel costs 22-47 us at H = 32 (never
-// ahead) and 25-39 us at H = 128 for 1-64 queries (ahead up to ~500 pairs).)
+// for hidden layers wider than 64 x 64 and SMALL_MAX_PAIRS for narrower ones.
+// (Device pointers, isolated calls.  bf16: the tensor path costs 31-33 us at
+// D = 32 and 38-40 us at D = 64 for 1 to 64 queries; the small-batch kernel
+// is ahead up to 256 pairs and behind from 512 on.  fp32: the fused kernel
+// costs ~21.5 us at H = 32 and ~33.5 us at H = 128 from 1 to 512 queries;
+// the small-batch kernel costs 20.5-21 us at H = 32 up to 256 pairs and more
+// beyond, 23.6-38 us at H = 128 for 1-64 queries: ahead up to ~500 pairs.)
 constexpr int TC_MIN_PAIRS = 257;
 constexpr int PIPE_CHUNK_MIN = 8192;   // smallest chunk of a pipelined host batch
 constexpr int SMALL_MAX_PAIRS = 256;
@@ -559,7 +559,7 @@ extern "C" hwr_status hwr_create(const hwr_deployment_table *table, const hwr_pr
         return s;
     }
     if (c->pairs_max < 0)
-        c->pairs_max = c->tc_ok ? SMALL_MAX_PAIRS : (c->H1 * c->H2 > 64 * 64 ? FP32_MAX_PAIRS : 0);
+        c->pairs_max = !c->tc_ok && c->H1 * c->H2 > 64 * 64 ? FP32_MAX_PAIRS : SMALL_MAX_PAIRS;
     *out = c;
     return HWR_OK;
 }

@@ -495,8 +495,7 @@ __global__ void __launch_bounds__(ROUTE_THREADS, CPT <= 4 ? 3 : 2) k_route_simt(
 //
 // Table layout (triangular): for c in [0, Qs), d in [0, D), i in [c, Qs):
 //   index = D * (c * Qs - c (c - 1) / 2) + d * (Qs - c) + (i - c).
-// A table block takes deployment d and the two groups c1 and Qs - 1 - c1,
-// whose row counts add up to Qs + 1.
+// A table block takes an equal run of consecutive entries.
 
 __host__ __device__ inline size_t tri_off(int D, int Qs, int c) {
     return (size_t)D * ((size_t)c * Qs - (size_t)c * (c - 1) / 2);
@@ -887,9 +886,11 @@ __global__ void __launch_bounds__(SIMT_THREADS) k_route_pairs(Model m, Queries q
         const int d = blockIdx.x - qq * D;
         float *h1 = sm, *h2 = sm + MAX_H;
         __shared__ float uv[3];
+        // the two query slots on two warps (their fp64 chains run side by side)
         if (tid == 0) {
-            const float o = q.out_len[qq];
             uv[0] = standardise(m.xform[F - 2], (double)q.in_len[qq], m.mu[F - 2], m.sd[F - 2]);
+        } else if (tid == 32) {
+            const float o = q.out_len[qq];
             uv[1] = standardise(m.xform[F - 1], (double)o, m.mu[F - 1], m.sd[F - 1]);
             uv[2] = o;
         }
