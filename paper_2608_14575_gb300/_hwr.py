@@ -231,6 +231,17 @@ class Router:
         if st != HWR_OK:
             raise HwrError(st, self.lib.hwr_last_error(None).decode())
         self.ctx = ctx
+        # snapshot staging: one persistent buffer whose six slices the
+        # prebuilt hwr_snapshot points at, so an update copies six small
+        # arrays instead of taking six pointers
+        D = self.D
+        self._snap_buf = np.empty(6 * D, np.uint32)
+        b = self._snap_buf
+        self._snap_views = (b[0:D].view(np.int32), b[D:2 * D].view(np.int32),
+                            b[2 * D:3 * D].view(np.float32), b[3 * D:4 * D].view(np.float32),
+                            b[4 * D:5 * D].view(np.float32), b[5 * D:6 * D].view(np.float32))
+        base = b.ctypes.data
+        self._snap_struct = hwr_snapshot(*[base + 4 * D * k for k in range(6)])
         self.update_snapshot(p["snap"])
 
     def _check(self, st):
@@ -238,11 +249,13 @@ class Router:
             raise HwrError(st, self.lib.hwr_last_error(self.ctx).decode())
 
     def update_snapshot(self, snap: dict):
-        arrs = [_c(snap["running"], np.int32), _c(snap["waiting"], np.int32),
-                _c(snap["kv"], np.float32), _c(snap["gpu_util"], np.float32),
-                _c(snap["ttft"], np.float32), _c(snap["tpot"], np.float32)]
-        s = hwr_snapshot(*[a.ctypes.data for a in arrs])
-        self._check(self.lib.hwr_update_snapshot(self.ctx, ct.byref(s)))
+        v = self._snap_views
+        for k, name in enumerate(("running", "waiting", "kv", "gpu_util", "ttft", "tpot")):
+            a = np.asarray(snap[name])
+            if a.shape != (self.D,):
+                raise ValueError(f"snapshot {name}: shape {a.shape}, want ({self.D},)")
+            v[k][...] = a
+        self._check(self.lib.hwr_update_snapshot(self.ctx, ct.byref(self._snap_struct)))
 
     def get_snapshot(self) -> np.ndarray:
         out = np.empty(self.D, np.int32)
@@ -257,15 +270,15 @@ class Router:
         ol = _c(p["out_len"] if out_len is None else out_len, np.float32)
         em = _c(p["emb"] if emb is None else emb, self.wdt)
         Q = il.size
-        chosen = np.empty(Q, np.int32)
-        lat = np.empty(Q, np.float32)
-        util = np.empty(Q, np.float32)
+        # the three outputs as views of one allocation (one pointer to take)
+        out = np.empty(3 * Q, np.uint32)
+        o = out.ctypes.data
         self._check(self.lib.hwr_route_batch(
             self.ctx, Q, il.ctypes.data, ol.ctypes.data, em.ctypes.data,
             float(p["slo"] if slo is None else slo),
             float(p["lam"] if lam is None else lam), int(flags) & ~HWR_DEVICE_PTRS,
-            chosen.ctypes.data, lat.ctypes.data, util.ctypes.data))
-        return chosen, lat, util
+            o, o + 4 * Q, o + 8 * Q))
+        return out[:Q].view(np.int32), out[Q:2 * Q].view(np.float32), out[2 * Q:].view(np.float32)
 
     def score(self, in_len=None, out_len=None, emb=None, *, flags=0, quality=True):
         """Cost [Q][D] and quality [Q][M] (None unless `quality`) of a host batch."""
@@ -327,14 +340,13 @@ class Router:
         em = _c(p["emb"] if emb is None else emb, self.wdt)
         Q = il.size
         spec, keep = self._spec(budgets, model, Q)
-        chosen = np.empty(Q, np.int32)
-        lat = np.empty(Q, np.float32)
-        util = np.empty(Q, np.float32)
+        out = np.empty(3 * Q, np.uint32)
+        o = out.ctypes.data
         self._check(self.lib.hwr_route_batch_slo(
             self.ctx, Q, il.ctypes.data, ol.ctypes.data, em.ctypes.data, ct.byref(spec),
             float(p["lam"] if lam is None else lam), int(flags) & ~HWR_DEVICE_PTRS,
-            chosen.ctypes.data, lat.ctypes.data, util.ctypes.data))
-        return chosen, lat, util
+            o, o + 4 * Q, o + 8 * Q))
+        return out[:Q].view(np.int32), out[Q:2 * Q].view(np.float32), out[2 * Q:].view(np.float32)
 
     def route_device_slo(self, in_len, out_len, emb, chosen, lat, util, *, budgets=None,
                          model=None, lam, flags=0):
