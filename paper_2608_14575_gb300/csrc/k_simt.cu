@@ -24,6 +24,7 @@
 
 #include "hwr_internal.cuh"
 #include "select.cuh"
+#include "umma.cuh"
 
 namespace hwr {
 
@@ -534,6 +535,7 @@ size_t seq_aux_floats(int D, int M, int H1, int Qs) {
 constexpr int PREP_THREADS = 128;
 
 __global__ void __launch_bounds__(PREP_THREADS) k_seq_prep(Model m, Queries q, int Qs, float *aux) {
+    umma::grid_launch_dependents();
     const SeqAux a = seq_aux(aux, m.D, m.M, Qs);
     const int tid = threadIdx.x, F = m.F, P = m.P, H1 = m.H1;
     const int nuv = (2 * Qs + PREP_THREADS - 1) / PREP_THREADS;
@@ -615,6 +617,10 @@ k_seq_table(Model m, Queries q, int Qs, int nb_qual, int rows_per_block, float *
     const int D = m.D, M = m.M;
     const SeqLayout L = seq_layout(m.H2);
     const SeqAux A = seq_aux(aux, D, M, Qs);
+    // launched as a programmatic dependent of the preparation kernel: the
+    // chain may be scheduled now; the quality blocks need nothing from the
+    // preparation kernel, the table blocks wait for it below
+    umma::grid_launch_dependents();
     if ((int)blockIdx.x < nb_qual) {
         // quality of the chunk's queries [q0, q0 + nq), staged through the whole
         // shared space
@@ -628,10 +634,6 @@ k_seq_table(Model m, Queries q, int Qs, int nb_qual, int rows_per_block, float *
     const int R = min(rows_per_block, T - t0);
     float *us = sm + L.us, *vs = sm + L.vs, *sp = sm + L.sp;
     int *gi = reinterpret_cast<int *>(sm + L.gi), *qi = reinterpret_cast<int *>(sm + L.qi);
-    for (int i = tid; i < Qs; i += SIMT_THREADS) {
-        us[i] = A.us[i];
-        vs[i] = A.vs[i];
-    }
     for (int r = tid; r < R; r += SIMT_THREADS) {
         // entry t: the count c with tri_off(c) <= t < tri_off(c + 1), then d and i
         const int t = t0 + r;
@@ -644,6 +646,11 @@ k_seq_table(Model m, Queries q, int Qs, int nb_qual, int rows_per_block, float *
         const int off = t - (int)tri_off(D, Qs, lo), len = Qs - lo, d = off / len;
         gi[r] = d * (Qs + 1) + lo;
         qi[r] = lo + off - d * len;
+    }
+    umma::grid_dependency_wait();    // the preparation kernel's features and prefixes
+    for (int i = tid; i < Qs; i += SIMT_THREADS) {
+        us[i] = A.us[i];
+        vs[i] = A.vs[i];
     }
     __syncthreads();
 
@@ -705,6 +712,12 @@ k_seq_chain(Model m, Queries q, int Qs, const float *ctab, float *aux) {
     float *o_lat = slo + Qs, *o_util = o_lat + Qs;
     int *o_ch = reinterpret_cast<int *>(o_util + Qs);
 
+    // launched as a programmatic dependent of the table kernel: budgets and
+    // the model map first, then wait for the table (and, through it, for the
+    // preparation kernel)
+    for (int i = tid; i < Qs; i += CHAIN_THREADS) slo[i] = query_budget(q, i);
+    for (int e = tid; e < D; e += CHAIN_THREADS) dm[e] = m.dep_model[e];
+    umma::grid_dependency_wait();
     // the table, by 16-byte asynchronous copies (both sides 16-byte aligned)
     const uint32_t tab_s = (uint32_t)__cvta_generic_to_shared(tab);
     for (size_t e = tid; e < T / 4; e += CHAIN_THREADS)
@@ -714,8 +727,6 @@ k_seq_chain(Model m, Queries q, int Qs, const float *ctab, float *aux) {
     asm volatile("cp.async.commit_group;" ::: "memory");
     for (size_t e = T / 4 * 4 + tid; e < T; e += CHAIN_THREADS) tab[e] = __ldcg(ctab + e);
     for (int e = tid; e < Qs * M; e += CHAIN_THREADS) qs[e] = __ldcg(A.qual + e);
-    for (int i = tid; i < Qs; i += CHAIN_THREADS) slo[i] = query_budget(q, i);
-    for (int e = tid; e < D; e += CHAIN_THREADS) dm[e] = m.dep_model[e];
     asm volatile("cp.async.wait_all;" ::: "memory");
     __syncthreads();
 
@@ -1025,6 +1036,27 @@ int seq_chunk(const Model &m) {
     return Qs;
 }
 
+// Launch configuration of a programmatic dependent launch: the grid may be
+// scheduled before the previous kernel in the stream has finished; it calls
+// griddepcontrol.wait before it reads that kernel's results.
+static cudaLaunchAttribute g_pdl_attr = [] {
+    cudaLaunchAttribute a = {};
+    a.id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    a.val.programmaticStreamSerializationAllowed = 1;
+    return a;
+}();
+
+static cudaLaunchConfig_t dependent_launch(int grid, int block, size_t smem, cudaStream_t s) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)grid);
+    cfg.blockDim = dim3((unsigned)block);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cfg.attrs = &g_pdl_attr;
+    cfg.numAttrs = 1;
+    return cfg;
+}
+
 template <class K>
 static cudaError_t opt_in(K kernel, int bytes) {
     return cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
@@ -1106,14 +1138,13 @@ cudaError_t launch_seq_table(const Model &m, const Queries &q, int Qs, int slots
     int rpb = ((T + want - 1) / want + 7) / 8 * 8;
     rpb = rpb < 8 ? 8 : (rpb > TILE_ROWS ? TILE_ROWS : rpb);
     const int blocks = nb_qual + (T + rpb - 1) / rpb;
-    const size_t smem = seq_layout(m.H2).total * sizeof(float);
+    cudaLaunchConfig_t cfg = dependent_launch(blocks, SIMT_THREADS, seq_layout(m.H2).total * sizeof(float), s);
     switch (cpt_for(m.H2)) {
-        case 1: k_seq_table<1><<<blocks, SIMT_THREADS, smem, s>>>(m, q, Qs, nb_qual, rpb, ctab, aux); break;
-        case 2: k_seq_table<2><<<blocks, SIMT_THREADS, smem, s>>>(m, q, Qs, nb_qual, rpb, ctab, aux); break;
-        case 4: k_seq_table<4><<<blocks, SIMT_THREADS, smem, s>>>(m, q, Qs, nb_qual, rpb, ctab, aux); break;
-        default: k_seq_table<8><<<blocks, SIMT_THREADS, smem, s>>>(m, q, Qs, nb_qual, rpb, ctab, aux); break;
+        case 1: return cudaLaunchKernelEx(&cfg, k_seq_table<1>, m, q, Qs, nb_qual, rpb, ctab, aux);
+        case 2: return cudaLaunchKernelEx(&cfg, k_seq_table<2>, m, q, Qs, nb_qual, rpb, ctab, aux);
+        case 4: return cudaLaunchKernelEx(&cfg, k_seq_table<4>, m, q, Qs, nb_qual, rpb, ctab, aux);
+        default: return cudaLaunchKernelEx(&cfg, k_seq_table<8>, m, q, Qs, nb_qual, rpb, ctab, aux);
     }
-    return cudaGetLastError();
 }
 
 int seq_table_slots(const Model &m) {
@@ -1135,8 +1166,8 @@ int seq_table_slots(const Model &m) {
 
 cudaError_t launch_seq_chain(const Model &m, const Queries &q, int Qs, const float *ctab,
                              float *aux, cudaStream_t s) {
-    k_seq_chain<<<1, CHAIN_THREADS, chain_smem(m.D, m.M, Qs), s>>>(m, q, Qs, ctab, aux);
-    return cudaGetLastError();
+    cudaLaunchConfig_t cfg = dependent_launch(1, CHAIN_THREADS, chain_smem(m.D, m.M, Qs), s);
+    return cudaLaunchKernelEx(&cfg, k_seq_chain, m, q, Qs, ctab, aux);
 }
 
 }  // namespace hwr
