@@ -316,6 +316,7 @@ __device__ void pair_mlp(const Model &m, int R, const Rows &rows, const float *u
         tile_sync();
         if (active) {
             const float *wb = w2b + (it & 1) * SIMT_KC * W;
+#pragma unroll 4
             for (int kk = 0; kk < kc; ++kk) {
                 const float4 a0 = *reinterpret_cast<const float4 *>(h1T + kk * TILE_ROWS + 8 * warp);
                 const float4 a1 =
