@@ -108,7 +108,8 @@ struct hwr_ctx {
     // I/O staging for host pointers: device [emb | in | out] and [chosen | lat | util]
     char *io_d = nullptr;    size_t io_cap = 0;
     char *out_d = nullptr;   size_t out_cap = 0;
-    char *pin_h = nullptr;   size_t pin_cap = 0;       // pinned host staging
+    char *pin_h = nullptr;   size_t pin_cap = 0;       // pinned, mapped host staging
+    char *pin_d = nullptr;                            // its device address
     cudaEvent_t pin_ev = nullptr;
     // large host-pointer batches: chunked copies on a second stream overlap
     // the kernels of the previous chunk
@@ -209,10 +210,13 @@ static hwr_status pin_grow(hwr_ctx *c, size_t bytes) {
     }
     size_t want = bytes + bytes / 4 + 4096;
     if (hook_fires(c)) return fail(c, HWR_ERR_OOM, "allocation %ld failed (test hook)", c->hook.count);
-    cudaError_t e = cudaHostAlloc((void **)&c->pin_h, want, cudaHostAllocDefault);
+    cudaError_t e = cudaHostAlloc((void **)&c->pin_h, want, cudaHostAllocMapped);
+    if (e == cudaSuccess) e = cudaHostGetDevicePointer((void **)&c->pin_d, c->pin_h, 0);
     if (e != cudaSuccess) {
         cudaGetLastError();
+        if (c->pin_h) cudaFreeHost(c->pin_h);
         c->pin_h = nullptr;
+        c->pin_d = nullptr;
         return fail(c, HWR_ERR_OOM, "cudaHostAlloc(%zu): %s", want, cudaGetErrorString(e));
     }
     c->pin_cap = want;
@@ -767,7 +771,7 @@ static hwr_status route_impl(hwr_ctx *c, int32_t Q, const float *in_len, const f
         TRY(grow(c, &c->io_d, &c->io_cap, in_total));
         TRY(grow(c, &c->out_d, &c->out_cap, out_total));
         if (packed) {
-            TRY(pin_grow(c, in_total > out_total ? in_total : out_total));
+            TRY(pin_grow(c, align_up(in_total, 256) + out_total));
             CK(c, cudaEventSynchronize(c->pin_ev), "wait for staging");
             memcpy(c->pin_h, q_emb, emb_b);
             memcpy(c->pin_h + off_in, in_len, len_b);
@@ -789,9 +793,12 @@ static hwr_status route_impl(hwr_ctx *c, int32_t Q, const float *in_len, const f
         if (budgets) q.slo_q = (const float *)(c->io_d + off_slo);
         q.in_len = (const float *)(c->io_d + off_in);
         q.out_len = (const float *)(c->io_d + off_out);
-        q.chosen = (int32_t *)c->out_d;
-        q.lat = (float *)(c->out_d + o_lat);
-        q.util = (float *)(c->out_d + o_util);
+        // small synchronous calls: the kernels write the outputs straight into
+        // the mapped staging (plain stores), so no device-to-host copy follows
+        char *ob = packed && !so ? c->pin_d + align_up(in_total, 256) : c->out_d;
+        q.chosen = (int32_t *)ob;
+        q.lat = (float *)(ob + o_lat);
+        q.util = (float *)(ob + o_util);
     }
 
     const Model mv = model_view(c);
@@ -890,14 +897,13 @@ static hwr_status route_impl(hwr_ctx *c, int32_t Q, const float *in_len, const f
                                   c->stream), "copy quality");
     } else if (!dev) {
         if (packed) {
-            CK(c, cudaMemcpyAsync(c->pin_h, c->out_d, out_total, cudaMemcpyDeviceToHost, c->stream),
-               "copy outputs");
+            const char *ob = c->pin_h + align_up(in_total, 256);
             CK(c, cudaEventRecord(c->pin_ev, c->stream), "record");
             CK(c, cudaStreamSynchronize(c->stream), "synchronize");
             synced = true;
-            memcpy(chosen, c->pin_h, outs_b);
-            memcpy(pred_latency, c->pin_h + o_lat, outs_b);
-            memcpy(utility, c->pin_h + o_util, outs_b);
+            memcpy(chosen, ob, outs_b);
+            memcpy(pred_latency, ob + o_lat, outs_b);
+            memcpy(utility, ob + o_util, outs_b);
         } else {
             CK(c, cudaMemcpyAsync(chosen, c->out_d, outs_b, cudaMemcpyDeviceToHost, c->stream),
                "copy chosen");
