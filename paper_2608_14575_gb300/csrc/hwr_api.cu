@@ -90,6 +90,7 @@ struct hwr_ctx {
 
     // snapshot staging (pinned) and its copy-done event
     void *snap_h = nullptr;
+    const uint32_t *snap_hd = nullptr;   // device address of the mapped snap_h
     void *snap_d = nullptr;
     cudaEvent_t snap_ev = nullptr;
 
@@ -496,7 +497,8 @@ static hwr_status build_ctx(hwr_ctx *c, const hwr_deployment_table *t, const hwr
 
     // snapshot staging: 6 arrays of D 4-byte values
     if (hook_fires(c)) return fail(c, HWR_ERR_OOM, "allocation %ld failed (test hook)", c->hook.count);
-    CK(c, cudaHostAlloc(&c->snap_h, 6 * (size_t)D * 4, cudaHostAllocDefault), "alloc snapshot staging");
+    CK(c, cudaHostAlloc(&c->snap_h, 6 * (size_t)D * 4, cudaHostAllocMapped), "alloc snapshot staging");
+    CK(c, cudaHostGetDevicePointer((void **)&c->snap_hd, c->snap_h, 0), "map snapshot staging");
     CK(c, cudaEventCreateWithFlags(&c->snap_ev, cudaEventDisableTiming), "create event");
     CK(c, cudaEventCreateWithFlags(&c->pin_ev, cudaEventDisableTiming), "create event");
     CK(c, cudaStreamCreateWithFlags(&c->copy_stream, cudaStreamNonBlocking), "create copy stream");
@@ -592,12 +594,12 @@ extern "C" hwr_status hwr_update_snapshot(hwr_ctx *c, const hwr_snapshot *s) {
     memcpy(h + 3 * n, s->gpu_util, n);
     memcpy(h + 4 * n, s->ttft_avg, n);
     memcpy(h + 5 * n, s->tpot_avg, n);
-    // one copy straight into the six device arrays (snap_d holds them back to back)
-    CK(c, cudaMemcpyAsync(c->snap_d, h, 6 * n, cudaMemcpyHostToDevice, c->stream), "copy snapshot");
-    CK(c, cudaEventRecord(c->snap_ev, c->stream), "record");
+    // the snapshot kernel reads the staging (mapped) into the six device arrays
+    // itself: no separate copy; the staging is free again once it has run
     LaunchScope ls(c, HWR_K_SNAPSHOT, false);
-    CK(c, launch_snapshot(model_view(c), c->stream), "snapshot kernel");
+    CK(c, launch_snapshot(model_view(c), c->snap_hd, c->stream), "snapshot kernel");
     ls.done();
+    CK(c, cudaEventRecord(c->snap_ev, c->stream), "record");
     c->have_snapshot = true;
     return HWR_OK;
 }

@@ -85,7 +85,11 @@ __device__ __forceinline__ float query_budget(const Queries &q, int row) {
 #endif
 
 // ---- SIMT kernels (k_simt.cu) -------------------------------------------
-cudaError_t launch_snapshot(const Model &m, cudaStream_t s);
+// The snapshot signals are read from `stage` ([6][D] 4-byte values in host
+// memory mapped into the device's address space, in the order running,
+// waiting, kv, gpu_util, ttft, tpot) into the six device arrays, which m.running
+// starts (they are contiguous, in that order).
+cudaError_t launch_snapshot(const Model &m, const uint32_t *stage, cudaStream_t s);
 // Fused gather -> MLP -> mask -> argmax for a batch.
 cudaError_t launch_route_simt(const Model &m, const Queries &q, cudaStream_t s);
 // Small-batch (latency) variant: one block per (query, deployment) pair plus

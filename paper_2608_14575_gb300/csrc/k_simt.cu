@@ -177,9 +177,15 @@ __device__ __forceinline__ float quality_staged(const Model &m, const Queries &q
 // K_snap: standardised deployment features and the deployment prefix of
 // layer 1 (the part of W1 x + b1 that does not depend on the query).
 
-__global__ void __launch_bounds__(SIMT_THREADS) k_snapshot(Model m) {
+__global__ void __launch_bounds__(SIMT_THREADS) k_snapshot(Model m, const uint32_t *stage) {
     extern __shared__ float xs[];
     const int d = blockIdx.x;
+    // this deployment's six signals, from the host's staging ([6][D], mapped)
+    // into the context's device arrays (running, waiting, kv, gpu_util, ttft, tpot)
+    if (threadIdx.x < 6)
+        reinterpret_cast<uint32_t *>(m.running)[(size_t)threadIdx.x * m.D + d] =
+            stage[(size_t)threadIdx.x * m.D + d];
+    __syncthreads();
     for (int k = threadIdx.x; k < m.F - 2; k += blockDim.x) {
         float x = standardise(m.xform[k], deployment_raw(m, d, k, m.running[d]),
                               m.mu[k], m.sd[k]);
@@ -1079,8 +1085,8 @@ cudaError_t simt_prepare() {
     return e;
 }
 
-cudaError_t launch_snapshot(const Model &m, cudaStream_t s) {
-    k_snapshot<<<m.D, SIMT_THREADS, (size_t)m.F * sizeof(float), s>>>(m);
+cudaError_t launch_snapshot(const Model &m, const uint32_t *stage, cudaStream_t s) {
+    k_snapshot<<<m.D, SIMT_THREADS, (size_t)m.F * sizeof(float), s>>>(m, stage);
     return cudaGetLastError();
 }
 
