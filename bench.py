@@ -40,6 +40,7 @@ wall-clock time of each micro-batch's route call through the C ABI.
 from __future__ import annotations
 
 import argparse
+import gc
 import json
 import os
 import statistics
@@ -254,6 +255,8 @@ def q1_latency(H, iters=10_000):
     ut = torch.empty(1, dtype=torch.float32).pin_memory()
     es = em.element_size() * p["E"]
     times = []
+    gc.collect()
+    gc.disable()      # a collector pause inside a timed call is not the library's
     for k in range(iters + 200):
         i = k % p["Q"]
         t = time.perf_counter()
@@ -262,6 +265,7 @@ def q1_latency(H, iters=10_000):
                           ut.data_ptr(), slo=p["slo"], lam=p["lam"])
         if k >= 200:
             times.append(time.perf_counter() - t)
+    gc.enable()
     r.close()
     a = np.array(times) * 1e6
     return {"p50": float(np.percentile(a, 50)), "p99": float(np.percentile(a, 99)),
@@ -302,6 +306,8 @@ def config_latencies(H, stream, dev, calls=300):
     p = W.make_config(2, Q=64 * 200)
     r = H.Router(p)
     n, times = 64, []
+    gc.collect()
+    gc.disable()      # a collector pause inside a timed call is not the library's
     for k in range(220):
         lo = (k % 200) * n
         t = time.perf_counter()
@@ -310,6 +316,7 @@ def config_latencies(H, stream, dev, calls=300):
                 flags=H.HWR_SEQUENTIAL)
         if k >= 20:
             times.append(time.perf_counter() - t)
+    gc.enable()
     r.close()
     a = np.array(times) * 1e6
     out["config2"] = {"workload": workload_name(p) + ", micro-batches of 64, sequential",
@@ -352,7 +359,12 @@ def online_report(args):
                     out = r.route(snap, lo, hi)
                     times.append(time.perf_counter() - t)
                     return out
-                tr = serve.run_online(p, route, r.score, static=static, **world)
+                gc.collect()
+                gc.disable()      # collector pauses are not the library's call latency
+                try:
+                    tr = serve.run_online(p, route, r.score, static=static, **world)
+                finally:
+                    gc.enable()
             m = MX.summarize(tr, p["dep_gpu"], p["G"], p["D"])
             us = np.array(times) * 1e6
             sizes = tr["batch_end"] - tr["batch_start"]
