@@ -202,3 +202,28 @@ def test_repeated_routes_and_scores_are_bitwise_identical():
         for a, b in zip(R, R0):
             assert np.array_equal(a, b, equal_nan=True)
     r.close()
+
+
+def test_tensor_route_after_sequential_sees_the_increments():
+    """A sequential call raises the running counts and refreshes the layer-1
+    prefix, fp32 and bf16; a tensor-core batch route afterwards must score
+    against the raised counts (and a new snapshot must undo them)."""
+    p = W.make_config(1, Q=600)                    # bf16, D = 12
+    r = H.Router(p)
+    seq_q = 64
+    got_seq = r.route(p["in_len"][:seq_q], p["out_len"][:seq_q], p["emb"][:seq_q],
+                      flags=H.HWR_SEQUENTIAL)
+    orc = O.Problem(p)
+    want = orc.route(p["in_len"][:seq_q], p["out_len"][:seq_q], p["emb"][:seq_q],
+                     mode=O.F32, sequential=True, nthreads=8)
+    assert np.array_equal(got_seq[0], want[0])
+    raised = r.get_snapshot()
+    assert np.array_equal(raised, want[3]) and not np.array_equal(raised, p["snap"]["running"])
+    after = r.route(flags=H.HWR_PATH_TENSOR)
+    snap = dict(p["snap"])
+    snap["running"] = raised
+    check_against_oracle(dict(p, snap=snap), after)
+    # a fresh snapshot restores the original counts for the tensor path too
+    r.update_snapshot(p["snap"])
+    check_against_oracle(p, r.route(flags=H.HWR_PATH_TENSOR))
+    r.close()
