@@ -173,10 +173,15 @@ hwr_status hwr_get_snapshot(hwr_ctx *ctx, int32_t *running_out);
  * host arrays must then stay valid until hwr_synchronize().
  * HWR_SEQUENTIAL: queries are routed in index order and each decision
  * increments its deployment's running count before the next query is scored;
- * the increments persist in the context until the next update_snapshot.
+ * the increments persist in the context until the next update_snapshot.  By
+ * default the scores follow the canonical fp32 order (SIMT kernels, also in
+ * bf16 contexts); with HWR_PATH_TENSOR as well (bf16 contexts) the score
+ * table is computed on the tensor cores (bf16 operands, fp32 accumulation:
+ * the tensor path's tolerance, and a near tie may then be decided the other
+ * way, which changes the later counts).
  * Routing before the first hwr_update_snapshot is rejected (INVALID_ARG).
- * Errors: INVALID_ARG, UNSUPPORTED (e.g. HWR_PATH_TENSOR on an fp32 context,
- * or together with HWR_SEQUENTIAL), STATE, OOM, CUDA, TIMEOUT.
+ * Errors: INVALID_ARG, UNSUPPORTED (e.g. HWR_PATH_TENSOR on an fp32 context),
+ * STATE, OOM, CUDA, TIMEOUT.
  */
 hwr_status hwr_route_batch(hwr_ctx *ctx, int32_t Q, const float *in_len,
                            const float *out_len, const void *q_emb, float slo,

@@ -104,6 +104,11 @@ struct hwr_ctx {
     float *ctab = nullptr;   size_t ctab_cap = 0;
     float *qseq = nullptr;   size_t qseq_cap = 0;
     int seq_qs = 0;
+    // sequential mode with the table on the tensor cores: costs [Qs][D (Qs+1)],
+    // bf16 prefixes [D (Qs+1)][H1], model of each (deployment, count) group
+    float *ptab = nullptr;   size_t ptab_cap = 0;
+    uint16_t *prebf = nullptr; size_t prebf_cap = 0;
+    int32_t *dmv = nullptr;  size_t dmv_cap = 0;
     int seq_slots = 0;       // sequential-table blocks resident at once
 
     // I/O staging for host pointers: device [emb | in | out] and [chosen | lat | util]
@@ -622,7 +627,17 @@ static hwr_status run_kernels(hwr_ctx *c, const Queries &q, uint32_t flags, bool
     const Model m = model_view(c);
     if (flags & HWR_SEQUENTIAL) {
         const int Qs = c->seq_qs;
-        TRY(grow(c, &c->ctab, &c->ctab_cap, seq_table_floats(c->D, Qs)));
+        // HWR_PATH_TENSOR: the table on the tensor cores (bf16 contexts)
+        const bool tcs = (flags & HWR_PATH_TENSOR) && c->tc_ok;
+        if (tcs) {
+            const size_t Dv = (size_t)c->D * (Qs + 1);
+            TRY(grow(c, &c->ptab, &c->ptab_cap, (size_t)Qs * Dv));
+            TRY(grow(c, &c->prebf, &c->prebf_cap, Dv * c->H1));
+            TRY(grow(c, &c->dmv, &c->dmv_cap, Dv));
+            TRY(grow(c, &c->qual, &c->qual_cap, (size_t)Qs * c->Mpad));
+        } else {
+            TRY(grow(c, &c->ctab, &c->ctab_cap, seq_table_floats(c->D, Qs)));
+        }
         TRY(grow(c, &c->qseq, &c->qseq_cap, seq_aux_floats(c->D, c->M, c->H1, Qs)));
         const size_t es = c->dtype == HWR_BF16 ? 2 : 4;
         for (int lo = 0; lo < q.Q; lo += Qs) {
@@ -636,6 +651,38 @@ static hwr_status run_kernels(hwr_ctx *c, const Queries &q, uint32_t flags, bool
             k.lat = q.lat + lo;
             k.util = q.util + lo;
             if (q.slo_q) k.slo_q = q.slo_q + lo;
+            if (tcs) {
+                // preparation (features, prefixes, their bf16 copies), then the
+                // chunk's quality and the cost of every (query, deployment,
+                // count) on the tensor cores, then the chain.  The predictor
+                // kernel runs as a dependent of the quality kernel: only its
+                // epilogue waits, and the prefixes it reads early come from the
+                // preparation kernel, which finished before the quality kernel
+                // began.
+                const TcModel t = tc_view(c);
+                TcModel tv = t;
+                tv.D = c->D * (n + 1);
+                tv.Abf = c->prebf;
+                tv.dep_model = c->dmv;
+                Queries kt = k;
+                kt.pair_C = c->ptab;
+                kt.no_select = 1;
+                kt.slo_mode = 0;      // budgets are the chain's business
+                kt.slo_q = nullptr;
+                LaunchScope a(c, HWR_K_SEQ_TABLE, prof);
+                CK(c, launch_seq_prep_tc(m, k, n, c->qseq, c->prebf, c->dmv, c->stream),
+                   "sequential preparation");
+                CK(c, launch_qual_tc(t, k, c->qual, c->status_d, c->stream), "quality kernel");
+                CK(c, launch_mlp_tc_scores(tv, kt, c->qual, c->status_d, c->stream),
+                   "sequential table (tensor cores)");
+                a.done();
+                CK(c, launch_seq_chain_tc(m, k, n, c->ptab, c->qseq, c->qual, c->Mpad, c->stream),
+                   "sequential chain");
+                // preparation, quality and chain beside the scope's table kernel
+                c->stats.kernel_launches += 3;
+                c->stats.launches[HWR_K_SEQ_TABLE] += 3;
+                continue;
+            }
             LaunchScope a(c, HWR_K_SEQ_TABLE, prof);
             CK(c, launch_seq_table(m, k, n, c->seq_slots, c->ctab, c->qseq, c->stream),
                "sequential table");
@@ -712,9 +759,9 @@ static hwr_status route_impl(hwr_ctx *c, int32_t Q, const float *in_len, const f
     if (!c->have_snapshot)
         return fail(c, HWR_ERR_INVALID_ARG, "route before the first hwr_update_snapshot");
     const bool seq = flags & HWR_SEQUENTIAL;
-    if ((flags & HWR_PATH_TENSOR) && (seq || !c->tc_ok))
-        return fail(c, HWR_ERR_UNSUPPORTED, "tensor-core path unavailable for this %s",
-                    seq ? "sequential call" : "context (fp32 or unsupported shape)");
+    if ((flags & HWR_PATH_TENSOR) && !c->tc_ok)
+        return fail(c, HWR_ERR_UNSUPPORTED,
+                    "tensor-core path unavailable for this context (fp32 or unsupported shape)");
     const bool tensor = !seq && c->tc_ok &&
                         ((flags & HWR_PATH_TENSOR) ||
                          (!(flags & HWR_PATH_SIMT) && (long)Q * c->D >= c->tc_min_pairs &&
@@ -724,7 +771,7 @@ static hwr_status route_impl(hwr_ctx *c, int32_t Q, const float *in_len, const f
     const int K = ml ? ml->K : 1;
     if ((ml || so) && seq)
         return fail(c, HWR_ERR_UNSUPPORTED, "HWR_SEQUENTIAL with several lambdas or scoring");
-    if (dev && tensor && ((uintptr_t)q_emb & 15))
+    if (dev && (tensor || (seq && (flags & HWR_PATH_TENSOR))) && ((uintptr_t)q_emb & 15))
         return fail(c, HWR_ERR_INVALID_ARG, "device q_emb must be 16-byte aligned");
 
     Queries q;
@@ -919,7 +966,7 @@ static hwr_status route_impl(hwr_ctx *c, int32_t Q, const float *in_len, const f
     if ((flags & HWR_ASYNC) && !synced) return HWR_OK;
     if (!synced) CK(c, cudaStreamSynchronize(c->stream), "synchronize");
     CK(c, cudaGetLastError(), "kernel");
-    if (tensor) TRY(check_status_word(c));
+    if (tensor || (seq && (flags & HWR_PATH_TENSOR))) TRY(check_status_word(c));
     return HWR_OK;
 }
 

@@ -62,6 +62,9 @@ struct Queries {
     // kernel) every query's quality [Q][M] for a later multi-lambda selection
     float *pair_C = nullptr;
     float *qual_out = nullptr;
+    // when set, the tensor-core predictor kernel only stores pair_C (no
+    // decision outputs, no partial results)
+    int no_select = 0;
 };
 
 // Several values of lambda applied to one set of scores.
@@ -111,6 +114,15 @@ cudaError_t launch_seq_table(const Model &m, const Queries &q, int Qs, int slots
 cudaError_t launch_seq_chain(const Model &m, const Queries &q, int Qs,
                              const float *ctab, float *aux, cudaStream_t s);
 size_t seq_aux_floats(int D, int M, int H1, int Qs);
+// Sequential mode with the table on the tensor cores (bf16 contexts): the
+// preparation kernel alone, also writing bf16 prefixes pre_bf [D (Qs + 1)][H1]
+// and the model of each (deployment, count) group dmv [D (Qs + 1)]; the chain
+// over a table of costs ptab [Qs][D (Qs + 1)] (query i, group d (Qs + 1) + c)
+// with quality rows qual [Qs][qstride].
+cudaError_t launch_seq_prep_tc(const Model &m, const Queries &q, int Qs, float *aux,
+                               uint16_t *pre_bf, int32_t *dmv, cudaStream_t s);
+cudaError_t launch_seq_chain_tc(const Model &m, const Queries &q, int Qs, const float *ptab,
+                                float *aux, const float *qual, int qstride, cudaStream_t s);
 int seq_table_slots(const Model &m);
 // Decision maker for K lambdas from stored scores: C [Q][D], quality
 // qual[q * qstride + model]; outputs [K][ostride] starting at query 0.
@@ -156,6 +168,10 @@ cudaError_t launch_mlp_tc(const TcModel &m, const Queries &q, const float *qual,
                           int nsplit, void *part, int32_t *count, int32_t *status,
                           cudaStream_t s);
 cudaError_t tc_prepare();
+// Costs of every (query, deployment) pair of at most 128 queries into
+// q.pair_C [Q][m.D] (q.no_select set), the deployments spread over the SMs.
+cudaError_t launch_mlp_tc_scores(const TcModel &m, const Queries &q, const float *qual,
+                                 int32_t *status, cudaStream_t s);
 size_t tc_head_consts_bytes();
 void tc_fill_head_consts(void *dst, const float *b2, const float *W3, const float *b3, int H2,
                          int NH);

@@ -541,7 +541,8 @@ size_t seq_aux_floats(int D, int M, int H1, int Qs) {
 // one block per (d, c).
 constexpr int PREP_THREADS = 128;
 
-__global__ void __launch_bounds__(PREP_THREADS) k_seq_prep(Model m, Queries q, int Qs, float *aux) {
+__global__ void __launch_bounds__(PREP_THREADS)
+k_seq_prep(Model m, Queries q, int Qs, float *aux, uint16_t *pre_bf, int32_t *dmv) {
     umma::grid_launch_dependents();
     const SeqAux a = seq_aux(aux, m.D, m.M, Qs);
     const int tid = threadIdx.x, F = m.F, P = m.P, H1 = m.H1;
@@ -561,6 +562,7 @@ __global__ void __launch_bounds__(PREP_THREADS) k_seq_prep(Model m, Queries q, i
     if (tid == 0) {
         xr = standardise(m.xform[P + 1], (double)(m.running[d] + c), m.mu[P + 1], m.sd[P + 1]);
         a.xr[g] = xr;
+        if (dmv) dmv[g] = m.dep_model[d];
     }
     __syncthreads();
     // continue the chain from slot P + 1 (running) with the deployment's other features
@@ -571,6 +573,7 @@ __global__ void __launch_bounds__(PREP_THREADS) k_seq_prep(Model m, Queries q, i
         acc = __fmaf_rn(m.W1T[(size_t)(P + 1) * H1 + j], xr, acc);
         for (int k = P + 2; k < F - 2; ++k) acc = __fmaf_rn(m.W1T[(size_t)k * H1 + j], x[k], acc);
         a.pre[(size_t)g * H1 + j] = acc;
+        if (pre_bf) pre_bf[(size_t)g * H1 + j] = __bfloat16_as_ushort(__float2bfloat16_rn(acc));
     }
 }
 
@@ -706,7 +709,8 @@ __device__ __forceinline__ uint64_t cand_key(float C, float U, int d, float slo)
 }
 
 __global__ void __launch_bounds__(CHAIN_THREADS)
-k_seq_chain(Model m, Queries q, int Qs, const float *ctab, float *aux) {
+k_seq_chain(Model m, Queries q, int Qs, const float *ctab, int Dv, float *aux, const float *qsrc,
+            int qstride) {
     extern __shared__ float4 sm4[];
     float *sm = reinterpret_cast<float *>(sm4);
     const int tid = threadIdx.x, lane = tid & 31;
@@ -725,15 +729,33 @@ k_seq_chain(Model m, Queries q, int Qs, const float *ctab, float *aux) {
     for (int i = tid; i < Qs; i += CHAIN_THREADS) slo[i] = query_budget(q, i);
     for (int e = tid; e < D; e += CHAIN_THREADS) dm[e] = m.dep_model[e];
     umma::grid_dependency_wait();
-    // the table, by 16-byte asynchronous copies (both sides 16-byte aligned)
     const uint32_t tab_s = (uint32_t)__cvta_generic_to_shared(tab);
-    for (size_t e = tid; e < T / 4; e += CHAIN_THREADS)
-        asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(tab_s + (uint32_t)(16 * e)),
-                     "l"(__cvta_generic_to_global(ctab + 4 * e))
-                     : "memory");
+    if (Dv == 0) {
+        // the triangular table, by 16-byte asynchronous copies (both sides
+        // 16-byte aligned)
+        for (size_t e = tid; e < T / 4; e += CHAIN_THREADS)
+            asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(tab_s + (uint32_t)(16 * e)),
+                         "l"(__cvta_generic_to_global(ctab + 4 * e))
+                         : "memory");
+        for (size_t e = T / 4 * 4 + tid; e < T; e += CHAIN_THREADS) tab[e] = __ldcg(ctab + e);
+    } else {
+        // costs per (query i, virtual deployment d (Qs + 1) + c) [Qs][Dv]:
+        // gather the entries with c <= i into the triangular layout, one
+        // (c, d) group per warp at a time
+        for (int g = tid >> 5; g < D * Qs; g += CHAIN_THREADS / 32) {
+            const int c = g / D, d = g - c * D, row = tab_row(D, Qs, c, d);
+            for (int i = c + lane; i < Qs; i += 32)
+                asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(
+                                 tab_s + 4u * (uint32_t)(row + i)),
+                             "l"(__cvta_generic_to_global(ctab + (size_t)i * Dv + d * (Qs + 1) + c))
+                             : "memory");
+        }
+    }
     asm volatile("cp.async.commit_group;" ::: "memory");
-    for (size_t e = T / 4 * 4 + tid; e < T; e += CHAIN_THREADS) tab[e] = __ldcg(ctab + e);
-    for (int e = tid; e < Qs * M; e += CHAIN_THREADS) qs[e] = __ldcg(A.qual + e);
+    for (int e = tid; e < Qs * M; e += CHAIN_THREADS) {
+        const int i = e / M;
+        qs[e] = __ldcg(qsrc + (size_t)i * qstride + e - i * M);
+    }
     asm volatile("cp.async.wait_all;" ::: "memory");
     __syncthreads();
 
@@ -1136,7 +1158,7 @@ cudaError_t launch_select_multi(const Model &m, const Queries &q, const float *C
 cudaError_t launch_seq_table(const Model &m, const Queries &q, int Qs, int slots, float *ctab,
                              float *aux, cudaStream_t s) {
     const int nuv = (2 * Qs + PREP_THREADS - 1) / PREP_THREADS;
-    k_seq_prep<<<nuv + m.D * (Qs + 1), PREP_THREADS, 0, s>>>(m, q, Qs, aux);
+    k_seq_prep<<<nuv + m.D * (Qs + 1), PREP_THREADS, 0, s>>>(m, q, Qs, aux, nullptr, nullptr);
     // rows per table block: a multiple of 8 (whole warps of the tile) that
     // spreads the table evenly over the blocks resident at once
     const int T = (int)tri_off(m.D, Qs, Qs);
@@ -1174,7 +1196,22 @@ int seq_table_slots(const Model &m) {
 cudaError_t launch_seq_chain(const Model &m, const Queries &q, int Qs, const float *ctab,
                              float *aux, cudaStream_t s) {
     cudaLaunchConfig_t cfg = dependent_launch(1, CHAIN_THREADS, chain_smem(m.D, m.M, Qs), s);
-    return cudaLaunchKernelEx(&cfg, k_seq_chain, m, q, Qs, ctab, aux);
+    const SeqAux A = seq_aux(aux, m.D, m.M, Qs);
+    return cudaLaunchKernelEx(&cfg, k_seq_chain, m, q, Qs, ctab, 0, aux, (const float *)A.qual, m.M);
+}
+
+cudaError_t launch_seq_prep_tc(const Model &m, const Queries &q, int Qs, float *aux,
+                               uint16_t *pre_bf, int32_t *dmv, cudaStream_t s) {
+    const int nuv = (2 * Qs + PREP_THREADS - 1) / PREP_THREADS;
+    k_seq_prep<<<nuv + m.D * (Qs + 1), PREP_THREADS, 0, s>>>(m, q, Qs, aux, pre_bf, dmv);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_seq_chain_tc(const Model &m, const Queries &q, int Qs, const float *ptab,
+                                float *aux, const float *qual, int qstride, cudaStream_t s) {
+    cudaLaunchConfig_t cfg = dependent_launch(1, CHAIN_THREADS, chain_smem(m.D, m.M, Qs), s);
+    return cudaLaunchKernelEx(&cfg, k_seq_chain, m, q, Qs, ptab, m.D * (Qs + 1), aux, qual,
+                              qstride);
 }
 
 }  // namespace hwr

@@ -556,7 +556,7 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
                 const Cand cd = make_cand(C, U, d, slo_r);
                 if (better(cd, best)) best = cd;
             }
-            if (!ok || !valid) continue;
+            if (!ok || !valid || q.no_select) continue;
             if (nsplit == 1) {
                 const bool sel = best.cls > 0;
                 q.chosen[row] = sel ? best.d : -1;
@@ -786,6 +786,16 @@ cudaError_t launch_qual_tc(const TcModel &m, const Queries &q, float *qual, int3
     const QualLayout L = qual_layout(m.Mpad, m.Epad);
     k_qual_tc<<<grid, QUAL_THREADS, L.total, s>>>(map, m, q.Q, qual, status);
     return cudaGetLastError();
+}
+
+cudaError_t launch_mlp_tc_scores(const TcModel &m, const Queries &q, const float *qual,
+                                 int32_t *status, cudaStream_t s) {
+    if (q.Q <= 0) return cudaSuccess;
+    if (q.Q > BM || !q.no_select || !q.pair_C) return cudaErrorInvalidValue;
+    // one tile: split its deployments into one part per SM
+    const int sms = g_num_sms > 0 ? g_num_sms : 1;
+    const int ns = m.D < sms ? m.D : sms;
+    return launch_mlp_tc(m, q, qual, ns, nullptr, nullptr, status, s);
 }
 
 // Deployment split per tile that minimises the busiest CTA's step count

@@ -96,12 +96,13 @@ def test_route_before_snapshot_and_argument_errors():
     assert lib.hwr_destroy(ctx) == 0
 
 
-def test_sequential_tensor_combination_unsupported():
-    p = W.make_config(1, Q=600)
+def test_sequential_tensor_needs_a_bf16_context():
+    p = W.make_config(2, Q=100)            # fp32: no tensor-core path
     r = H.Router(p)
     with pytest.raises(H.HwrError) as e:
         r.route(flags=H.HWR_SEQUENTIAL | H.HWR_PATH_TENSOR)
     assert e.value.status == _hwr.HWR_ERR_UNSUPPORTED
+    assert r.route(flags=H.HWR_SEQUENTIAL)[0].shape == (100,)     # still usable
     r.close()
 
 

@@ -227,3 +227,43 @@ def test_tensor_route_after_sequential_sees_the_increments():
     r.update_snapshot(p["snap"])
     check_against_oracle(p, r.route(flags=H.HWR_PATH_TENSOR))
     r.close()
+
+
+# ---------------------------------------------------------------------------
+# sequential mode with the score table on the tensor cores (HWR_SEQUENTIAL |
+# HWR_PATH_TENSOR): every query's choice is checked against the fp64 oracle
+# at the running counts the GPU's own earlier picks imply (a near tie may go
+# the other way, after which the counts legitimately differ from the
+# canonical run), and the persisted counts must be exactly those picks
+
+def _replay_check(p, got):
+    ch, lat, util = got
+    D = p["D"]
+    r0 = np.asarray(p["snap"]["running"], np.int64)
+    clear = []
+    for i in range(len(ch)):
+        prev = ch[:i][ch[:i] >= 0]
+        snap = dict(p["snap"])
+        snap["running"] = (r0 + np.bincount(prev, minlength=D)).astype(np.int32)
+        pi = dict(W.query_subset(p, [i]), snap=snap)
+        clear.append(check_against_oracle(pi, (ch[i:i + 1], lat[i:i + 1], util[i:i + 1]),
+                                          min_checked=0.0))
+    return float(np.mean(clear))
+
+
+@pytest.mark.parametrize("c,Q", [(1, 150), (4, 70), (3, 45)])
+def test_sequential_tensor_table_valid(c, Q):
+    p = W.make_config(c, Q=Q)
+    r = H.Router(p)
+    got = r.route(flags=H.HWR_SEQUENTIAL | H.HWR_PATH_TENSOR)
+    final = r.get_snapshot()
+    canon = None
+    r.update_snapshot(p["snap"])
+    canon = r.route(flags=H.HWR_SEQUENTIAL)           # canonical fp32 order
+    r.close()
+    ch = got[0]
+    assert np.array_equal(final, np.asarray(p["snap"]["running"]) +
+                          np.bincount(ch[ch >= 0], minlength=p["D"]))
+    assert _replay_check(p, got) >= 0.5
+    # most decisions agree with the canonical run
+    assert np.mean(ch == canon[0]) >= 0.5
