@@ -104,9 +104,8 @@ struct hwr_ctx {
     float *ctab = nullptr;   size_t ctab_cap = 0;
     float *qseq = nullptr;   size_t qseq_cap = 0;
     int seq_qs = 0;
-    // sequential mode with the table on the tensor cores: costs [Qs][D (Qs+1)],
-    // bf16 prefixes [D (Qs+1)][H1], model of each (deployment, count) group
-    float *ptab = nullptr;   size_t ptab_cap = 0;
+    // sequential mode with the table on the tensor cores: bf16 prefixes
+    // [D (Qs+1)][H1], model of each (deployment, count) group
     uint16_t *prebf = nullptr; size_t prebf_cap = 0;
     int32_t *dmv = nullptr;  size_t dmv_cap = 0;
     int seq_slots = 0;       // sequential-table blocks resident at once
@@ -631,13 +630,11 @@ static hwr_status run_kernels(hwr_ctx *c, const Queries &q, uint32_t flags, bool
         const bool tcs = (flags & HWR_PATH_TENSOR) && c->tc_ok;
         if (tcs) {
             const size_t Dv = (size_t)c->D * (Qs + 1);
-            TRY(grow(c, &c->ptab, &c->ptab_cap, (size_t)Qs * Dv));
             TRY(grow(c, &c->prebf, &c->prebf_cap, Dv * c->H1));
             TRY(grow(c, &c->dmv, &c->dmv_cap, Dv));
             TRY(grow(c, &c->qual, &c->qual_cap, (size_t)Qs * c->Mpad));
-        } else {
-            TRY(grow(c, &c->ctab, &c->ctab_cap, seq_table_floats(c->D, Qs)));
         }
+        TRY(grow(c, &c->ctab, &c->ctab_cap, seq_table_floats(c->D, Qs)));
         TRY(grow(c, &c->qseq, &c->qseq_cap, seq_aux_floats(c->D, c->M, c->H1, Qs)));
         const size_t es = c->dtype == HWR_BF16 ? 2 : 4;
         for (int lo = 0; lo < q.Q; lo += Qs) {
@@ -665,7 +662,8 @@ static hwr_status run_kernels(hwr_ctx *c, const Queries &q, uint32_t flags, bool
                 tv.Abf = c->prebf;
                 tv.dep_model = c->dmv;
                 Queries kt = k;
-                kt.pair_C = c->ptab;
+                kt.pair_C = c->ctab;
+                kt.seq_n = n;
                 kt.no_select = 1;
                 kt.slo_mode = 0;      // budgets are the chain's business
                 kt.slo_q = nullptr;
@@ -676,7 +674,7 @@ static hwr_status run_kernels(hwr_ctx *c, const Queries &q, uint32_t flags, bool
                 CK(c, launch_mlp_tc_scores(tv, kt, c->qual, c->status_d, c->stream),
                    "sequential table (tensor cores)");
                 a.done();
-                CK(c, launch_seq_chain_tc(m, k, n, c->ptab, c->qseq, c->qual, c->Mpad, c->stream),
+                CK(c, launch_seq_chain_tc(m, k, n, c->ctab, c->qseq, c->qual, c->Mpad, c->stream),
                    "sequential chain");
                 // preparation, quality and chain beside the scope's table kernel
                 c->stats.kernel_launches += 3;

@@ -65,7 +65,22 @@ struct Queries {
     // when set, the tensor-core predictor kernel only stores pair_C (no
     // decision outputs, no partial results)
     int no_select = 0;
+    // sequential table on the tensor cores: when > 0, deployment v of the
+    // predictor is (deployment v / (seq_n + 1), count v % (seq_n + 1)) and
+    // pair_C is the triangular sequential table of seq_n queries (tab_row)
+    int seq_n = 0;
 };
+
+// The sequential score table of a chunk of Qs queries over D deployments:
+// entry (picks so far c, deployment d, query i >= c) sits at
+//   D * (c * Qs - c (c - 1) / 2) + d * (Qs - c) + (i - c);
+// tri_off(c) is the offset of count c's block, tab_row(c, d) + i the entry.
+__host__ __device__ inline size_t tri_off(int D, int Qs, int c) {
+    return (size_t)D * ((size_t)c * Qs - (size_t)c * (c - 1) / 2);
+}
+__host__ __device__ __forceinline__ int tab_row(int D, int Qs, int c, int d) {
+    return D * (c * Qs - (c * (c - 1)) / 2) + d * (Qs - c) - c;
+}
 
 // Several values of lambda applied to one set of scores.
 constexpr int MAX_LAMBDAS = 16;
@@ -116,12 +131,12 @@ cudaError_t launch_seq_chain(const Model &m, const Queries &q, int Qs,
 size_t seq_aux_floats(int D, int M, int H1, int Qs);
 // Sequential mode with the table on the tensor cores (bf16 contexts): the
 // preparation kernel alone, also writing bf16 prefixes pre_bf [D (Qs + 1)][H1]
-// and the model of each (deployment, count) group dmv [D (Qs + 1)]; the chain
-// over a table of costs ptab [Qs][D (Qs + 1)] (query i, group d (Qs + 1) + c)
-// with quality rows qual [Qs][qstride].
+// and the model of each (deployment, count) group dmv [D (Qs + 1)] (group
+// d (Qs + 1) + c); the chain over the triangular table ctab (written by the
+// predictor kernel with q.seq_n = Qs) with quality rows qual [Qs][qstride].
 cudaError_t launch_seq_prep_tc(const Model &m, const Queries &q, int Qs, float *aux,
                                uint16_t *pre_bf, int32_t *dmv, cudaStream_t s);
-cudaError_t launch_seq_chain_tc(const Model &m, const Queries &q, int Qs, const float *ptab,
+cudaError_t launch_seq_chain_tc(const Model &m, const Queries &q, int Qs, const float *ctab,
                                 float *aux, const float *qual, int qstride, cudaStream_t s);
 int seq_table_slots(const Model &m);
 // Decision maker for K lambdas from stored scores: C [Q][D], quality

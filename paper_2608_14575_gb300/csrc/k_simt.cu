@@ -505,10 +505,6 @@ __global__ void __launch_bounds__(ROUTE_THREADS, CPT <= 4 ? 3 : 2) k_route_simt(
 //   index = D * (c * Qs - c (c - 1) / 2) + d * (Qs - c) + (i - c).
 // A table block takes an equal run of consecutive entries.
 
-__host__ __device__ inline size_t tri_off(int D, int Qs, int c) {
-    return (size_t)D * ((size_t)c * Qs - (size_t)c * (c - 1) / 2);
-}
-
 size_t seq_table_floats(int D, int Qs) { return tri_off(D, Qs, Qs); }
 
 // Per-chunk auxiliary arrays (one scratch buffer, seq_aux_floats floats):
@@ -538,8 +534,12 @@ size_t seq_aux_floats(int D, int M, int H1, int Qs) {
 // K_seq_prep: the chunk's standardised features and layer-1 prefixes, each
 // computed once (double arithmetic is scarce on this GPU, and every table
 // block would otherwise repeat it).  Blocks [0, nuv): the query slots; then
-// one block per (d, c).
+// one block per deployment d and run of PREP_COUNTS counts c.
 constexpr int PREP_THREADS = 128;
+constexpr int PREP_COUNTS = 8;   // counts c per preparation block
+__host__ __device__ inline int seq_prep_blocks_per_dep(int Qs) {
+    return (Qs + PREP_COUNTS) / PREP_COUNTS;   // counts 0 .. Qs
+}
 
 __global__ void __launch_bounds__(PREP_THREADS)
 k_seq_prep(Model m, Queries q, int Qs, float *aux, uint16_t *pre_bf, int32_t *dmv) {
@@ -557,23 +557,44 @@ k_seq_prep(Model m, Queries q, int Qs, float *aux, uint16_t *pre_bf, int32_t *dm
         }
         return;
     }
-    const int g = blockIdx.x - nuv, d = g / (Qs + 1), c = g - d * (Qs + 1);
-    __shared__ float xr;
-    if (tid == 0) {
-        xr = standardise(m.xform[P + 1], (double)(m.running[d] + c), m.mu[P + 1], m.sd[P + 1]);
-        a.xr[g] = xr;
-        if (dmv) dmv[g] = m.dep_model[d];
+    // block: deployment d, counts c0 .. c0 + cn - 1
+    const int nc = seq_prep_blocks_per_dep(Qs);
+    const int gb = blockIdx.x - nuv, d = gb / nc, c0 = (gb - d * nc) * PREP_COUNTS;
+    const int cn = Qs + 1 - c0 < PREP_COUNTS ? Qs + 1 - c0 : PREP_COUNTS;
+    const int g0 = d * (Qs + 1) + c0;
+    __shared__ float xr[PREP_COUNTS];
+    if (tid < cn) {
+        const float v = standardise(m.xform[P + 1], (double)(m.running[d] + c0 + tid), m.mu[P + 1],
+                                    m.sd[P + 1]);
+        xr[tid] = v;
+        a.xr[g0 + tid] = v;
+        if (dmv) dmv[g0 + tid] = m.dep_model[d];
+    } else if (tid < PREP_COUNTS) {
+        xr[tid] = 0.f;   // past the last count: computed, never stored
     }
     __syncthreads();
-    // continue the chain from slot P + 1 (running) with the deployment's other features
-    // (W1 read slot-major: a warp's loads of one slot are contiguous)
+    // continue the chain from slot P + 1 (running) with the deployment's other
+    // features, every count of the block at once (W1 read slot-major: a warp's
+    // loads of one slot are contiguous)
+    const float *x = m.X + (size_t)d * F;
     for (int j = tid; j < H1; j += PREP_THREADS) {
-        const float *x = m.X + (size_t)d * F;
-        float acc = m.Spre[(size_t)d * H1 + j];
-        acc = __fmaf_rn(m.W1T[(size_t)(P + 1) * H1 + j], xr, acc);
-        for (int k = P + 2; k < F - 2; ++k) acc = __fmaf_rn(m.W1T[(size_t)k * H1 + j], x[k], acc);
-        a.pre[(size_t)g * H1 + j] = acc;
-        if (pre_bf) pre_bf[(size_t)g * H1 + j] = __bfloat16_as_ushort(__float2bfloat16_rn(acc));
+        const float s0 = m.Spre[(size_t)d * H1 + j], w = m.W1T[(size_t)(P + 1) * H1 + j];
+        float acc[PREP_COUNTS];
+#pragma unroll
+        for (int c = 0; c < PREP_COUNTS; ++c) acc[c] = __fmaf_rn(w, xr[c], s0);
+        for (int k = P + 2; k < F - 2; ++k) {
+            const float wk = m.W1T[(size_t)k * H1 + j], xk = x[k];
+#pragma unroll
+            for (int c = 0; c < PREP_COUNTS; ++c) acc[c] = __fmaf_rn(wk, xk, acc[c]);
+        }
+#pragma unroll
+        for (int c = 0; c < PREP_COUNTS; ++c) {
+            if (c < cn) {
+                a.pre[(size_t)(g0 + c) * H1 + j] = acc[c];
+                if (pre_bf)
+                    pre_bf[(size_t)(g0 + c) * H1 + j] = __bfloat16_as_ushort(__float2bfloat16_rn(acc[c]));
+            }
+        }
     }
 }
 
@@ -683,11 +704,6 @@ __host__ __device__ inline size_t chain_tab_floats(int D, int Qs) {
     return (tri_off(D, Qs, Qs) + 3) & ~(size_t)3;
 }
 
-// Offset of the table entry (picks c, deployment d, query 0) (only i >= c is stored).
-__device__ __forceinline__ int tab_row(int D, int Qs, int c, int d) {
-    return D * (c * Qs - (c * (c - 1)) / 2) + d * (Qs - c) - c;
-}
-
 // The decision maker's candidate order as one 40-bit integer: class + 1
 // (bits 38-39), the key within the class (bits 6-37: larger U for a
 // feasible candidate, smaller C for an infeasible one, as order-preserving
@@ -709,7 +725,7 @@ __device__ __forceinline__ uint64_t cand_key(float C, float U, int d, float slo)
 }
 
 __global__ void __launch_bounds__(CHAIN_THREADS)
-k_seq_chain(Model m, Queries q, int Qs, const float *ctab, int Dv, float *aux, const float *qsrc,
+k_seq_chain(Model m, Queries q, int Qs, const float *ctab, float *aux, const float *qsrc,
             int qstride) {
     extern __shared__ float4 sm4[];
     float *sm = reinterpret_cast<float *>(sm4);
@@ -730,27 +746,13 @@ k_seq_chain(Model m, Queries q, int Qs, const float *ctab, int Dv, float *aux, c
     for (int e = tid; e < D; e += CHAIN_THREADS) dm[e] = m.dep_model[e];
     umma::grid_dependency_wait();
     const uint32_t tab_s = (uint32_t)__cvta_generic_to_shared(tab);
-    if (Dv == 0) {
-        // the triangular table, by 16-byte asynchronous copies (both sides
-        // 16-byte aligned)
-        for (size_t e = tid; e < T / 4; e += CHAIN_THREADS)
-            asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(tab_s + (uint32_t)(16 * e)),
-                         "l"(__cvta_generic_to_global(ctab + 4 * e))
-                         : "memory");
-        for (size_t e = T / 4 * 4 + tid; e < T; e += CHAIN_THREADS) tab[e] = __ldcg(ctab + e);
-    } else {
-        // costs per (query i, virtual deployment d (Qs + 1) + c) [Qs][Dv]:
-        // gather the entries with c <= i into the triangular layout, one
-        // (c, d) group per warp at a time
-        for (int g = tid >> 5; g < D * Qs; g += CHAIN_THREADS / 32) {
-            const int c = g / D, d = g - c * D, row = tab_row(D, Qs, c, d);
-            for (int i = c + lane; i < Qs; i += 32)
-                asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(
-                                 tab_s + 4u * (uint32_t)(row + i)),
-                             "l"(__cvta_generic_to_global(ctab + (size_t)i * Dv + d * (Qs + 1) + c))
-                             : "memory");
-        }
-    }
+    // the triangular table, by 16-byte asynchronous copies (both sides
+    // 16-byte aligned)
+    for (size_t e = tid; e < T / 4; e += CHAIN_THREADS)
+        asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(tab_s + (uint32_t)(16 * e)),
+                     "l"(__cvta_generic_to_global(ctab + 4 * e))
+                     : "memory");
+    for (size_t e = T / 4 * 4 + tid; e < T; e += CHAIN_THREADS) tab[e] = __ldcg(ctab + e);
     asm volatile("cp.async.commit_group;" ::: "memory");
     for (int e = tid; e < Qs * M; e += CHAIN_THREADS) {
         const int i = e / M;
@@ -1158,7 +1160,7 @@ cudaError_t launch_select_multi(const Model &m, const Queries &q, const float *C
 cudaError_t launch_seq_table(const Model &m, const Queries &q, int Qs, int slots, float *ctab,
                              float *aux, cudaStream_t s) {
     const int nuv = (2 * Qs + PREP_THREADS - 1) / PREP_THREADS;
-    k_seq_prep<<<nuv + m.D * (Qs + 1), PREP_THREADS, 0, s>>>(m, q, Qs, aux, nullptr, nullptr);
+    k_seq_prep<<<nuv + m.D * seq_prep_blocks_per_dep(Qs), PREP_THREADS, 0, s>>>(m, q, Qs, aux, nullptr, nullptr);
     // rows per table block: a multiple of 8 (whole warps of the tile) that
     // spreads the table evenly over the blocks resident at once
     const int T = (int)tri_off(m.D, Qs, Qs);
@@ -1197,21 +1199,20 @@ cudaError_t launch_seq_chain(const Model &m, const Queries &q, int Qs, const flo
                              float *aux, cudaStream_t s) {
     cudaLaunchConfig_t cfg = dependent_launch(1, CHAIN_THREADS, chain_smem(m.D, m.M, Qs), s);
     const SeqAux A = seq_aux(aux, m.D, m.M, Qs);
-    return cudaLaunchKernelEx(&cfg, k_seq_chain, m, q, Qs, ctab, 0, aux, (const float *)A.qual, m.M);
+    return cudaLaunchKernelEx(&cfg, k_seq_chain, m, q, Qs, ctab, aux, (const float *)A.qual, m.M);
 }
 
 cudaError_t launch_seq_prep_tc(const Model &m, const Queries &q, int Qs, float *aux,
                                uint16_t *pre_bf, int32_t *dmv, cudaStream_t s) {
     const int nuv = (2 * Qs + PREP_THREADS - 1) / PREP_THREADS;
-    k_seq_prep<<<nuv + m.D * (Qs + 1), PREP_THREADS, 0, s>>>(m, q, Qs, aux, pre_bf, dmv);
+    k_seq_prep<<<nuv + m.D * seq_prep_blocks_per_dep(Qs), PREP_THREADS, 0, s>>>(m, q, Qs, aux, pre_bf, dmv);
     return cudaGetLastError();
 }
 
-cudaError_t launch_seq_chain_tc(const Model &m, const Queries &q, int Qs, const float *ptab,
+cudaError_t launch_seq_chain_tc(const Model &m, const Queries &q, int Qs, const float *ctab,
                                 float *aux, const float *qual, int qstride, cudaStream_t s) {
     cudaLaunchConfig_t cfg = dependent_launch(1, CHAIN_THREADS, chain_smem(m.D, m.M, Qs), s);
-    return cudaLaunchKernelEx(&cfg, k_seq_chain, m, q, Qs, ptab, m.D * (Qs + 1), aux, qual,
-                              qstride);
+    return cudaLaunchKernelEx(&cfg, k_seq_chain, m, q, Qs, ctab, aux, qual, qstride);
 }
 
 }  // namespace hwr

@@ -552,7 +552,17 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
                 // N_out of Eq. 2: the third head, or the query's given length
                 const float C = fmaf(NH == 3 ? softplus_fast(z2) : ol, tpot, ttft);
                 const float U = fmaf(-lam, C, wq * qs[r * QS + dms[d]]);
-                if (q.pair_C && valid) q.pair_C[(size_t)row * D + d] = C;
+                if (q.pair_C && valid) {
+                    if (q.seq_n == 0) {
+                        q.pair_C[(size_t)row * D + d] = C;
+                    } else {
+                        // (deployment, count) slot d: keep the entries with
+                        // count <= query (the lanes of a warp write
+                        // consecutive queries of one table row)
+                        const int np = q.seq_n + 1, dd = d / np, cc = d - dd * np;
+                        if (cc <= row) q.pair_C[tab_row(D / np, q.seq_n, cc, dd) + row] = C;
+                    }
+                }
                 const Cand cd = make_cand(C, U, d, slo_r);
                 if (better(cd, best)) best = cd;
             }
@@ -792,6 +802,7 @@ cudaError_t launch_mlp_tc_scores(const TcModel &m, const Queries &q, const float
                                  int32_t *status, cudaStream_t s) {
     if (q.Q <= 0) return cudaSuccess;
     if (q.Q > BM || !q.no_select || !q.pair_C) return cudaErrorInvalidValue;
+    if (q.seq_n && (q.seq_n != q.Q || m.D % (q.seq_n + 1))) return cudaErrorInvalidValue;
     // one tile: split its deployments into one part per SM
     const int sms = g_num_sms > 0 ? g_num_sms : 1;
     const int ns = m.D < sms ? m.D : sms;
