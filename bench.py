@@ -325,6 +325,34 @@ def config_latencies(H, stream, dev, calls=300):
                       "requests_per_s": float(n / (np.median(a) * 1e-6)),
                       "note": "snapshot upload + sequential route of one micro-batch, "
                               "host buffers, wall clock"}
+    # sequential mode on a bf16 cluster (the sweep's shapes, D = 32, H = 256):
+    # the score table on the SIMT path (canonical fp32 order) and on the
+    # tensor cores (HWR_PATH_TENSOR)
+    p = W.make_config(4, Q=64 * 50)
+    r = H.Router(p)
+    seq = {}
+    gc.collect()
+    gc.disable()
+    for name, fl in (("simt_table", H.HWR_SEQUENTIAL),
+                     ("tensor_table", H.HWR_SEQUENTIAL | H.HWR_PATH_TENSOR)):
+        times = []
+        for k in range(120):
+            lo = (k % 50) * n
+            t = time.perf_counter()
+            r.update_snapshot(p["snap"])
+            r.route(p["in_len"][lo:lo + n], p["out_len"][lo:lo + n], p["emb"][lo:lo + n],
+                    flags=fl)
+            if k >= 20:
+                times.append(time.perf_counter() - t)
+        a = np.array(times) * 1e6
+        seq[name] = {"p50_us": float(np.median(a)), "p99_us": float(np.percentile(a, 99)),
+                     "requests_per_s": float(n / (np.median(a) * 1e-6))}
+    gc.enable()
+    r.close()
+    out["sequential_bf16"] = {"workload": workload_name(p) + ", micro-batches of 64, sequential",
+                              "calls": 100, **seq,
+                              "note": "snapshot upload + sequential route of one micro-batch, "
+                                      "host buffers, wall clock"}
     return out
 
 
