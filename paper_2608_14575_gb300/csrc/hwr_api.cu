@@ -36,17 +36,17 @@ struct AllocHook {
 // kernel; larger bf16 batches of at least tc_min_pairs pairs take the
 // tensor-core kernels; the rest the fused SIMT kernel.  pairs_max is
 // SMALL_MAX_PAIRS where the tensor-core path exists; otherwise FP32_MAX_PAIRS
-// for hidden layers wider than 64 x 64 and SMALL_MAX_PAIRS for narrower ones.
+// for hidden layers wider than 64 x 64 and 0 for narrower ones.
 // (Device pointers, isolated calls.  bf16: the tensor path costs 31-33 us at
 // D = 32 and 38-40 us at D = 64 for 1 to 64 queries; the small-batch kernel
 // is ahead up to 256 pairs and behind from 512 on.  fp32: the fused kernel
-// costs ~21.5 us at H = 32 and ~33.5 us at H = 128 from 1 to 512 queries;
-// the small-batch kernel costs 20.5-21 us at H = 32 up to 256 pairs and more
-// beyond, 23.6-38 us at H = 128 for 1-64 queries: ahead up to ~500 pairs.)
+// costs ~21 us at H = 32 and ~33 us at H = 128 from 1 to 512 queries; the
+// small-batch kernel costs ~24 us at H = 32 whatever the size, and 25.5-29 us
+// at H = 128, D = 12 from 1 to 170 queries (2,040 pairs).)
 constexpr int TC_MIN_PAIRS = 257;
 constexpr int PIPE_CHUNK_MIN = 8192;   // smallest chunk of a pipelined host batch
 constexpr int SMALL_MAX_PAIRS = 256;
-constexpr int FP32_MAX_PAIRS = 512;
+constexpr int FP32_MAX_PAIRS = PAIRS_MAX_PAIRS;
 
 }  // namespace
 
@@ -99,6 +99,7 @@ struct hwr_ctx {
     char *part = nullptr;    size_t part_cap = 0;     // split-deployment partials
     int32_t *count = nullptr; size_t count_cap = 0;   // per-row arrivals (self-resetting)
     float *pairC = nullptr;  float *pairQ = nullptr;  int32_t *pairN = nullptr;  // small batches
+    float *pairH = nullptr;
     float *mC = nullptr;     size_t mC_cap = 0;       // multi-lambda: pair costs [Q][D]
     float *mQ = nullptr;     size_t mQ_cap = 0;       // multi-lambda: quality [Q][M]
     float *ctab = nullptr;   size_t ctab_cap = 0;
@@ -423,7 +424,8 @@ static hwr_status build_ctx(hwr_ctx *c, const hwr_deployment_table *t, const hwr
     TRY(dev_alloc(c, &c->W1T, (size_t)F * H1));
     TRY(dev_alloc(c, &c->pairC, (size_t)PAIRS_MAX_PAIRS));
     TRY(dev_alloc(c, &c->pairQ, (size_t)PAIRS_MAX_PAIRS * M));
-    TRY(dev_alloc(c, &c->pairN, (size_t)PAIRS_MAX_PAIRS));
+    TRY(dev_alloc(c, &c->pairN, 2 * (size_t)PAIRS_MAX_PAIRS));
+    TRY(dev_alloc(c, &c->pairH, (size_t)PAIRS_MAX_PAIRS * H2));
     // the six snapshot arrays, contiguous: an upload lands in them directly
     TRY(dev_alloc(c, (char **)&c->snap_d, 6 * (size_t)D * 4));
     c->running = (int32_t *)c->snap_d;
@@ -464,7 +466,7 @@ static hwr_status build_ctx(hwr_ctx *c, const hwr_deployment_table *t, const hwr
     for (int j = 0; j < H1; ++j)
         for (int k = 0; k < F; ++k) w1t[(size_t)k * H1 + j] = w1[(size_t)j * F + k];
     TRY(upload(c, c->W1T, w1t.data(), w1t.size() * 4, "upload W1 transposed"));
-    CK(c, cudaMemset(c->pairN, 0, PAIRS_MAX_PAIRS * sizeof(int32_t)), "zero counters");
+    CK(c, cudaMemset(c->pairN, 0, 2 * PAIRS_MAX_PAIRS * sizeof(int32_t)), "zero counters");
     c->mu_in = p->feat_mean[F - 2]; c->sd_in = p->feat_std[F - 2]; c->xf_in = p->feat_xform[F - 2];
     c->mu_out = p->feat_mean[F - 1]; c->sd_out = p->feat_std[F - 1]; c->xf_out = p->feat_xform[F - 1];
 
@@ -569,7 +571,7 @@ extern "C" hwr_status hwr_create(const hwr_deployment_table *table, const hwr_pr
         return s;
     }
     if (c->pairs_max < 0)
-        c->pairs_max = !c->tc_ok && c->H1 * c->H2 > 64 * 64 ? FP32_MAX_PAIRS : SMALL_MAX_PAIRS;
+        c->pairs_max = c->tc_ok ? SMALL_MAX_PAIRS : c->H1 * c->H2 > 64 * 64 ? FP32_MAX_PAIRS : 0;
     *out = c;
     return HWR_OK;
 }
@@ -714,7 +716,7 @@ static hwr_status run_kernels(hwr_ctx *c, const Queries &q, uint32_t flags, bool
     }
     LaunchScope a(c, HWR_K_ROUTE_SIMT, prof);
     if ((long)q.Q * c->D <= c->pairs_max)
-        CK(c, launch_route_pairs(m, q, c->pairC, c->pairQ, c->pairN, c->stream),
+        CK(c, launch_route_pairs(m, q, c->pairC, c->pairQ, c->pairH, c->pairN, c->stream),
            "route kernel");
     else
         CK(c, launch_route_simt(m, q, c->stream), "route kernel");

@@ -110,12 +110,14 @@ __device__ __forceinline__ float query_budget(const Queries &q, int row) {
 cudaError_t launch_snapshot(const Model &m, const uint32_t *stage, cudaStream_t s);
 // Fused gather -> MLP -> mask -> argmax for a batch.
 cudaError_t launch_route_simt(const Model &m, const Queries &q, cudaStream_t s);
-// Small-batch (latency) variant: one block per (query, deployment) pair plus
-// quality blocks; scratch pairC [Q][D], qualS [Q][M], count [Q] (zeroed once,
-// self-resetting).  Reads W2 through m.W2T.
+// Small-batch (latency) variant: groups of (query, deployment) pairs with
+// layer 2 split by columns over several blocks, plus quality blocks; scratch
+// pairC [Q][D], qualS [Q][M], h2 [Q D][H2], count [2 PAIRS_MAX_PAIRS] (query
+// and group arrivals; zeroed once, self-resetting).  Q * D <= PAIRS_MAX_PAIRS.
+// Reads W2 through m.W2T and layer 1's query columns through m.W1T.
 constexpr int PAIRS_MAX_PAIRS = 2048;   // default upper bound on Q * D for this kernel
 cudaError_t launch_route_pairs(const Model &m, const Queries &q, float *pairC, float *qualS,
-                               int32_t *count, cudaStream_t s);
+                               float *h2, int32_t *count, cudaStream_t s);
 size_t route_pairs_smem(const Model &m);
 // Sequential mode over one chunk of Qs <= seq_chunk(m) queries: the chunk's
 // standardised features and layer-1 prefixes, and the score table (every

@@ -879,24 +879,36 @@ k_seq_chain(Model m, Queries q, int Qs, const float *ctab, float *aux, const flo
 }
 
 // ---------------------------------------------------------------------------
-// K_route_pairs: the small-batch (latency) variant.  One block per (query,
-// deployment) pair computes that pair's predictor with one thread per hidden
-// unit (W2 read transposed so a warp's loads are contiguous); quality blocks
-// run the per-(query, model) chains from shared memory; the last block to
-// finish a query (per-query arrival counter, self-resetting) applies the
-// decision maker.  Same canonical order as the kernels above.
+// K_route_pairs: the small-batch (latency) variant.  The (query, deployment)
+// pairs p = qq D + d are taken in groups of PAIR_G consecutive pairs, and a
+// group's layer 2 is split by columns over ncb = ceil(H2 / PAIR_COLS) blocks:
+// each stages its W2 columns (16-byte async copies) and the group's layer-1
+// rows in shared memory, runs its columns' serial chains (warp w: columns
+// 4w .. 4w + 3, lane: pair, so a W2 load is a broadcast) and stores them to a
+// scratch h2 [groups][H2][PAIR_G].  The last column block of a group (arrival
+// counter, self-resetting) copies the group's h2 block back with 16-byte
+// async copies and runs the head chains and the cost of Eq. 2.
+// Quality blocks run the per-(query, model) chains from shared memory.  A
+// query is decided by the block that completes its count of D pairs and
+// qblocks quality blocks (self-resetting).  Same canonical order as the
+// kernels above: every chain is the same sequence of roundings.
 
 struct PairArgs {
     float *pairC;       // [Q][D] scratch
     float *qualS;       // [Q][M] scratch
+    float *h2;          // [groups][H2][PAIR_G] scratch
     int32_t *count;     // [Q] arrivals, zero between calls
+    int32_t *gcount;    // [groups] column-block arrivals, zero between calls
     int qblocks;        // quality blocks per query
+    int ncb;            // column blocks per group
 };
 
-constexpr int PAIR_MPB = 8;  // models per quality block
+constexpr int PAIR_MPB = 8;    // models per quality block
+constexpr int PAIR_G = 32;     // pairs per group
+constexpr int PAIR_COLS = 32;  // layer-2 columns per block
 
 __device__ void pair_select(const Model &m, const Queries &q, const PairArgs &a, int qq) {
-    // warp 0 of the last block of query qq: utility, SLO mask, argmax
+    // one warp: utility, SLO mask, argmax over the query's stored costs
     const int lane = threadIdx.x & 31;
     Cand best = no_cand();
     const float slo = query_budget(q, qq);
@@ -917,96 +929,208 @@ __device__ void pair_select(const Model &m, const Queries &q, const PairArgs &a,
     }
 }
 
+__host__ __device__ inline int pair_groups(int npair) { return (npair + PAIR_G - 1) / PAIR_G; }
+
 __global__ void __launch_bounds__(SIMT_THREADS) k_route_pairs(Model m, Queries q, PairArgs a) {
-    extern __shared__ float sm[];
+    extern __shared__ float4 sm4[];   // 16-byte aligned: W2 columns arrive as 16-byte copies
+    float *sm = reinterpret_cast<float *>(sm4);
     __shared__ int s_last;
-    const int tid = threadIdx.x, F = m.F, H1 = m.H1, H2 = m.H2, D = m.D, M = m.M;
-    const int npair = q.Q * D;
-    int qq;
-    if ((int)blockIdx.x < npair) {
-        qq = blockIdx.x / D;
-        const int d = blockIdx.x - qq * D;
-        float *h1 = sm, *h2 = sm + MAX_H;
-        __shared__ float uv[3];
-        // the two query slots on two warps (their fp64 chains run side by side)
-        if (tid == 0) {
-            uv[0] = standardise(m.xform[F - 2], (double)q.in_len[qq], m.mu[F - 2], m.sd[F - 2]);
-        } else if (tid == 32) {
-            const float o = q.out_len[qq];
-            uv[1] = standardise(m.xform[F - 1], (double)o, m.mu[F - 1], m.sd[F - 1]);
-            uv[2] = o;
-        }
-        __syncthreads();
-        for (int k = tid; k < H1; k += SIMT_THREADS) {
-            const float *w = m.W1 + (size_t)k * F;
-            float x = m.A[(size_t)d * H1 + k];
-            x = __fmaf_rn(w[F - 2], uv[0], x);
-            x = __fmaf_rn(w[F - 1], uv[1], x);
-            h1[k] = x > 0.f ? x : 0.f;
-        }
-        __syncthreads();
-        float *w3s = sm + 2 * MAX_H;   // W3 [NH][H2], staged for the head chains
-        for (int i = tid; i < m.NH * H2; i += SIMT_THREADS) w3s[i] = m.W3[i];
-        for (int n = tid; n < H2; n += SIMT_THREADS) {
-            // serial chain over k (canonical order); W2 values fetched 32 at a
-            // time, the next block in flight while this one is accumulated
-            float acc = m.b2[n];
-            float w[32], wn[32];
-#pragma unroll
-            for (int j = 0; j < 32; ++j) w[j] = j < H1 ? m.W2T[(size_t)j * m.H2p + n] : 0.f;
-            for (int k0 = 0; k0 < H1; k0 += 32) {
-#pragma unroll
-                for (int j = 0; j < 32; ++j)
-                    wn[j] = k0 + 32 + j < H1 ? m.W2T[(size_t)(k0 + 32 + j) * m.H2p + n] : 0.f;
-#pragma unroll
-                for (int j = 0; j < 32; ++j)
-                    if (k0 + j < H1) acc = __fmaf_rn(w[j], h1[k0 + j], acc);
-#pragma unroll
-                for (int j = 0; j < 32; ++j) w[j] = wn[j];
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int F = m.F, H1 = m.H1, H2 = m.H2, D = m.D, M = m.M;
+    const int npair = q.Q * D, ncolb = pair_groups(npair) * a.ncb;
+    if ((int)blockIdx.x < ncolb) {
+        const int g = blockIdx.x / a.ncb, cb = blockIdx.x - g * a.ncb;
+        const int p0 = g * PAIR_G, np = min(PAIR_G, npair - p0);
+        const int q0 = p0 / D, nq = (p0 + np - 1) / D - q0 + 1;   // queries touched, <= PAIR_G
+        const int n0 = cb * PAIR_COLS, nb = min(PAIR_COLS, H2 - n0);
+        float *qu = sm, *qv = sm + PAIR_G, *qo = sm + 2 * PAIR_G;
+        float *w2s = sm + 3 * PAIR_G;               // [H1][PAIR_COLS]
+        const int ld1 = H1 | 1;                     // odd: rows of 4 pairs in distinct banks
+        float *h1s = w2s + (size_t)H1 * PAIR_COLS;  // [PAIR_G][ld1]
+        // W2 columns n0 .. n0 + 31 of every k (only within the padded row)
+        {
+            const int c4n = min(PAIR_COLS, m.H2p - n0) >> 2;
+            const uint32_t base = (uint32_t)__cvta_generic_to_shared(w2s);
+            for (int e = tid; e < H1 * c4n; e += SIMT_THREADS) {
+                const int k = e / c4n, c4 = e - k * c4n;
+                asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(
+                                 base + (uint32_t)(4 * (k * PAIR_COLS + 4 * c4))),
+                             "l"(__cvta_generic_to_global(m.W2T + (size_t)k * m.H2p + n0 + 4 * c4)) : "memory");
             }
-            h2[n] = acc > 0.f ? acc : 0.f;
+            asm volatile("cp.async.commit_group;" ::: "memory");
         }
-        __syncthreads();
-        __shared__ float heads[3];
-        if (tid < 32 * m.NH) {
-            // the output heads, one warp each
-            const int o = tid >> 5;
-            if ((tid & 31) == 0) {
-                const float *w3 = w3s + (size_t)o * H2;
-                float z = m.b3[o];
-                for (int n = 0; n < H2; ++n) z = __fmaf_rn(w3[n], h2[n], z);
-                heads[o] = softplus_c(z);
+        // the query slots of the group's queries (fp64 chains side by side)
+        if (tid < nq) {
+            qu[tid] = standardise(m.xform[F - 2], (double)q.in_len[q0 + tid], m.mu[F - 2], m.sd[F - 2]);
+        } else if (tid >= 32 && tid < 32 + nq) {
+            const float o = q.out_len[q0 + tid - 32];
+            qv[tid - 32] = standardise(m.xform[F - 1], (double)o, m.mu[F - 1], m.sd[F - 1]);
+            qo[tid - 32] = o;
+        }
+        // this thread's unit k of layer 1 for every pair of the group: the
+        // prefix loads first, all in flight together
+        const int k = tid;
+        const bool hk = k < H1;
+        float av[PAIR_G];
+        {
+            int qq = q0, d = p0 - q0 * D;
+#pragma unroll
+            for (int p = 0; p < PAIR_G; ++p) {
+                av[p] = hk && p < np ? m.A[(size_t)d * H1 + k] : 0.f;
+                if (++d == D) {
+                    d = 0;
+                    ++qq;
+                }
             }
         }
+        const float wi = hk ? m.W1T[(size_t)(F - 2) * H1 + k] : 0.f;
+        const float wo = hk ? m.W1T[(size_t)(F - 1) * H1 + k] : 0.f;
         __syncthreads();
-        if (tid == 0)
-            a.pairC[(size_t)qq * D + d] =
-                __fmaf_rn(m.NH == 3 ? heads[2] : uv[2], heads[1], heads[0]);
-    } else {
-        // quality of models [m0, m0 + PAIR_MPB) for one query
-        const int b = blockIdx.x - npair;
-        qq = b / a.qblocks;
-        const int m0 = (b - qq * a.qblocks) * PAIR_MPB, mn = min(PAIR_MPB, M - m0), E = m.E;
-        float *er = sm, *mb = sm + E;   // emb row [E], model columns [mn][E]
-        const size_t row = (size_t)qq * E;
-        for (int k = tid; k < E; k += SIMT_THREADS) {
-            er[k] = emb_at(q.emb, q.emb_bf16, row + k);
-            for (int j = 0; j < mn; ++j) mb[(size_t)j * E + k] = m.memb[(size_t)k * M + m0 + j];
+        if (hk) {
+            int ql = 0, d = p0 - q0 * D;
+#pragma unroll
+            for (int p = 0; p < PAIR_G; ++p) {
+                if (p < np) {
+                    float x = __fmaf_rn(wi, qu[ql], av[p]);
+                    x = __fmaf_rn(wo, qv[ql], x);
+                    h1s[p * ld1 + k] = x > 0.f ? x : 0.f;
+                }
+                if (++d == D) {
+                    d = 0;
+                    ++ql;
+                }
+            }
         }
+        asm volatile("cp.async.wait_all;" ::: "memory");
         __syncthreads();
-        if (tid < mn) {
-            const float *c = mb + (size_t)tid * E;
-            float s = 0.f;
+        // layer 2: thread (pair p = lane, columns c .. c + 3 of warp w), serial over k
+        {
+            const int p = lane, c = 4 * warp;
+            if (p < np && c < nb) {
+                float acc[4];
+#pragma unroll
+                for (int j = 0; j < 4; ++j) acc[j] = c + j < nb ? m.b2[n0 + c + j] : 0.f;
+                const float *hr = h1s + p * ld1;
+                const float *wr = w2s + c;
 #pragma unroll 8
-            for (int k = 0; k < E; ++k) s = __fmaf_rn(er[k], c[k], s);
-            a.qualS[(size_t)qq * M + m0 + tid] = sigmoid_c(s);
+                for (int kk = 0; kk < H1; ++kk) {
+                    const float4 w = *reinterpret_cast<const float4 *>(wr + kk * PAIR_COLS);
+                    const float h = hr[kk];
+                    acc[0] = __fmaf_rn(w.x, h, acc[0]);
+                    acc[1] = __fmaf_rn(w.y, h, acc[1]);
+                    acc[2] = __fmaf_rn(w.z, h, acc[2]);
+                    acc[3] = __fmaf_rn(w.w, h, acc[3]);
+                }
+                float *dst = a.h2 + ((size_t)g * H2 + n0 + c) * PAIR_G + p;
+#pragma unroll
+                for (int j = 0; j < 4; ++j)
+                    if (c + j < nb) dst[j * PAIR_G] = acc[j] > 0.f ? acc[j] : 0.f;
+                __threadfence();   // before the group's arrival below
+            }
+        }
+        __syncthreads();
+        if (tid == 0) {
+            __threadfence();
+            s_last = atomicAdd(&a.gcount[g], 1) == a.ncb - 1;
+        }
+        __syncthreads();
+        if (!s_last) return;
+        // the group's last column block: heads and cost of every pair
+        __threadfence();
+        float *h2s = w2s;                            // [H2][PAIR_G]
+        float *w3s = h2s + (size_t)H2 * PAIR_G;      // [NH][H2]
+        {
+            // the group's whole block (rows of pairs past np are not read),
+            // L2 to shared memory by 16-byte copies that skip L1
+            const uint32_t base = (uint32_t)__cvta_generic_to_shared(h2s);
+            const float *src = a.h2 + (size_t)g * H2 * PAIR_G;
+            for (int e = tid; e < H2 * PAIR_G / 4; e += SIMT_THREADS)
+                asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(base + 16u * e),
+                             "l"(__cvta_generic_to_global(src + 4 * e)) : "memory");
+            asm volatile("cp.async.commit_group;" ::: "memory");
+        }
+        for (int i = tid; i < m.NH * H2; i += SIMT_THREADS) w3s[i] = m.W3[i];
+        asm volatile("cp.async.wait_all;" ::: "memory");
+        __syncthreads();
+        __shared__ float hd[PAIR_G * 3];
+        if (warp < m.NH) {
+            // head o = warp of pair p = lane: W3 reads are broadcasts, h2
+            // reads consecutive words
+            const int o = warp, p = lane;
+            const float *w3 = w3s + (size_t)o * H2;
+            float z = m.b3[o];
+#pragma unroll 8
+            for (int n = 0; n < H2; ++n) z = __fmaf_rn(w3[n], h2s[n * PAIR_G + p], z);
+            if (p < np) hd[p * m.NH + o] = softplus_c(z);
+        }
+        __syncthreads();
+        for (int p = tid; p < np; p += SIMT_THREADS) {
+            const int qq = (p0 + p) / D, NH = m.NH;
+            a.pairC[p0 + p] =
+                __fmaf_rn(NH == 3 ? hd[p * NH + 2] : qo[qq - q0], hd[p * NH + 1], hd[p * NH]);
+        }
+        if (tid == 0) a.gcount[g] = 0;
+        __threadfence();
+        __syncthreads();
+        // each query of the group: its pairs arrive; the warp that completes
+        // the query's count decides it
+        for (int ql = warp; ql < nq; ql += SIMT_THREADS / 32) {
+            const int qq = q0 + ql;
+            const int cnt = min(p0 + np, (qq + 1) * D) - max(p0, qq * D);
+            int done = 0;
+            if (lane == 0) done = atomicAdd(&a.count[qq], cnt) + cnt == D + a.qblocks;
+            done = __shfl_sync(0xffffffffu, done, 0);
+            if (done) {
+                __threadfence();
+                pair_select(m, q, a, qq);
+            }
+        }
+        return;
+    }
+    // quality of models [m0, m0 + PAIR_MPB) for one query
+    const int b = blockIdx.x - ncolb;
+    const int qq = b / a.qblocks;
+    const int m0 = (b - qq * a.qblocks) * PAIR_MPB, mn = min(PAIR_MPB, M - m0), E = m.E;
+    // emb row [E] and the block's model columns as [E / 4][mn][4] (E is a
+    // multiple of 8), so that a chain reads 4 consecutive k of its column as
+    // one 16-byte load and the mn chains' loads fall in distinct banks; a
+    // thread's staging loads are issued before its stores
+    float *er = sm, *mb = sm + E;
+    const size_t row = (size_t)qq * E;
+    for (int k0 = 0; k0 < E; k0 += SIMT_THREADS) {
+        const int k = k0 + tid;
+        const bool ok = k < E;
+        float v[PAIR_MPB];
+        const float ev = ok ? emb_at(q.emb, q.emb_bf16, row + k) : 0.f;
+#pragma unroll
+        for (int j = 0; j < PAIR_MPB; ++j) v[j] = ok && j < mn ? m.memb[(size_t)k * M + m0 + j] : 0.f;
+        if (ok) {
+            er[k] = ev;
+#pragma unroll
+            for (int j = 0; j < PAIR_MPB; ++j)
+                if (j < mn) mb[((size_t)(k >> 2) * mn + j) * 4 + (k & 3)] = v[j];
         }
     }
-    // the last of the query's D + qblocks blocks applies the decision maker
+    __syncthreads();
+    if (tid < mn) {
+        const float4 *c = reinterpret_cast<const float4 *>(mb) + tid;
+        const float4 *e4 = reinterpret_cast<const float4 *>(er);
+        float s = 0.f;
+#pragma unroll 4
+        for (int k4 = 0; k4 < E / 4; ++k4) {
+            const float4 x = e4[k4], y = c[(size_t)k4 * mn];
+            s = __fmaf_rn(x.x, y.x, s);
+            s = __fmaf_rn(x.y, y.y, s);
+            s = __fmaf_rn(x.z, y.z, s);
+            s = __fmaf_rn(x.w, y.w, s);
+        }
+        a.qualS[(size_t)qq * M + m0 + tid] = sigmoid_c(s);
+        __threadfence();
+    }
     __syncthreads();
     if (tid == 0) {
         __threadfence();
-        s_last = atomicAdd(&a.count[qq], 1) == D + a.qblocks - 1;
+        s_last = atomicAdd(&a.count[qq], 1) + 1 == D + a.qblocks;
     }
     __syncthreads();
     if (s_last && tid < 32) {
@@ -1129,20 +1253,27 @@ cudaError_t launch_route_simt(const Model &m, const Queries &q, cudaStream_t s) 
 }
 
 size_t route_pairs_smem(const Model &m) {
-    const size_t pair = 5 * MAX_H * sizeof(float);
-    const size_t qual = (size_t)m.E * (1 + PAIR_MPB) * sizeof(float);
-    return pair > qual ? pair : qual;
+    const size_t cols = 3 * PAIR_G + (size_t)m.H1 * PAIR_COLS + (size_t)PAIR_G * (m.H1 | 1);
+    const size_t fin = 3 * PAIR_G + (size_t)m.H2 * PAIR_G + (size_t)m.NH * m.H2;
+    const size_t qual = (size_t)m.E * (1 + PAIR_MPB);
+    size_t f = cols > fin ? cols : fin;
+    f = f > qual ? f : qual;
+    return f * sizeof(float);
 }
 
-cudaError_t launch_route_pairs(const Model &m, const Queries &q, float *pairC,
-                               float *qualS, int32_t *count, cudaStream_t s) {
+cudaError_t launch_route_pairs(const Model &m, const Queries &q, float *pairC, float *qualS,
+                               float *h2, int32_t *count, cudaStream_t s) {
     if (q.Q <= 0) return cudaSuccess;
+    if ((long)q.Q * m.D > PAIRS_MAX_PAIRS) return cudaErrorInvalidValue;
     PairArgs a;
     a.pairC = pairC;
     a.qualS = qualS;
+    a.h2 = h2;
     a.count = count;
+    a.gcount = count + PAIRS_MAX_PAIRS;
     a.qblocks = (m.M + PAIR_MPB - 1) / PAIR_MPB;
-    const int blocks = q.Q * (m.D + a.qblocks);
+    a.ncb = (m.H2 + PAIR_COLS - 1) / PAIR_COLS;
+    const int blocks = pair_groups(q.Q * m.D) * a.ncb + q.Q * a.qblocks;
     k_route_pairs<<<blocks, SIMT_THREADS, route_pairs_smem(m), s>>>(m, q, a);
     return cudaGetLastError();
 }

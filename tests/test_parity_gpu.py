@@ -245,6 +245,33 @@ def test_small_batch_kernels_both_exact(monkeypatch, pairs_max, c, Q):
     assert np.array_equal(qual, qw.astype(np.float32))
 
 
+# the small-batch kernel groups 32 consecutive (query, deployment) pairs and
+# splits their layer 2 by 32-column blocks: groups holding many queries
+# (D = 1), queries straddling two groups (D = 15), every query spanning two
+# groups (D = 33), a ragged last column block (H2 = 200, 96 + 4 padding), and
+# a bf16 context
+@pytest.mark.parametrize("shape,Q", [
+    (dict(M=1, G=1, F=12, H1=8, H2=8, E=8), 70),
+    (dict(M=5, G=3, F=24, H1=96, H2=200, E=40), 37),
+    (dict(M=11, G=3, F=24, H1=64, H2=98, E=24), 20),
+    ("cfg4", 5),
+])
+def test_pairs_kernel_group_shapes_exact(monkeypatch, shape, Q):
+    monkeypatch.setenv("HWR_PAIRS_MAX_PAIRS", "2048")
+    if shape == "cfg4":
+        p = W.make_config(4, Q=Q)
+    else:
+        p = W.make_problem(Q=Q, dtype="f32", lam=0.3, slo=3.0, seed=43, bias_std=0.2, **shape)
+    r = H.Router(p)
+    got = r.route()
+    C, qual = r.score()
+    r.close()
+    orc = O.Problem(p)
+    assert_exact(got, orc.route(mode=O.F32, nthreads=8), str(shape))
+    Cw, _ = orc.score_all(mode=O.F32, nthreads=8)
+    assert np.array_equal(C, Cw.astype(np.float32))
+
+
 # ---------------------------------------------------------------------------
 # sequential mode on more shapes: D > 32 (two deployments per lane of the
 # chain's warp), odd D, D = 1, a bf16 context, several chunks each
