@@ -37,15 +37,17 @@ struct AllocHook {
 // tensor-core kernels; the rest the fused SIMT kernel.  pairs_max is
 // SMALL_MAX_PAIRS where the tensor-core path exists; otherwise FP32_MAX_PAIRS
 // for hidden layers wider than 64 x 64 and 0 for narrower ones.
-// (Device pointers, isolated calls.  bf16: the tensor path costs 31-33 us at
-// D = 32 and 38-40 us at D = 64 for 1 to 64 queries; the small-batch kernel
-// is ahead up to 256 pairs and behind from 512 on.  fp32: the fused kernel
+// (Device pointers, isolated calls.  bf16, H = 256: the tensor path costs
+// 32-33.5 us at D = 32 for 16-64 queries and 36-37 us at D = 64 for 8-32; the
+// small-batch kernel 29.7 / 30.5 / 34.3 / 44 us at D = 32 for 1 / 16 / 32 /
+// 64 queries and 29.5 / 31.1 / 34.8 / 44.6 us at D = 64 for 1 / 8 / 16 / 32:
+// ahead up to about 768 pairs.  fp32: the fused kernel
 // costs ~21 us at H = 32 and ~33 us at H = 128 from 1 to 512 queries; the
 // small-batch kernel costs ~24 us at H = 32 whatever the size, and 25.5-29 us
 // at H = 128, D = 12 from 1 to 170 queries (2,040 pairs).)
 constexpr int TC_MIN_PAIRS = 257;
 constexpr int PIPE_CHUNK_MIN = 8192;   // smallest chunk of a pipelined host batch
-constexpr int SMALL_MAX_PAIRS = 256;
+constexpr int SMALL_MAX_PAIRS = 768;
 constexpr int FP32_MAX_PAIRS = PAIRS_MAX_PAIRS;
 
 }  // namespace
