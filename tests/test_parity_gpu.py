@@ -248,12 +248,14 @@ def test_small_batch_kernels_both_exact(monkeypatch, pairs_max, c, Q):
 # the small-batch kernel groups 32 consecutive (query, deployment) pairs and
 # splits their layer 2 by 32-column blocks: groups holding many queries
 # (D = 1), queries straddling two groups (D = 15), every query spanning two
-# groups (D = 33), a ragged last column block (H2 = 200, 96 + 4 padding), and
-# a bf16 context
+# groups (D = 33), ragged last column blocks (H2 = 200: 8 columns; H2 = 98: 2
+# columns and 2 of padding), the largest batch the kernel takes (64 groups)
+# and a bf16 context
 @pytest.mark.parametrize("shape,Q", [
     (dict(M=1, G=1, F=12, H1=8, H2=8, E=8), 70),
     (dict(M=5, G=3, F=24, H1=96, H2=200, E=40), 37),
     (dict(M=11, G=3, F=24, H1=64, H2=98, E=24), 20),
+    (dict(M=16, G=4, F=48, H1=40, H2=72, E=16), 32),      # D = 64: 2,048 pairs, the limit
     ("cfg4", 5),
 ])
 def test_pairs_kernel_group_shapes_exact(monkeypatch, shape, Q):
