@@ -807,6 +807,11 @@ static hwr_status route_impl(hwr_ctx *c, int32_t Q, const float *in_len, const f
     const int nchunk = (!dev && !packed && !seq && Q >= 2 * PIPE_CHUNK_MIN)
                            ? (Q / PIPE_CHUNK_MIN < 8 ? Q / PIPE_CHUNK_MIN : 8) : 1;
     const bool pipelined = nchunk > 1;
+    // a small synchronous call for the small-batch kernel: that kernel reads
+    // its inputs with plain loads only, so it reads them from the mapped
+    // staging itself (no host-to-device copy)
+    const bool zero_copy = packed && !seq && !tensor && !ml && !so && c->pin_d &&
+                           (long)Q * c->D <= c->pairs_max;
 
     if (dev) {
         q.in_len = in_len; q.out_len = out_len; q.emb = q_emb;
@@ -828,8 +833,9 @@ static hwr_status route_impl(hwr_ctx *c, int32_t Q, const float *in_len, const f
             memcpy(c->pin_h + off_in, in_len, len_b);
             memcpy(c->pin_h + off_out, out_len, len_b);
             if (budgets) memcpy(c->pin_h + off_slo, spec->budget, len_b);
-            CK(c, cudaMemcpyAsync(c->io_d, c->pin_h, in_total, cudaMemcpyHostToDevice, c->stream),
-               "copy inputs");
+            if (!zero_copy)
+                CK(c, cudaMemcpyAsync(c->io_d, c->pin_h, in_total, cudaMemcpyHostToDevice,
+                                      c->stream), "copy inputs");
         } else if (!pipelined) {
             CK(c, cudaMemcpyAsync(c->io_d, q_emb, emb_b, cudaMemcpyHostToDevice, c->stream), "copy emb");
             CK(c, cudaMemcpyAsync(c->io_d + off_in, in_len, len_b, cudaMemcpyHostToDevice, c->stream),
@@ -840,10 +846,11 @@ static hwr_status route_impl(hwr_ctx *c, int32_t Q, const float *in_len, const f
                 CK(c, cudaMemcpyAsync(c->io_d + off_slo, spec->budget, len_b, cudaMemcpyHostToDevice,
                                       c->stream), "copy budgets");
         }
-        q.emb = c->io_d;
-        if (budgets) q.slo_q = (const float *)(c->io_d + off_slo);
-        q.in_len = (const float *)(c->io_d + off_in);
-        q.out_len = (const float *)(c->io_d + off_out);
+        const char *ib = zero_copy ? c->pin_d : c->io_d;
+        q.emb = ib;
+        if (budgets) q.slo_q = (const float *)(ib + off_slo);
+        q.in_len = (const float *)(ib + off_in);
+        q.out_len = (const float *)(ib + off_out);
         // small synchronous calls: the kernels write the outputs straight into
         // the mapped staging (plain stores), so no device-to-host copy follows
         char *ob = packed && !so ? c->pin_d + align_up(in_total, 256) : c->out_d;
