@@ -807,11 +807,11 @@ static hwr_status route_impl(hwr_ctx *c, int32_t Q, const float *in_len, const f
     const int nchunk = (!dev && !packed && !seq && Q >= 2 * PIPE_CHUNK_MIN)
                            ? (Q / PIPE_CHUNK_MIN < 8 ? Q / PIPE_CHUNK_MIN : 8) : 1;
     const bool pipelined = nchunk > 1;
-    // a small synchronous call for the small-batch kernel: that kernel reads
-    // its inputs with plain loads only, so it reads them from the mapped
-    // staging itself (no host-to-device copy)
-    const bool zero_copy = packed && !seq && !tensor && !ml && !so && c->pin_d &&
-                           (long)Q * c->D <= c->pairs_max;
+    // a small synchronous call for the small-batch kernel or the SIMT
+    // sequential kernels: they read the inputs from the mapped staging itself
+    // with plain loads (no host-to-device copy)
+    const bool zero_copy = packed && !tensor && !ml && !so && c->pin_d &&
+                           (seq ? !(flags & HWR_PATH_TENSOR) : (long)Q * c->D <= c->pairs_max);
 
     if (dev) {
         q.in_len = in_len; q.out_len = out_len; q.emb = q_emb;
@@ -847,6 +847,7 @@ static hwr_status route_impl(hwr_ctx *c, int32_t Q, const float *in_len, const f
                                       c->stream), "copy budgets");
         }
         const char *ib = zero_copy ? c->pin_d : c->io_d;
+        q.inputs_host = zero_copy;
         q.emb = ib;
         if (budgets) q.slo_q = (const float *)(ib + off_slo);
         q.in_len = (const float *)(ib + off_in);

@@ -65,6 +65,9 @@ struct Queries {
     // when set, the tensor-core predictor kernel only stores pair_C (no
     // decision outputs, no partial results)
     int no_select = 0;
+    // the query inputs sit in host memory mapped into the device's address
+    // space: kernels read them with plain loads only (no cp.async)
+    int inputs_host = 0;
     // sequential table on the tensor cores: when > 0, deployment v of the
     // predictor is (deployment v / (seq_n + 1), count v % (seq_n + 1)) and
     // pair_C is the triangular sequential table of seq_n queries (tab_row)

@@ -96,7 +96,7 @@ __device__ void quality_group(const Model &m, const Queries &q, int q0, int nq, 
                               int stage_floats, int t, float (&res)[CH]) {
     const int tid = t, M = m.M, E = m.E;
     const int es = q.emb_bf16 ? 2 : 4;
-    const bool async = ((uintptr_t)q.emb & 15) == 0;
+    const bool async = !q.inputs_host && ((uintptr_t)q.emb & 15) == 0;
     // row stride ld (elements): 16-byte rows whose 4-byte word stride is 4
     // mod 32, so the chains of one warp (up to 8 rows) read distinct banks
     auto stride = [&](int ek) {
