@@ -194,6 +194,16 @@ def _c(a, dtype):
     return np.ascontiguousarray(a, dtype=dtype)
 
 
+def _addr(a):
+    """Address of a contiguous array's data.  Through the buffer protocol for
+    writable non-empty arrays (about a third of the cost of ndarray.ctypes,
+    which a small call pays several times), else through ndarray.ctypes."""
+    try:
+        return ct.addressof(ct.c_char.from_buffer(a))
+    except (TypeError, ValueError):
+        return a.ctypes.data
+
+
 class Router:
     """One routing context built from a problem dict (see workload.gen).
 
@@ -259,7 +269,7 @@ class Router:
 
     def get_snapshot(self) -> np.ndarray:
         out = np.empty(self.D, np.int32)
-        self._check(self.lib.hwr_get_snapshot(self.ctx, out.ctypes.data))
+        self._check(self.lib.hwr_get_snapshot(self.ctx, _addr(out)))
         return out
 
     def route(self, in_len=None, out_len=None, emb=None, *, slo=None, lam=None,
@@ -272,9 +282,9 @@ class Router:
         Q = il.size
         # the three outputs as views of one allocation (one pointer to take)
         out = np.empty(3 * Q, np.uint32)
-        o = out.ctypes.data
+        o = _addr(out)
         self._check(self.lib.hwr_route_batch(
-            self.ctx, Q, il.ctypes.data, ol.ctypes.data, em.ctypes.data,
+            self.ctx, Q, _addr(il), _addr(ol), _addr(em),
             float(p["slo"] if slo is None else slo),
             float(p["lam"] if lam is None else lam), int(flags) & ~HWR_DEVICE_PTRS,
             o, o + 4 * Q, o + 8 * Q))
@@ -290,9 +300,9 @@ class Router:
         cost = np.empty((Q, p["D"]), np.float32)
         qual = np.empty((Q, p["M"]), np.float32) if quality else None
         self._check(self.lib.hwr_score_batch(
-            self.ctx, Q, il.ctypes.data, ol.ctypes.data, em.ctypes.data,
-            int(flags) & ~HWR_DEVICE_PTRS, cost.ctypes.data,
-            qual.ctypes.data if quality else None))
+            self.ctx, Q, _addr(il), _addr(ol), _addr(em),
+            int(flags) & ~HWR_DEVICE_PTRS, _addr(cost),
+            _addr(qual) if quality else None))
         return cost, qual
 
     def score_device(self, in_len, out_len, emb, cost, quality=None, *, flags=0):
@@ -315,10 +325,10 @@ class Router:
         lat = np.empty((K, Q), np.float32)
         util = np.empty((K, Q), np.float32)
         self._check(self.lib.hwr_route_batch_multi(
-            self.ctx, Q, il.ctypes.data, ol.ctypes.data, em.ctypes.data,
-            float(p["slo"] if slo is None else slo), lam.ctypes.data, K,
-            int(flags) & ~HWR_DEVICE_PTRS, chosen.ctypes.data, lat.ctypes.data,
-            util.ctypes.data))
+            self.ctx, Q, _addr(il), _addr(ol), _addr(em),
+            float(p["slo"] if slo is None else slo), _addr(lam), K,
+            int(flags) & ~HWR_DEVICE_PTRS, _addr(chosen), _addr(lat),
+            _addr(util)))
         return chosen, lat, util
 
     def route_device_multi(self, lambdas, in_len, out_len, emb, chosen, lat, util, *, slo,
@@ -327,7 +337,7 @@ class Router:
         lam = _c(lambdas, np.float32)
         self._check(self.lib.hwr_route_batch_multi(
             self.ctx, int(in_len.numel()), in_len.data_ptr(), out_len.data_ptr(),
-            emb.data_ptr(), float(slo), lam.ctypes.data, int(lam.size),
+            emb.data_ptr(), float(slo), _addr(lam), int(lam.size),
             int(flags) | HWR_DEVICE_PTRS, chosen.data_ptr(), lat.data_ptr(), util.data_ptr()))
 
     def route_slo(self, in_len=None, out_len=None, emb=None, *, budgets=None,
@@ -341,9 +351,9 @@ class Router:
         Q = il.size
         spec, keep = self._spec(budgets, model, Q)
         out = np.empty(3 * Q, np.uint32)
-        o = out.ctypes.data
+        o = _addr(out)
         self._check(self.lib.hwr_route_batch_slo(
-            self.ctx, Q, il.ctypes.data, ol.ctypes.data, em.ctypes.data, ct.byref(spec),
+            self.ctx, Q, _addr(il), _addr(ol), _addr(em), ct.byref(spec),
             float(p["lam"] if lam is None else lam), int(flags) & ~HWR_DEVICE_PTRS,
             o, o + 4 * Q, o + 8 * Q))
         return out[:Q].view(np.int32), out[Q:2 * Q].view(np.float32), out[2 * Q:].view(np.float32)

@@ -118,3 +118,15 @@ def test_calls_on_null_context(lib):
 def test_binding_fails_loudly_without_library(tmp_path):
     with pytest.raises(RuntimeError, match="not built"):
         _hwr.load(str(tmp_path / "missing.so"))
+
+
+def test_binding_address_helper_matches_ndarray_ctypes():
+    # the binding takes data addresses through the buffer protocol where it
+    # can; it must give the same address as ndarray.ctypes in every case
+    from paper_2608_14575_gb300._hwr import _addr
+    a = np.arange(12, dtype=np.float32).reshape(3, 4)
+    cases = [a, a[1:], a[2], np.zeros((2, 8), np.uint16)[1],
+             np.frombuffer(b"abcdabcd", dtype=np.float32),      # read-only
+             np.empty(0, np.float32)]                          # empty
+    for x in cases:
+        assert _addr(x) == x.ctypes.data
