@@ -256,24 +256,33 @@ __device__ __forceinline__ void w2_chunk_async(const Model &m, int k0, int kc, f
     asm volatile("cp.async.commit_group;" ::: "memory");
 }
 
-template <int CPT, class Rows>
-__device__ void pair_mlp(const Model &m, int R, const Rows &rows, const float *us,
-                         const float *vs, float *tile, float *w3s, float *w1q, float *sp) {
-    constexpr int VW = CPT < 4 ? CPT : 4, W = 32 * CPT;
-    static_assert(SIMT_THREADS == 4 * TILE_ROWS, "layer-1 map: 4 threads per row");
-    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int H1 = m.H1, H2 = m.H2, F = m.F;
-    float *h1T = tile;
-    float *w2b = tile + SIMT_KC * TILE_ROWS;
-
-    // W3 for the head chains and the two query columns of W1 (visible after
-    // the first barrier of the K loop)
+// The tile's weights that no row depends on: W3 for the head chains, the two
+// query columns of W1 (both visible after the first barrier of the K loop)
+// and the first W2 chunk (one cp.async group).  pair_mlp runs this itself
+// unless the caller did, e.g. before waiting for a preceding kernel.
+template <int CPT>
+__device__ void pair_mlp_stage(const Model &m, float *tile, float *w3s, float *w1q) {
+    const int tid = threadIdx.x, H1 = m.H1, H2 = m.H2, F = m.F;
     for (int i = tid; i < m.NH * H2; i += SIMT_THREADS) w3s[i] = m.W3[i];
     for (int k = tid; k < H1; k += SIMT_THREADS) {
         w1q[k] = m.W1[(size_t)k * F + F - 2];
         w1q[H1 + k] = m.W1[(size_t)k * F + F - 1];
     }
-    w2_chunk_async(m, 0, min(SIMT_KC, H1), w2b, W);
+    w2_chunk_async(m, 0, min(SIMT_KC, H1), tile + SIMT_KC * TILE_ROWS, 32 * CPT);
+}
+
+template <int CPT, class Rows>
+__device__ void pair_mlp(const Model &m, int R, const Rows &rows, const float *us,
+                         const float *vs, float *tile, float *w3s, float *w1q, float *sp,
+                         bool staged = false) {
+    constexpr int VW = CPT < 4 ? CPT : 4, W = 32 * CPT;
+    static_assert(SIMT_THREADS == 4 * TILE_ROWS, "layer-1 map: 4 threads per row");
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int H1 = m.H1, H2 = m.H2;
+    float *h1T = tile;
+    float *w2b = tile + SIMT_KC * TILE_ROWS;
+
+    if (!staged) pair_mlp_stage<CPT>(m, tile, w3s, w1q);
     // layer-1 map: thread t fills row t % 64 at k offsets t / 64 + 4 j of a chunk
     const int r1 = tid % TILE_ROWS, kq = tid / TILE_ROWS;
     const bool rv = r1 < R;
@@ -678,6 +687,8 @@ k_seq_table(Model m, Queries q, int Qs, int nb_qual, int rows_per_block, float *
         gi[r] = d * (Qs + 1) + lo;
         qi[r] = lo + off - d * len;
     }
+    // the weights need nothing from the preparation kernel
+    pair_mlp_stage<CPT>(m, sm + L.tile, sm + L.w3, sm + L.w1q);
     umma::grid_dependency_wait();    // the preparation kernel's features and prefixes
     for (int i = tid; i < Qs; i += SIMT_THREADS) {
         us[i] = A.us[i];
@@ -686,7 +697,7 @@ k_seq_table(Model m, Queries q, int Qs, int nb_qual, int rows_per_block, float *
     __syncthreads();
 
     FlatRows rows{A.pre, gi, qi, m.H1};
-    pair_mlp<CPT>(m, R, rows, us, vs, sm + L.tile, sm + L.w3, sm + L.w1q, sp);
+    pair_mlp<CPT>(m, R, rows, us, vs, sm + L.tile, sm + L.w3, sm + L.w1q, sp, true);
 
     for (int r = tid; r < R; r += SIMT_THREADS) {
         const float *h = sp + m.NH * r;
