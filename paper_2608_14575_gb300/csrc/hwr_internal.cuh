@@ -47,6 +47,11 @@ struct Model {
 
 struct Queries {
     int Q;
+    // the query inputs sit in host memory mapped into the device's address
+    // space: kernels read them with plain loads only (no cp.async).  Kept in
+    // the padding after Q: the struct stays 128 bytes (a larger parameter
+    // block measured 2.6 % slower in the tensor-core predictor kernel)
+    int inputs_host = 0;
     const float *in_len, *out_len;
     const void *emb;            // [Q][E], fp32 or bf16 bits
     int emb_bf16;
@@ -65,14 +70,12 @@ struct Queries {
     // when set, the tensor-core predictor kernel only stores pair_C (no
     // decision outputs, no partial results)
     int no_select = 0;
-    // the query inputs sit in host memory mapped into the device's address
-    // space: kernels read them with plain loads only (no cp.async)
-    int inputs_host = 0;
     // sequential table on the tensor cores: when > 0, deployment v of the
     // predictor is (deployment v / (seq_n + 1), count v % (seq_n + 1)) and
     // pair_C is the triangular sequential table of seq_n queries (tab_row)
     int seq_n = 0;
 };
+static_assert(sizeof(Queries) == 128, "Queries: a larger parameter block slows k_mlp_tc");
 
 // The sequential score table of a chunk of Qs queries over D deployments:
 // entry (picks so far c, deployment d, query i >= c) sits at
