@@ -47,8 +47,11 @@ def test_budget_array_simt_exact(c, Q):
     r.close()
 
 
-def test_budget_model_simt_exact():
-    p = W.make_config(0, Q=256)
+# (0, 256): the fused kernel; (2, 64): the small-batch kernel, which reads the
+# lengths from the mapped host staging
+@pytest.mark.parametrize("c,Q", [(0, 256), (2, 64)])
+def test_budget_model_simt_exact(c, Q):
+    p = W.make_config(c, Q=Q)
     want_b = O.slo_budget(*MODEL, p["in_len"], p["out_len"], mode=O.F32).astype(np.float32)
     r = H.Router(p)
     got = r.route_slo(model=MODEL)
@@ -56,6 +59,17 @@ def test_budget_model_simt_exact():
     # the same budgets given as an array route identically
     got2 = r.route_slo(budgets=want_b)
     assert all(np.array_equal(a, b) for a, b in zip(got, got2))
+    r.close()
+
+
+def test_budget_model_sequential_exact():
+    p = W.make_config(2, Q=70)
+    want_b = O.slo_budget(*MODEL, p["in_len"], p["out_len"], mode=O.F32).astype(np.float32)
+    r = H.Router(p)
+    got = r.route_slo(model=MODEL, flags=H.HWR_SEQUENTIAL)
+    want = O.Problem(p).route_slo(want_b, mode=O.F32, sequential=True)
+    _exact(got, want)
+    assert np.array_equal(r.get_snapshot(), want[3])
     r.close()
 
 
