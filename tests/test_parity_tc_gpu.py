@@ -257,7 +257,6 @@ def test_sequential_tensor_table_valid(c, Q):
     r = H.Router(p)
     got = r.route(flags=H.HWR_SEQUENTIAL | H.HWR_PATH_TENSOR)
     final = r.get_snapshot()
-    canon = None
     r.update_snapshot(p["snap"])
     canon = r.route(flags=H.HWR_SEQUENTIAL)           # canonical fp32 order
     r.close()
