@@ -11,6 +11,7 @@
 #include <stdlib.h>
 #include <string.h>
 
+#include <chrono>
 #include <string>
 #include <vector>
 
@@ -728,6 +729,23 @@ static hwr_status run_kernels(hwr_ctx *c, const Queries &q, uint32_t flags, bool
 
 static size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
+// Outputs of a small synchronous call on the small-batch kernel: the kernel
+// stores each query's chosen index last, after a system-scope fence, into
+// mapped host memory that held a value it never writes; wait for all Q of
+// them (acquire loads).  False after a second: the caller then synchronises
+// the stream, which reports a failed launch.
+constexpr int32_t OUT_PENDING = INT32_MIN;
+static bool wait_chosen(const int32_t *ch, int Q) {
+    const auto t0 = std::chrono::steady_clock::now();
+    for (int i = 0; i < Q; ++i) {
+        unsigned n = 0;
+        while (__atomic_load_n(ch + i, __ATOMIC_ACQUIRE) == OUT_PENDING)
+            if ((++n & 1023u) == 0 && std::chrono::steady_clock::now() - t0 > std::chrono::seconds(1))
+                return false;
+    }
+    return true;
+}
+
 // Shared body of hwr_route_batch and hwr_route_batch_slo.  `spec` (may be
 // NULL) replaces the scalar SLO by per-query budgets or the Eq. 4-5 model.
 // Score outputs of hwr_score_batch: cost [Q][D] and quality [Q][M] (either may be NULL).
@@ -812,6 +830,9 @@ static hwr_status route_impl(hwr_ctx *c, int32_t Q, const float *in_len, const f
     // with plain loads (no host-to-device copy)
     const bool zero_copy = packed && !tensor && !ml && !so && c->pin_d &&
                            (seq ? !(flags & HWR_PATH_TENSOR) : (long)Q * c->D <= c->pairs_max);
+    // ... and on the small-batch kernel the host waits for the outputs
+    // themselves instead of synchronising the stream
+    const bool poll = zero_copy && !seq;
 
     if (dev) {
         q.in_len = in_len; q.out_len = out_len; q.emb = q_emb;
@@ -833,6 +854,10 @@ static hwr_status route_impl(hwr_ctx *c, int32_t Q, const float *in_len, const f
             memcpy(c->pin_h + off_in, in_len, len_b);
             memcpy(c->pin_h + off_out, out_len, len_b);
             if (budgets) memcpy(c->pin_h + off_slo, spec->budget, len_b);
+            if (poll) {
+                int32_t *ch = (int32_t *)(c->pin_h + align_up(in_total, 256));
+                for (int i = 0; i < Q; ++i) ch[i] = OUT_PENDING;
+            }
             if (!zero_copy)
                 CK(c, cudaMemcpyAsync(c->io_d, c->pin_h, in_total, cudaMemcpyHostToDevice,
                                       c->stream), "copy inputs");
@@ -958,7 +983,8 @@ static hwr_status route_impl(hwr_ctx *c, int32_t Q, const float *in_len, const f
         if (packed) {
             const char *ob = c->pin_h + align_up(in_total, 256);
             CK(c, cudaEventRecord(c->pin_ev, c->stream), "record");
-            CK(c, cudaStreamSynchronize(c->stream), "synchronize");
+            if (!(poll && wait_chosen((const int32_t *)ob, Q)))
+                CK(c, cudaStreamSynchronize(c->stream), "synchronize");
             synced = true;
             memcpy(chosen, ob, outs_b);
             memcpy(pred_latency, ob + o_lat, outs_b);

@@ -933,10 +933,13 @@ __device__ void pair_select(const Model &m, const Queries &q, const PairArgs &a,
     best = warp_best(best);
     if (lane == 0) {
         const bool ok = best.cls > 0;
-        q.chosen[qq] = ok ? best.d : -1;
         q.lat[qq] = ok ? best.C : __int_as_float(0x7fc00000);
         q.util[qq] = ok ? best.U : __int_as_float(0x7fc00000);
         a.count[qq] = 0;
+        // outputs in mapped host memory: the host polls chosen, so latency
+        // and utility must be visible to it first
+        if (q.inputs_host) __threadfence_system();
+        q.chosen[qq] = ok ? best.d : -1;
     }
 }
 
