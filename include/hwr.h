@@ -167,7 +167,10 @@ hwr_status hwr_get_snapshot(hwr_ctx *ctx, int32_t *running_out);
  *   utility[Q]             utility U of the chosen deployment.
  * Without HWR_DEVICE_PTRS all six arrays are host memory; the call copies the
  * inputs host -> device and the outputs back, and (without HWR_ASYNC)
- * returns after the results are in place.  Pinned host memory gives the full
+ * returns after the results are in place (small batches on the small-batch
+ * kernel return as soon as every output is written, possibly before the
+ * kernel's last blocks retire; a failure after that point is reported by the
+ * next call on the context or by hwr_synchronize).  Pinned host memory gives the full
  * link bandwidth.  With HWR_DEVICE_PTRS they are device pointers read and
  * written in stream order.  With HWR_ASYNC the call returns after enqueueing;
  * host arrays must then stay valid until hwr_synchronize().
