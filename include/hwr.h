@@ -116,7 +116,9 @@ typedef struct {
 } hwr_snapshot;
 
 /*
- * Create a routing context.
+ * Create a routing context: the router's static problem of Sec. 3.1 -- the
+ * deployment set (M_i, g_i) -- with the cost predictor f_cost of Sec. 3.2 (2)
+ * (Eq. 1) and the model embeddings of the quality predictor, Sec. 3.2 (3).
  *   table, pred   host structs as above (copied).
  *   model_emb     host [E][n_models] model embedding matrix (copied), in
  *                 emb_dtype.  Quality of model m for query q is
@@ -129,8 +131,10 @@ typedef struct {
  * Limits (HWR_ERR_UNSUPPORTED beyond them): 1 <= D <= 64; M <= 32 (bf16) or
  * M <= 64 (fp32); H1, H2 in [1, 256]; F <= 256.  The bf16 tensor-core path
  * further needs H1 % 64 == 0 and H2 % 16 == 0 (else the SIMT kernels run).
- * The context holds no snapshot until hwr_update_snapshot is called.
- * Errors: INVALID_ARG, DTYPE, UNSUPPORTED, OOM, CUDA.
+ * The context holds no snapshot until hwr_update_snapshot is called.  The
+ * CUDA device current at this call is the context's device: every later call
+ * on the context must be made with it current.
+ * Errors: INVALID_ARG, DTYPE, UNSUPPORTED, OOM, CUDA (also: no CUDA device).
  */
 hwr_status hwr_create(const hwr_deployment_table *table,
                       const hwr_predictor *pred, const void *model_emb,
@@ -142,13 +146,19 @@ hwr_status hwr_create(const hwr_deployment_table *table,
  * Copies D entries of every array host -> device and recomputes the
  * deployment part of the predictor's first layer on the device.  Ordered on
  * the context stream; returns once the host arrays may be reused.
- * Errors: INVALID_ARG (NULL), STATE, CUDA.
+ * Every value must lie in the domain of its feature's transform: running and
+ * waiting >= 0; every float finite; > 0 where the slot's feat_xform is log,
+ * > -1 where it is log1p.  A snapshot with any other value is rejected
+ * (INVALID_ARG, the context keeps its previous snapshot): such a value would
+ * turn the deployment's features, and so its cost, into NaN.
+ * Errors: INVALID_ARG (NULL array or a value outside its domain), STATE, CUDA.
  */
 hwr_status hwr_update_snapshot(hwr_ctx *ctx, const hwr_snapshot *snap);
 
 /*
- * Copy the context's current running counts (D int32, host memory) -- these
- * include the increments made by HWR_SEQUENTIAL routing.  Synchronises the
+ * Copy the context's current running counts (D int32, host memory): the
+ * running-queue signal of the cached monitor view (Sec. 3.2 (1), Table 2),
+ * including the increments made by HWR_SEQUENTIAL routing.  Synchronises the
  * context stream.  Errors: INVALID_ARG, STATE, CUDA.
  */
 hwr_status hwr_get_snapshot(hwr_ctx *ctx, int32_t *running_out);
@@ -170,7 +180,10 @@ hwr_status hwr_get_snapshot(hwr_ctx *ctx, int32_t *running_out);
  * returns after the results are in place (small batches on the small-batch
  * kernel return as soon as every output is written, possibly before the
  * kernel's last blocks retire; a failure after that point is reported by the
- * next call on the context or by hwr_synchronize).  Pinned host memory gives the full
+ * next call on the context or by hwr_synchronize.  When earlier work is still
+ * queued on the stream -- after an HWR_ASYNC call, or the caller's own work on
+ * a stream it passed to hwr_create -- the call synchronises the stream
+ * instead of waiting on the outputs).  Pinned host memory gives the full
  * link bandwidth.  With HWR_DEVICE_PTRS they are device pointers read and
  * written in stream order.  With HWR_ASYNC the call returns after enqueueing;
  * host arrays must then stay valid until hwr_synchronize().

@@ -64,6 +64,10 @@ struct hwr_ctx {
     bool have_snapshot = false;
     int test_stall = 0;          // HWR_TEST_STALL: tensor-path producers never signal
     int tc_min_pairs = TC_MIN_PAIRS, pairs_max = -1;   // -1: by the context's paths
+    int device = -1;             // the CUDA device current at hwr_create
+    long poll_us = 1000000;      // small-batch output poll limit (HWR_TEST_POLL_US)
+    bool async_pending = false;  // an HWR_ASYNC call may still have work queued
+    std::vector<uint8_t> xform_h;   // feature transforms (host copy, snapshot checks)
     std::string err;
     AllocHook hook;
     std::vector<void *> allocs;  // device buffers (cudaMalloc)
@@ -470,6 +474,7 @@ static hwr_status build_ctx(hwr_ctx *c, const hwr_deployment_table *t, const hwr
         for (int k = 0; k < F; ++k) w1t[(size_t)k * H1 + j] = w1[(size_t)j * F + k];
     TRY(upload(c, c->W1T, w1t.data(), w1t.size() * 4, "upload W1 transposed"));
     CK(c, cudaMemset(c->pairN, 0, 2 * PAIRS_MAX_PAIRS * sizeof(int32_t)), "zero counters");
+    c->xform_h.assign(p->feat_xform, p->feat_xform + F);
     c->mu_in = p->feat_mean[F - 2]; c->sd_in = p->feat_std[F - 2]; c->xf_in = p->feat_xform[F - 2];
     c->mu_out = p->feat_mean[F - 1]; c->sd_out = p->feat_std[F - 1]; c->xf_out = p->feat_xform[F - 1];
 
@@ -562,7 +567,13 @@ extern "C" hwr_status hwr_create(const hwr_deployment_table *table, const hwr_pr
     c->F = pred->F; c->H1 = pred->H1; c->H2 = pred->H2; c->E = E; c->P = c->M + c->G;
     c->dtype = pred->dtype;
     c->NH = pred->n_heads == 3 ? 3 : 2;
+    if (cudaGetDevice(&c->device) != cudaSuccess) {
+        cudaGetLastError();
+        delete c;
+        return fail(nullptr, HWR_ERR_CUDA, "no current CUDA device");
+    }
     if (const char *h = getenv("HWR_TEST_FAIL_ALLOC")) c->hook.fail_at = atol(h);
+    if (const char *h = getenv("HWR_TEST_POLL_US")) c->poll_us = atol(h) < 0 ? 0 : atol(h);
     if (const char *h = getenv("HWR_TEST_STALL")) c->test_stall = atoi(h) != 0;
     if (const char *h = getenv("HWR_TC_MIN_PAIRS")) c->tc_min_pairs = atoi(h) > 1 ? atoi(h) : 1;
     if (const char *h = getenv("HWR_PAIRS_MAX_PAIRS"))
@@ -593,6 +604,23 @@ extern "C" hwr_status hwr_update_snapshot(hwr_ctx *c, const hwr_snapshot *s) {
     if (!s || !s->running || !s->waiting || !s->kv_util || !s->gpu_util || !s->ttft_avg ||
         !s->tpot_avg)
         return fail(c, HWR_ERR_INVALID_ARG, "NULL snapshot array");
+    // every signal must be a value its feature transform accepts: counts
+    // >= 0, finite values, > 0 under log, > -1 under log1p
+    const float *fs[4] = {s->kv_util, s->gpu_util, s->ttft_avg, s->tpot_avg};
+    static const char *names[6] = {"running", "waiting", "kv_util", "gpu_util", "ttft_avg",
+                                   "tpot_avg"};
+    for (int k = 0; k < 6; ++k) {
+        const uint8_t xf = c->xform_h[c->P + 1 + k];
+        for (int d = 0; d < c->D; ++d) {
+            const double v = k < 2 ? (double)(k == 0 ? s->running : s->waiting)[d] : (double)fs[k - 2][d];
+            const bool bad = !isfinite(v) || (k < 2 && v < 0) || (xf == 2 && !(v > 0)) ||
+                             (xf == 1 && !(v > -1));
+            if (bad)
+                return fail(c, HWR_ERR_INVALID_ARG,
+                            "snapshot %s[%d] = %g is outside the domain of its feature%s", names[k],
+                            d, v, xf == 2 ? " (log)" : xf == 1 ? " (log1p)" : "");
+        }
+    }
     const size_t n = (size_t)c->D * 4;
     // the previous snapshot copy must have left the staging buffer
     CK(c, cudaEventSynchronize(c->snap_ev), "wait for snapshot staging");
@@ -735,13 +763,13 @@ static size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 // them (acquire loads).  False after a second: the caller then synchronises
 // the stream, which reports a failed launch.
 constexpr int32_t OUT_PENDING = INT32_MIN;
-static bool wait_chosen(const int32_t *ch, int Q) {
+static bool wait_chosen(const int32_t *ch, int Q, long limit_us) {
     const auto t0 = std::chrono::steady_clock::now();
+    const auto limit = std::chrono::microseconds(limit_us);
     for (int i = 0; i < Q; ++i) {
         unsigned n = 0;
         while (__atomic_load_n(ch + i, __ATOMIC_ACQUIRE) == OUT_PENDING)
-            if ((++n & 1023u) == 0 && std::chrono::steady_clock::now() - t0 > std::chrono::seconds(1))
-                return false;
+            if ((++n & 1023u) == 0 && std::chrono::steady_clock::now() - t0 > limit) return false;
     }
     return true;
 }
@@ -832,7 +860,19 @@ static hwr_status route_impl(hwr_ctx *c, int32_t Q, const float *in_len, const f
                            (seq ? !(flags & HWR_PATH_TENSOR) : (long)Q * c->D <= c->pairs_max);
     // ... and on the small-batch kernel the host waits for the outputs
     // themselves instead of synchronising the stream
-    const bool poll = zero_copy && !seq;
+    // ... unless work queued earlier on the stream (an HWR_ASYNC call, or the
+    // caller's own work on a stream it passed in) is still running: then
+    // the kernel starts late and the host synchronises instead of spinning
+    bool poll = zero_copy && !seq && c->poll_us > 0;
+    if (poll && (c->async_pending || !c->own_stream)) {
+        const cudaError_t e = cudaStreamQuery(c->stream);
+        if (e == cudaSuccess) {
+            c->async_pending = false;
+        } else {
+            if (e != cudaErrorNotReady) return cuda_fail(c, e, "query stream");
+            poll = false;
+        }
+    }
 
     if (dev) {
         q.in_len = in_len; q.out_len = out_len; q.emb = q_emb;
@@ -983,7 +1023,7 @@ static hwr_status route_impl(hwr_ctx *c, int32_t Q, const float *in_len, const f
         if (packed) {
             const char *ob = c->pin_h + align_up(in_total, 256);
             CK(c, cudaEventRecord(c->pin_ev, c->stream), "record");
-            if (!(poll && wait_chosen((const int32_t *)ob, Q)))
+            if (!(poll && wait_chosen((const int32_t *)ob, Q, c->poll_us)))
                 CK(c, cudaStreamSynchronize(c->stream), "synchronize");
             synced = true;
             memcpy(chosen, ob, outs_b);
@@ -999,8 +1039,12 @@ static hwr_status route_impl(hwr_ctx *c, int32_t Q, const float *in_len, const f
         }
     }
     c->stats.queries_routed += Q;
-    if ((flags & HWR_ASYNC) && !synced) return HWR_OK;
+    if ((flags & HWR_ASYNC) && !synced) {
+        c->async_pending = true;
+        return HWR_OK;
+    }
     if (!synced) CK(c, cudaStreamSynchronize(c->stream), "synchronize");
+    c->async_pending = false;
     CK(c, cudaGetLastError(), "kernel");
     if (tensor || (seq && (flags & HWR_PATH_TENSOR))) TRY(check_status_word(c));
     return HWR_OK;
@@ -1058,6 +1102,7 @@ extern "C" hwr_status hwr_synchronize(hwr_ctx *c) {
     if (!c) return fail(nullptr, HWR_ERR_INVALID_ARG, "ctx is NULL");
     if (c->broken) return HWR_ERR_STATE;
     CK(c, cudaStreamSynchronize(c->stream), "synchronize");
+    c->async_pending = false;
     return check_status_word(c);
 }
 
@@ -1100,6 +1145,8 @@ hwr_status hwr_internal_fail(hwr_ctx *c, hwr_status s, const char *msg) {
     return fail(c, s, "%s", msg);
 }
 
+int hwr_internal_device(const hwr_ctx *c) { return c->device; }
+
 hwr_status hwr_internal_route_tensor_scratch(hwr_ctx *c, int32_t Q, const float *in_len,
                                              const float *out_len, const void *q_emb, float slo,
                                              float lambda, uint32_t flags, int32_t *chosen,
@@ -1140,8 +1187,12 @@ hwr_status hwr_internal_route_tensor_scratch(hwr_ctx *c, int32_t Q, const float 
     c->stats.kernel_launches++;
     c->stats.launches[HWR_K_MLP_TC]++;
     c->stats.queries_routed += Q;
-    if (flags & HWR_ASYNC) return HWR_OK;
+    if (flags & HWR_ASYNC) {
+        c->async_pending = true;
+        return HWR_OK;
+    }
     CK(c, cudaStreamSynchronize(c->stream), "synchronize");
+    c->async_pending = false;
     CK(c, cudaGetLastError(), "kernel");
     return check_status_word(c);
 }

@@ -20,6 +20,7 @@
 #include "hwr_internal.cuh"
 
 hwr_status hwr_internal_fail(hwr_ctx *c, hwr_status s, const char *msg);
+int hwr_internal_device(const hwr_ctx *c);
 hwr_status hwr_internal_route_tensor_scratch(hwr_ctx *c, int32_t Q, const float *in_len,
                                              const float *out_len, const void *q_emb, float slo,
                                              float lambda, uint32_t flags, int32_t *chosen,
@@ -45,12 +46,10 @@ unsigned char *g_dev_ptr[MAX_DEVICES];
 // its device address comes from cudaGetSymbolAddress, per device.
 static __device__ __align__(256) unsigned char g_noalloc_scratch[SCRATCH_BYTES];
 
-// Device address of the scratch on the current device, resolved on the first
-// call made with that device current.
-static cudaError_t scratch_on_current_device(unsigned char **out) {
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e != cudaSuccess) return e;
+// Device address of the scratch on device `dev` (the current device),
+// resolved on the first call made with that device current.
+static cudaError_t scratch_on_device(int dev, unsigned char **out) {
+    cudaError_t e;
     if (dev < 0 || dev >= MAX_DEVICES) return cudaErrorInvalidDevice;
     std::lock_guard<std::mutex> lock(g_mu);
     if (!g_dev_ptr[dev]) {
@@ -80,8 +79,18 @@ extern "C" hwr_status hwr_route_batch_noalloc(hwr_ctx *ctx, int32_t Q, const flo
                  NOALLOC_MAX_Q);
         return hwr_internal_fail(ctx, HWR_ERR_UNSUPPORTED, msg);
     }
+    // the scratch of the context's own device: one device's array handed to
+    // kernels on another would be the wrong memory
+    int dev = -1;
+    if (cudaGetDevice(&dev) != cudaSuccess) {
+        cudaGetLastError();
+        return hwr_internal_fail(ctx, HWR_ERR_CUDA, "no current CUDA device");
+    }
+    if (dev != hwr_internal_device(ctx))
+        return hwr_internal_fail(ctx, HWR_ERR_INVALID_ARG,
+                                 "the current CUDA device is not the context's device");
     unsigned char *base = nullptr;
-    const cudaError_t e = scratch_on_current_device(&base);
+    const cudaError_t e = scratch_on_device(dev, &base);
     if (e != cudaSuccess) {
         cudaGetLastError();
         return hwr_internal_fail(ctx, HWR_ERR_CUDA, "cannot resolve the noalloc scratch address");

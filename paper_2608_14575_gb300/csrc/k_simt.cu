@@ -936,10 +936,16 @@ __device__ void pair_select(const Model &m, const Queries &q, const PairArgs &a,
         q.lat[qq] = ok ? best.C : __int_as_float(0x7fc00000);
         q.util[qq] = ok ? best.U : __int_as_float(0x7fc00000);
         a.count[qq] = 0;
-        // outputs in mapped host memory: the host polls chosen, so latency
-        // and utility must be visible to it first
-        if (q.inputs_host) __threadfence_system();
-        q.chosen[qq] = ok ? best.d : -1;
+        const int32_t v = ok ? best.d : -1;
+        if (q.inputs_host) {
+            // outputs in mapped host memory: the host polls chosen with
+            // acquire loads, so chosen is stored with release semantics at
+            // system scope, after latency and utility
+            asm volatile("st.release.sys.global.b32 [%0], %1;" ::"l"(q.chosen + qq), "r"(v)
+                         : "memory");
+        } else {
+            q.chosen[qq] = v;
+        }
     }
 }
 

@@ -335,20 +335,21 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
     return d;
 }
 
+// Four columns of the second hidden layer into the output heads.  With
+// nb = -b2, relu(acc + b2) = max(acc, nb) + b2 exactly, so
+// sum_n w[n] relu(acc[n] + b2[n]) = sum_n w[n] max(acc[n], nb[n]) + sum_n w[n] b2[n];
+// the constant second sum is folded into the head bias b3 on the host (in
+// double), which leaves one max per column and packed FMAs for the heads.
 template <int NH>
-__device__ __forceinline__ void head_pair(const uint32_t *v, int j, const float4 &bb,
+__device__ __forceinline__ void head_pair(const uint32_t *v, int j, const float4 &nb,
                                           const float4 &w0, const float4 &w1, const float4 &w2,
                                           float2 &t0a, float2 &t0b, float2 &t1a, float2 &t1b,
                                           float2 &t2a, float2 &t2b) {
-    // relu(acc + b2) for four columns, then both output heads as packed FMAs
-    float2 x01 = __fadd2_rn(make_float2(__uint_as_float(v[j]), __uint_as_float(v[j + 1])),
-                            make_float2(bb.x, bb.y));
-    float2 x23 = __fadd2_rn(make_float2(__uint_as_float(v[j + 2]), __uint_as_float(v[j + 3])),
-                            make_float2(bb.z, bb.w));
-    x01.x = fmaxf(x01.x, 0.f);
-    x01.y = fmaxf(x01.y, 0.f);
-    x23.x = fmaxf(x23.x, 0.f);
-    x23.y = fmaxf(x23.y, 0.f);
+    float2 x01, x23;
+    x01.x = fmaxf(__uint_as_float(v[j]), nb.x);
+    x01.y = fmaxf(__uint_as_float(v[j + 1]), nb.y);
+    x23.x = fmaxf(__uint_as_float(v[j + 2]), nb.z);
+    x23.y = fmaxf(__uint_as_float(v[j + 3]), nb.w);
     t0a = __ffma2_rn(x01, make_float2(w0.x, w0.y), t0a);
     t0b = __ffma2_rn(x23, make_float2(w0.z, w0.w), t0b);
     t1a = __ffma2_rn(x01, make_float2(w1.x, w1.y), t1a);
@@ -361,9 +362,10 @@ __device__ __forceinline__ void head_pair(const uint32_t *v, int j, const float4
 
 // Output-layer constants passed by value: they sit in the kernel-parameter
 // constant bank, so the fully unrolled epilogue reads them as instruction
-// operands instead of shared-memory loads.
+// operands instead of shared-memory loads.  nb2 = -b2; b3 holds the head
+// biases plus sum_n W3[o][n] b2[n] (see head_pair).
 struct HeadConsts {
-    float b2[MAX_H], w0[MAX_H], w1[MAX_H], w2[MAX_H], b3[3];
+    float nb2[MAX_H], w0[MAX_H], w1[MAX_H], w2[MAX_H], b3[3];
 };
 
 template <int H2T, int NH>
@@ -411,12 +413,12 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
         fence_mbar_init();
     }
     for (int i = tid; i < H2; i += MLP_THREADS) {
-        b2s[i] = m.b2[i];
+        b2s[i] = hc.nb2[i];
         w30s[i] = m.W3[i];
         w31s[i] = m.W3[H2 + i];
         w32s[i] = NH == 3 ? m.W3[2 * H2 + i] : 0.f;
     }
-    if (tid < NH) b3s[tid] = m.b3[tid];
+    if (tid < NH) b3s[tid] = hc.b3[tid];
     for (int i = tid; i < D; i += MLP_THREADS) dms[i] = m.dep_model[i];
     if (warp == 0) {
         tmem_alloc(tslot, tcols);
@@ -514,7 +516,7 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
 #pragma unroll
                         for (int j = 0; j < 32; j += 4) {
                             const int n = c * 32 + j;
-                            head_pair<NH>(cur, j, make_float4(hc.b2[n], hc.b2[n + 1], hc.b2[n + 2], hc.b2[n + 3]),
+                            head_pair<NH>(cur, j, make_float4(hc.nb2[n], hc.nb2[n + 1], hc.nb2[n + 2], hc.nb2[n + 3]),
                                           make_float4(hc.w0[n], hc.w0[n + 1], hc.w0[n + 2], hc.w0[n + 3]),
                                           make_float4(hc.w1[n], hc.w1[n + 1], hc.w1[n + 2], hc.w1[n + 3]),
                                           make_float4(hc.w2[n], hc.w2[n + 1], hc.w2[n + 2], hc.w2[n + 3]),
@@ -866,12 +868,16 @@ void tc_fill_head_consts(void *dst, const float *b2, const float *W3, const floa
     HeadConsts *h = (HeadConsts *)dst;
     memset(h, 0, sizeof *h);
     for (int i = 0; i < H2; ++i) {
-        h->b2[i] = b2[i];
+        h->nb2[i] = -b2[i];
         h->w0[i] = W3[i];
         h->w1[i] = W3[H2 + i];
         h->w2[i] = NH == 3 ? W3[2 * H2 + i] : 0.f;
     }
-    for (int o = 0; o < NH; ++o) h->b3[o] = b3[o];
+    for (int o = 0; o < NH; ++o) {
+        double s = b3[o];
+        for (int i = 0; i < H2; ++i) s += (double)W3[(size_t)o * H2 + i] * b2[i];
+        h->b3[o] = (float)s;
+    }
 }
 
 }  // namespace hwr
