@@ -91,17 +91,64 @@ def bytes_per_query(p):
 
 
 class ClockSampler:
-    """nvidia-smi clocks and throttle reasons, sampled during the timed region."""
+    """SM clock and clock-event (throttle) reasons, sampled during the timed
+    region.  Read-only NVML queries from a host thread every ~2 ms (the
+    driver's management library, through ctypes), so that timed regions of a
+    few milliseconds still get samples; nvidia-smi every 200 ms if NVML cannot
+    be loaded."""
     FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
               "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    # NVML clock-event reason bits
+    REASONS = {0x4: "sw_power_cap", 0x8: "hw_slowdown", 0x20: "sw_thermal_slowdown",
+               0x40: "hw_thermal_slowdown", 0x80: "hw_power_brake_slowdown"}
+    NVML_CLOCK_SM = 1
 
-    def __init__(self, gpu_index):
-        self.gpu = gpu_index
+    def __init__(self, gpu_index, uuid=None):
+        self.gpu, self.uuid = gpu_index, uuid
         self.proc = None
         self.file = None
+        self.thread = None
+        self.nvml = self._nvml_handle()
+
+    def _nvml_handle(self):
+        import ctypes as ct
+        try:
+            lib = ct.CDLL("libnvidia-ml.so.1")
+            if lib.nvmlInit_v2() != 0:
+                return None
+            h = ct.c_void_p()
+            rc = -1
+            if self.uuid:
+                rc = lib.nvmlDeviceGetHandleByUUID(self.uuid.encode(), ct.byref(h))
+            if rc != 0:
+                rc = lib.nvmlDeviceGetHandleByIndex_v2(ct.c_uint(self.gpu), ct.byref(h))
+            if rc != 0:
+                return None
+            reasons = getattr(lib, "nvmlDeviceGetCurrentClocksEventReasons", None) or \
+                lib.nvmlDeviceGetCurrentClocksThrottleReasons
+            return lib, h, reasons
+        except (OSError, AttributeError):
+            return None
+
+    def _poll(self):
+        import ctypes as ct
+        lib, h, reasons = self.nvml
+        mhz, mask, mw = ct.c_uint(), ct.c_ulonglong(), ct.c_uint()
+        while not self.done.is_set():
+            if (lib.nvmlDeviceGetClockInfo(h, self.NVML_CLOCK_SM, ct.byref(mhz)) == 0 and
+                    reasons(h, ct.byref(mask)) == 0):
+                pw = mw.value if lib.nvmlDeviceGetPowerUsage(h, ct.byref(mw)) == 0 else 0
+                self.samples.append((mhz.value, mask.value, pw))
+            time.sleep(0.002)
 
     def start(self):
+        if self.nvml:
+            import threading
+            self.samples, self.done = [], threading.Event()
+            self.thread = threading.Thread(target=self._poll, daemon=True)
+            self.thread.start()
+            return
         try:
             self.file = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
             self.proc = subprocess.Popen(
@@ -111,7 +158,26 @@ class ClockSampler:
         except OSError:
             self.proc = None
 
+    def _stop_nvml(self):
+        import ctypes as ct
+        self.done.set()
+        self.thread.join(timeout=5)
+        self.thread = None
+        if not self.samples:
+            return None
+        lib, h, _ = self.nvml
+        mx = ct.c_uint()
+        smax = mx.value if lib.nvmlDeviceGetMaxClockInfo(h, self.NVML_CLOCK_SM,
+                                                         ct.byref(mx)) == 0 else None
+        reasons = sorted({n for _, m, _ in self.samples for bit, n in self.REASONS.items()
+                          if m & bit})
+        return {"sm_mhz": statistics.median(s[0] for s in self.samples), "sm_max_mhz": smax,
+                "reasons": reasons, "samples": len(self.samples),
+                "power_w_max": max(s[2] for s in self.samples) / 1e3, "source": "nvml"}
+
     def stop(self):
+        if self.thread:
+            return self._stop_nvml()
         if not self.proc:
             return None
         self.proc.terminate()
@@ -139,7 +205,7 @@ class ClockSampler:
         if not sm:
             return None
         return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx),
-                "reasons": sorted(reasons), "samples": len(sm)}
+                "reasons": sorted(reasons), "samples": len(sm), "source": "nvidia-smi"}
 
 
 def kernel_sources_sha256():
@@ -180,6 +246,66 @@ def max_over_ranks(x, dist=None, device=None):
 def whole_job_rate(queries_per_rank, world, seconds):
     """Units processed by all ranks over the slowest rank's time."""
     return world * queries_per_rank / seconds
+
+
+class EventTimer:
+    """Seconds between start() and stop(), from CUDA events recorded on the
+    stream the kernels run on (torch's events see only the stream they are
+    recorded on)."""
+
+    def __init__(self, torch, stream):
+        self.torch, self.stream = torch, stream
+        self.e0 = torch.cuda.Event(enable_timing=True)
+        self.e1 = torch.cuda.Event(enable_timing=True)
+
+    def sync(self):
+        self.torch.cuda.synchronize()
+
+    def start(self):
+        self.sync()
+        self.e0.record(self.stream)
+
+    def stop(self):
+        self.e1.record(self.stream)
+        self.sync()
+        return self.e0.elapsed_time(self.e1) * 1e-3
+
+
+class WallTimer:
+    """Host wall-clock seconds (CPU ranks, end-to-end host loops)."""
+
+    def sync(self):
+        pass
+
+    def start(self):
+        self.t = time.perf_counter()
+
+    def stop(self):
+        return time.perf_counter() - self.t
+
+
+def timed_route_loop(route, steps, warmup, timer, dist=None, device=None, before=None,
+                     after=None):
+    """The per-rank timed region: `warmup` untimed calls route(k), then
+    `steps` timed ones between barriers; returns the max over ranks of the
+    seconds per step.  `before` runs after the warm-up (reset counters, start
+    the clock sampler), `after` once the timed calls have finished."""
+    for k in range(warmup):
+        route(k)
+    timer.sync()
+    if before:
+        before()
+    if dist:
+        dist.barrier()
+    timer.start()
+    for k in range(steps):
+        route(k)
+    sec = timer.stop()
+    if after:
+        after()
+    if dist:
+        dist.barrier()
+    return max_over_ranks(sec / steps, dist, device)
 
 
 def dist_env():
@@ -566,29 +692,26 @@ def main():
         r.route_device(il, ol, em, ch, lat, ut, slo=p["slo"], lam=p["lam"],
                        flags=flags | extra)
 
-    for k in range(args.warmup):
-        step(k)
-    torch.cuda.synchronize()
-    r.stats(reset=True)
-    before = r.stats()["kernel_launches"]
-    clocks = ClockSampler(local)
-    if not args.no_clocks:
-        clocks.start()
-    if dist:
-        dist.barrier()
-    torch.cuda.synchronize()
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    for k in range(args.steps):     # queued back to back; status checked after
-        step(k, H.HWR_ASYNC)
-    e1.record(stream)
-    torch.cuda.synchronize()
-    r.synchronize()
-    if dist:
-        dist.barrier()
+    try:
+        uuid = "GPU-" + str(torch.cuda.get_device_properties(dev).uuid)
+    except (AttributeError, RuntimeError):
+        uuid = None
+    clocks = ClockSampler(local, uuid)
+    marks = {}
+
+    def before():
+        r.stats(reset=True)
+        marks["launches"] = r.stats()["kernel_launches"]
+        if not args.no_clocks:
+            clocks.start()
+
+    # warm-up steps synchronous, timed steps queued back to back (the status
+    # word is checked after them)
+    ms = 1e3 * timed_route_loop(lambda k: step(k, H.HWR_ASYNC if marks else 0), args.steps,
+                                args.warmup, EventTimer(torch, stream), dist, dev,
+                                before=before, after=r.synchronize)
     clk = clocks.stop()
-    ms = max_over_ranks(e0.elapsed_time(e1) / args.steps, dist, dev)
-    launches = r.stats(reset=True)["kernel_launches"] - before
+    launches = r.stats(reset=True)["kernel_launches"] - marks["launches"]
     value = whole_job_rate(Q, world, ms * 1e-3)
     # Per-kernel durations: a second pass of the same K steps with CUDA events
     # around every launch (the events sit between the quality and predictor
@@ -657,14 +780,8 @@ def main():
             r.route_host_ptrs(Q, pin[0].data_ptr(), pin[1].data_ptr(), pin[2].data_ptr(),
                               och.data_ptr(), olat.data_ptr(), out_.data_ptr(),
                               slo=p["slo"], lam=p["lam"], flags=flags)
-        for _ in range(args.warmup):
-            host_step()
-        if dist:
-            dist.barrier()
-        t = time.perf_counter()
-        for _ in range(args.steps):
-            host_step()
-        dt = max_over_ranks((time.perf_counter() - t) / args.steps, dist, dev)
+        dt = timed_route_loop(lambda k: host_step(), args.steps, args.warmup, WallTimer(),
+                              dist, dev)
         line["e2e"] = {"value": whole_job_rate(Q, world, dt), "unit": "queries/s",
                        "h2d_bytes_per_step": Q * (bytes_per_query(p) - 12),
                        "d2h_bytes_per_step": Q * 12, "ms_per_step": dt * 1e3}

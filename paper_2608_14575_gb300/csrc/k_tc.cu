@@ -103,39 +103,42 @@ __host__ __device__ inline QualLayout qual_layout(int Mpad, int Epad) {
 constexpr int APRE_SLOTS = 4;   // deployment-prefix ring (layer-1 A_d rows)
 
 struct MlpLayout {
-    uint32_t w2, ring, qual, consts, apre, bars, misc, total;
+    uint32_t w2, ring, qual, consts, w1q, apre, bars, misc, total;
     int ns;
 };
 
-__host__ __device__ inline MlpLayout mlp_layout(int H1, int H2, int Mpad, int D) {
+// Layout with ns ring stages of 16 KB.
+__host__ __device__ inline MlpLayout mlp_layout_ns(int H1, int H2, int Mpad, int D, int ns) {
     MlpLayout L;
-    uint32_t fixed = (uint32_t)H1 * H2 * 2                  // W2 image
-                     + BM * (Mpad + 1) * 4                  // quality rows
-                     + (4 * H2 + 4) * 4 + D * 4 + 16        // b2, W3 (<= 3 rows), b3, dep_model
-                     + APRE_SLOTS * H1 * 2                  // deployment-prefix ring
-                     + (2 * MLP_MAX_STAGES + 6 + 2 * APRE_SLOTS) * 8 + 16   // barriers, misc
-                     + 1024 + 1024;                         // alignment slack
-    int ns = (int)((SMEM_LIMIT - fixed) / CHUNK_BYTES);
-    L.ns = ns > MLP_MAX_STAGES ? MLP_MAX_STAGES : ns;
+    L.ns = ns;
     uint32_t o = 0;
-    L.w2 = o;
+    L.w2 = o;                                   // W2 image (B operand)
     o += (uint32_t)H1 * H2 * 2;
     o = (o + 1023) & ~1023u;
-    L.ring = o;
-    o += (uint32_t)(L.ns > 0 ? L.ns : 0) * CHUNK_BYTES;
-    L.qual = o;
+    L.ring = o;                                 // A-operand ring
+    o += (uint32_t)(ns > 0 ? ns : 0) * CHUNK_BYTES;
+    L.qual = o;                                 // quality rows of the tile
     o += BM * (Mpad + 1) * 4;
-    L.consts = o;
+    L.consts = o;                               // b2, W3 (<= 3 rows), b3, dep_model
     o += (4 * H2 + 4) * 4 + D * 4;
     o = (o + 15) & ~15u;
-    L.apre = o;
+    L.w1q = o;                                  // W1's query columns, pairs interleaved
+    o += (uint32_t)H1 * 2 * 4;
+    L.apre = o;                                 // deployment-prefix ring
     o += APRE_SLOTS * H1 * 2;
     L.bars = o;
     o += (2 * MLP_MAX_STAGES + 6 + 2 * APRE_SLOTS) * 8;
     L.misc = o;
     o += 16;
-    L.total = o + 1024;
+    L.total = o + 1024;                         // slack for aligning the dynamic base
     return L;
+}
+
+// As many ring stages as fit (at most MLP_MAX_STAGES).
+__host__ __device__ inline MlpLayout mlp_layout(int H1, int H2, int Mpad, int D) {
+    const uint32_t base = mlp_layout_ns(H1, H2, Mpad, D, 0).total;
+    int ns = base < SMEM_LIMIT ? (int)((SMEM_LIMIT - base) / CHUNK_BYTES) : 0;
+    return mlp_layout_ns(H1, H2, Mpad, D, ns > MLP_MAX_STAGES ? MLP_MAX_STAGES : ns);
 }
 
 __device__ __forceinline__ uint8_t *align1024(uint8_t *p) {
@@ -420,6 +423,11 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
     }
     if (tid < NH) b3s[tid] = hc.b3[tid];
     for (int i = tid; i < D; i += MLP_THREADS) dms[i] = m.dep_model[i];
+    // W1's two query columns as {W1[k][in], W1[k+1][in], W1[k][out], W1[k+1][out]}
+    // per pair of rows k: one 16-byte load serves a pair for every query row
+    float4 *w1qs = (float4 *)(sm + L.w1q);
+    for (int i = tid; i < H1 / 2; i += MLP_THREADS)
+        w1qs[i] = make_float4(m.W1q[2 * i], m.W1q[2 * i + 1], m.W1q[H1 + 2 * i], m.W1q[H1 + 2 * i + 1]);
     if (warp == 0) {
         tmem_alloc(tslot, tcols);
         tmem_relinquish();
@@ -627,23 +635,27 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
         uint32_t dn = 0;
         for (int u = blockIdx.x; ok && u < nunits; u += gridDim.x) {
             const Unit un = unit_of(u, ntiles, nsplit, D);
+            // this thread's rows' standardised query slots, then the query
+            // part of its granules (W1 pairs from shared memory, each used
+            // for the four rows)
+            float uu[4], vv[4];
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
                 const int row = un.tile * BM + rb + 32 * i;
                 const bool valid = row < q.Q;
-                const float uu = valid ? standardise_fast(m.xf_in, q.in_len[row], m.mu_in, m.sd_in) : 0.f;
-                const float vv = valid ? standardise_fast(m.xf_out, q.out_len[row], m.mu_out, m.sd_out) : 0.f;
+                uu[i] = valid ? standardise_fast(m.xf_in, q.in_len[row], m.mu_in, m.sd_in) : 0.f;
+                vv[i] = valid ? standardise_fast(m.xf_out, q.out_len[row], m.mu_out, m.sd_out) : 0.f;
+            }
 #pragma unroll
-                for (int c = 0; c < 4; ++c) {
-                    if (c < nch) {
-                        const int k0 = c * KCH + gi * 8;
+            for (int c = 0; c < 4; ++c) {
+                if (c < nch) {
 #pragma unroll
-                        for (int e = 0; e < 4; ++e) {
-                            const float2 wi = *(const float2 *)(m.W1q + k0 + 2 * e);
-                            const float2 wo = *(const float2 *)(m.W1q + H1 + k0 + 2 * e);
-                            Bq[i][c][e] = pack_bf16x2(fmaf(vv, wo.x, uu * wi.x),
-                                                      fmaf(vv, wo.y, uu * wi.y));
-                        }
+                    for (int e = 0; e < 4; ++e) {
+                        const float4 w = w1qs[c * (KCH / 2) + gi * 4 + e];
+#pragma unroll
+                        for (int i = 0; i < 4; ++i)
+                            Bq[i][c][e] = pack_bf16x2(fmaf(vv[i], w.z, uu[i] * w.x),
+                                                      fmaf(vv[i], w.w, uu[i] * w.y));
                     }
                 }
             }

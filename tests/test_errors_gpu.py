@@ -4,6 +4,9 @@
   every n must give HWR_ERR_OOM and leave the process able to create the next
   context.
 * Argument errors leave the context usable.
+* A snapshot value outside the domain of its feature's transform (negative
+  queue, non-finite value, <= 0 under log, <= -1 under log1p) is rejected and
+  the previous snapshot stays in force.
 * HWR_TEST_STALL=1 makes the tensor-path producers never signal their tiles,
   so the predictor kernel's bounded waits (about a second) run out: the call
   returns HWR_ERR_TIMEOUT, the context refuses further work (HWR_ERR_STATE),
@@ -124,4 +127,39 @@ def test_bounded_wait_expires_into_timeout_status(monkeypatch):
     simt = r.route(flags=H.HWR_PATH_SIMT)
     same = tc[0] == simt[0]
     assert same.mean() > 0.95
+    r.close()
+
+
+@pytest.mark.parametrize("key,value", [("running", -1), ("waiting", -2), ("kv", np.nan),
+                                       ("gpu_util", np.inf), ("ttft", 0.0), ("tpot", -1e-3)])
+def test_snapshot_values_outside_their_domain_are_rejected(key, value):
+    p = W.make_config(0, Q=32)
+    r = H.Router(p)
+    want = r.route()
+    bad = {k: np.array(v, copy=True) for k, v in p["snap"].items()}
+    bad[key][1] = value
+    with pytest.raises(H.HwrError) as e:
+        r.update_snapshot(bad)
+    assert e.value.status == _hwr.HWR_ERR_INVALID_ARG, e.value
+    assert "[1]" in str(e.value)
+    # the context keeps its previous snapshot and routes as before
+    got = r.route()
+    assert all(np.array_equal(a, b) for a, b in zip(got, want))
+    r.close()
+
+
+def test_log1p_slot_accepts_values_above_minus_one_only():
+    p = W.make_config(0, Q=8)
+    P = p["M"] + p["G"]
+    p["xform"] = np.array(p["xform"], copy=True)
+    p["xform"][P + 3] = 1                  # KV utilisation through log1p
+    r = H.Router(p)
+    snap = {k: np.array(v, copy=True) for k, v in p["snap"].items()}
+    snap["kv"][0] = -0.5                   # log1p(-0.5) is defined
+    r.update_snapshot(snap)
+    snap["kv"][0] = -1.0
+    with pytest.raises(H.HwrError) as e:
+        r.update_snapshot(snap)
+    assert e.value.status == _hwr.HWR_ERR_INVALID_ARG and "log1p" in str(e.value)
+    assert r.route()[0].min() >= 0
     r.close()

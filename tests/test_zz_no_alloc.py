@@ -6,7 +6,8 @@ cache, or a serving loop that must not take cudaMalloc's device-wide
 synchronisation).  The call must give the same decisions as hwr_route_batch
 on the same inputs -- on two calls in a row, with different batches, so that
 what the first call leaves in the shared scratch cannot leak into the second
--- must not allocate, and must reject batches larger than its fixed scratch.
+-- and agree with the fp64 oracle within the tensor path's tolerance; it must
+not allocate, and must reject batches larger than its fixed scratch.
 
 Collected last on purpose (file name), so a run that stops at the first
 failure has run every other test before this one.
@@ -16,6 +17,7 @@ import pytest
 
 import workload as W
 import paper_2608_14575_gb300 as H
+from tc_check import check_against_oracle
 
 pytestmark = pytest.mark.gpu
 TOL = 2e-2
@@ -57,6 +59,11 @@ def test_noalloc_matches_route_batch_on_two_calls():
         r.route_device_noalloc(*inp, *got, slo=p["slo"], lam=p["lam"])
         torch.cuda.synchronize()
         _close(got, ref)
+        # and against the oracle, on every 13th query of the batch
+        full = [np.zeros(p["Q"], dt) for dt in (np.int32, np.float32, np.float32)]
+        for f, x in zip(full, got):
+            f[lo:hi] = x.cpu().numpy()
+        check_against_oracle(p, full, idx=np.arange(lo, hi, 13))
     r.close()
 
 
