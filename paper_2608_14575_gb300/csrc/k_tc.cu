@@ -103,12 +103,17 @@ __host__ __device__ inline QualLayout qual_layout(int Mpad, int Epad) {
 constexpr int APRE_SLOTS = 4;   // deployment-prefix ring (layer-1 A_d rows)
 
 struct MlpLayout {
-    uint32_t w2, ring, qual, consts, w1q, apre, bars, misc, total;
+    uint32_t w2, ring, qual, consts, w1q, uvs, apre, bars, misc, total;
     int ns;
 };
 
-// Layout with ns ring stages of 16 KB.
-__host__ __device__ inline MlpLayout mlp_layout_ns(int H1, int H2, int Mpad, int D, int ns) {
+constexpr int MLP_BARS = 2 * MLP_MAX_STAGES + 6 + 2 * APRE_SLOTS + 4;
+
+// Layout with ns ring stages of 16 KB.  head_smem: the output-layer
+// constants b2, W3 also in shared memory (kernels without a fixed H2 read
+// them there; the others take them from the kernel-parameter bank).
+__host__ __device__ inline MlpLayout mlp_layout_ns(int H1, int H2, int Mpad, int D, int ns,
+                                                   bool head_smem) {
     MlpLayout L;
     L.ns = ns;
     uint32_t o = 0;
@@ -119,15 +124,17 @@ __host__ __device__ inline MlpLayout mlp_layout_ns(int H1, int H2, int Mpad, int
     o += (uint32_t)(ns > 0 ? ns : 0) * CHUNK_BYTES;
     L.qual = o;                                 // quality rows of the tile
     o += BM * (Mpad + 1) * 4;
-    L.consts = o;                               // b2, W3 (<= 3 rows), b3, dep_model
-    o += (4 * H2 + 4) * 4 + D * 4;
+    L.consts = o;                               // [b2, W3 (<= 3 rows)], b3, dep_model
+    o += (head_smem ? 4 * H2 * 4 : 0) + 16 + D * 4;
     o = (o + 15) & ~15u;
     L.w1q = o;                                  // W1's query columns, pairs interleaved
     o += (uint32_t)H1 * 2 * 4;
+    L.uvs = o;                                  // standardised query slots [2][2][BM]
+    o += 2 * 2 * BM * 4;
     L.apre = o;                                 // deployment-prefix ring
     o += APRE_SLOTS * H1 * 2;
     L.bars = o;
-    o += (2 * MLP_MAX_STAGES + 6 + 2 * APRE_SLOTS) * 8;
+    o += MLP_BARS * 8;
     L.misc = o;
     o += 16;
     L.total = o + 1024;                         // slack for aligning the dynamic base
@@ -135,11 +142,15 @@ __host__ __device__ inline MlpLayout mlp_layout_ns(int H1, int H2, int Mpad, int
 }
 
 // As many ring stages as fit (at most MLP_MAX_STAGES).
-__host__ __device__ inline MlpLayout mlp_layout(int H1, int H2, int Mpad, int D) {
-    const uint32_t base = mlp_layout_ns(H1, H2, Mpad, D, 0).total;
+__host__ __device__ inline MlpLayout mlp_layout(int H1, int H2, int Mpad, int D, bool head_smem) {
+    const uint32_t base = mlp_layout_ns(H1, H2, Mpad, D, 0, head_smem).total;
     int ns = base < SMEM_LIMIT ? (int)((SMEM_LIMIT - base) / CHUNK_BYTES) : 0;
-    return mlp_layout_ns(H1, H2, Mpad, D, ns > MLP_MAX_STAGES ? MLP_MAX_STAGES : ns);
+    return mlp_layout_ns(H1, H2, Mpad, D, ns > MLP_MAX_STAGES ? MLP_MAX_STAGES : ns, head_smem);
 }
+
+// The predictor kernel has a variant with H2 fixed at compile time for these
+// widths (output-layer constants in the parameter bank).
+__host__ __device__ inline bool mlp_fixed_h2(int H2) { return H2 == 128 || H2 == 256; }
 
 __device__ __forceinline__ uint8_t *align1024(uint8_t *p) {
     const uint32_t a = smem_u32(p);
@@ -363,6 +374,16 @@ __device__ __forceinline__ void head_pair(const uint32_t *v, int j, const float4
     }
 }
 
+// Standardised query slots of query `row` into slot r of a [2][BM] buffer
+// (u: input length, v: output length), then arrive on `full`.
+__device__ __forceinline__ void put_slots(const TcModel &m, const Queries &q, int row, int r,
+                                          float *uv, uint64_t *full) {
+    const bool v = row < q.Q;
+    uv[r] = v ? standardise_fast(m.xf_in, q.in_len[row], m.mu_in, m.sd_in) : 0.f;
+    uv[BM + r] = v ? standardise_fast(m.xf_out, q.out_len[row], m.mu_out, m.sd_out) : 0.f;
+    mbar_arrive(full);
+}
+
 // Output-layer constants passed by value: they sit in the kernel-parameter
 // constant bank, so the fully unrolled epilogue reads them as instruction
 // operands instead of shared-memory loads.  nb2 = -b2; b3 holds the head
@@ -379,16 +400,19 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
     uint8_t *sm = align1024(smem_raw);
     constexpr bool FIXED = H2T > 0;
     const int H1 = m.H1, H2 = FIXED ? H2T : m.H2, D = m.D, Mpad = m.Mpad, QS = Mpad + 1;
-    const MlpLayout L = mlp_layout(H1, H2, Mpad, D);
+    const MlpLayout L = mlp_layout(H1, H2, Mpad, D, !FIXED);
     const int NS = L.ns;
     uint8_t *w2s = sm + L.w2, *ring = sm + L.ring;
     float *qs = (float *)(sm + L.qual);
+    // b2 (negated), W3 rows: only without a fixed H2
     float *b2s = (float *)(sm + L.consts), *w30s = b2s + H2, *w31s = w30s + H2;
-    float *w32s = w31s + H2, *b3s = w32s + H2;
+    float *w32s = w31s + H2, *b3s = FIXED ? b2s : w32s + H2;
     int *dms = (int *)(b3s + 4);
+    float *uvs = (float *)(sm + L.uvs);        // [buffer][u / v][row]
     uint64_t *full = (uint64_t *)(sm + L.bars), *empty = full + MLP_MAX_STAGES;
     uint64_t *accf = empty + MLP_MAX_STAGES, *acce = accf + 2, *wbar = acce + 2, *dbar = wbar + 1;
     uint64_t *afull = dbar + 1, *afree = afull + APRE_SLOTS;   // prefix ring
+    uint64_t *uvfull = afree + APRE_SLOTS, *uvfree = uvfull + 2;   // query slots
     uint8_t *apre = sm + L.apre;
     uint32_t *tslot = (uint32_t *)(sm + L.misc);
     volatile int *abort_f = (volatile int *)(tslot + 1);
@@ -412,14 +436,20 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
             mbar_init(&afull[j], 1);
             mbar_init(&afree[j], MLP_PRODUCERS);
         }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&uvfull[b], 128);
+            mbar_init(&uvfree[b], MLP_PRODUCERS / 32);
+        }
         *abort_f = 0;
         fence_mbar_init();
     }
-    for (int i = tid; i < H2; i += MLP_THREADS) {
-        b2s[i] = hc.nb2[i];
-        w30s[i] = m.W3[i];
-        w31s[i] = m.W3[H2 + i];
-        w32s[i] = NH == 3 ? m.W3[2 * H2 + i] : 0.f;
+    if (!FIXED) {
+        for (int i = tid; i < H2; i += MLP_THREADS) {
+            b2s[i] = hc.nb2[i];
+            w30s[i] = m.W3[i];
+            w31s[i] = m.W3[H2 + i];
+            w32s[i] = NH == 3 ? m.W3[2 * H2 + i] : 0.f;
+        }
     }
     if (tid < NH) b3s[tid] = hc.b3[tid];
     for (int i = tid; i < D; i += MLP_THREADS) dms[i] = m.dep_model[i];
@@ -490,11 +520,26 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
         const int ncol = H2 / 32;
         uint32_t g = 0;
         bool ok = true;
+        // The standardised query slots u, v of row r for the producers (one
+        // row per thread), one unit ahead: the local unit k uses buffer k & 1,
+        // refilled once the producers have read it for unit k - 2.
+        if (blockIdx.x < nunits)   // the lengths are inputs: no wait for the kernel before
+            put_slots(m, q, unit_of(blockIdx.x, ntiles, nsplit, D).tile * BM + r, r, uvs,
+                      &uvfull[0]);
         // the quality matrix comes from the kernel before (a dependent launch
         // may start this grid before that one has finished)
         grid_dependency_wait();
-        for (int u = blockIdx.x; ok && u < nunits; u += gridDim.x) {
+        int lk = 0;
+        for (int u = blockIdx.x; ok && u < nunits; u += gridDim.x, ++lk) {
             const Unit un = unit_of(u, ntiles, nsplit, D);
+            if (u + (int)gridDim.x < nunits) {
+                const int k = lk + 1, b = k & 1;
+                if (k >= 2) ok = mbar_wait(&uvfree[b], ((k >> 1) & 1) ^ 1, abort_f, status);
+                ok = __all_sync(0xffffffffu, ok);
+                if (!ok) break;
+                put_slots(m, q, unit_of(u + gridDim.x, ntiles, nsplit, D).tile * BM + r, r,
+                          uvs + 2 * b * BM, &uvfull[b]);
+            }
             const int row = un.tile * BM + r;
             const bool valid = row < q.Q;
             const float ol = valid ? q.out_len[row] : 0.f;
@@ -633,19 +678,26 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
         // built every chunk from its granules.  dn counts this CTA's deployments.
         const uint32_t abytes = (uint32_t)H1 * 2;
         uint32_t dn = 0;
-        for (int u = blockIdx.x; ok && u < nunits; u += gridDim.x) {
+        int lk = 0;
+        for (int u = blockIdx.x; ok && u < nunits; u += gridDim.x, ++lk) {
             const Unit un = unit_of(u, ntiles, nsplit, D);
-            // this thread's rows' standardised query slots, then the query
-            // part of its granules (W1 pairs from shared memory, each used
-            // for the four rows)
+            // standardised query slots of this thread's four rows, prepared by
+            // the epilogue warps
+            const int ub = lk & 1;
+            ok = mbar_wait(&uvfull[ub], (lk >> 1) & 1, abort_f, status);
+            ok = __all_sync(0xffffffffu, ok);
+            if (!ok) break;
             float uu[4], vv[4];
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
-                const int row = un.tile * BM + rb + 32 * i;
-                const bool valid = row < q.Q;
-                uu[i] = valid ? standardise_fast(m.xf_in, q.in_len[row], m.mu_in, m.sd_in) : 0.f;
-                vv[i] = valid ? standardise_fast(m.xf_out, q.out_len[row], m.mu_out, m.sd_out) : 0.f;
+                uu[i] = uvs[(2 * ub) * BM + rb + 32 * i];
+                vv[i] = uvs[(2 * ub + 1) * BM + rb + 32 * i];
             }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&uvfree[ub]);
+            // the query part of this thread's granules: W1 pairs from shared
+            // memory, each used for the four rows, as packed fp32 products
+            // (per lane: fma(v, W1[out], u * W1[in]))
 #pragma unroll
             for (int c = 0; c < 4; ++c) {
                 if (c < nch) {
@@ -653,12 +705,15 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
                     for (int e = 0; e < 4; ++e) {
                         const float4 w = w1qs[c * (KCH / 2) + gi * 4 + e];
 #pragma unroll
-                        for (int i = 0; i < 4; ++i)
-                            Bq[i][c][e] = pack_bf16x2(fmaf(vv[i], w.z, uu[i] * w.x),
-                                                      fmaf(vv[i], w.w, uu[i] * w.y));
+                        for (int i = 0; i < 4; ++i) {
+                            const float2 pr = __fmul2_rn(make_float2(uu[i], uu[i]), make_float2(w.x, w.y));
+                            const float2 h = __ffma2_rn(make_float2(vv[i], vv[i]), make_float2(w.z, w.w), pr);
+                            Bq[i][c][e] = pack_bf16x2(h.x, h.y);
+                        }
                     }
                 }
             }
+
             uint4 a[4];
             for (int d = un.d0; ok && d < un.d1; ++d, ++dn) {
                 const int j = dn & (APRE_SLOTS - 1);
@@ -760,7 +815,7 @@ bool tc_supported(int M, int H1, int H2, int E) {
     if (E < 8 || E % 8) return false;
     const int Mpad = M <= 16 ? 16 : 32, Epad = (E + 63) / 64 * 64;
     if (qual_layout(Mpad, Epad).total > SMEM_LIMIT) return false;
-    const MlpLayout L = mlp_layout(H1, H2, Mpad, 64);
+    const MlpLayout L = mlp_layout(H1, H2, Mpad, 64, !mlp_fixed_h2(H2));
     return L.ns >= 2 && L.total <= SMEM_LIMIT;
 }
 
@@ -845,7 +900,7 @@ cudaError_t launch_mlp_tc(const TcModel &m, const Queries &q, const float *qual,
     if (q.Q <= 0) return cudaSuccess;
     const long units = (long)((q.Q + BM - 1) / BM) * nsplit;
     const int grid = units < g_num_sms ? (int)units : g_num_sms;
-    const MlpLayout L = mlp_layout(m.H1, m.H2, m.Mpad, m.D);
+    const MlpLayout L = mlp_layout(m.H1, m.H2, m.Mpad, m.D, !mlp_fixed_h2(m.H2));
     const HeadConsts &hc = *m.head;
     int4 *pt = (int4 *)part;
     // programmatic dependent launch: the grid may start while the quality
