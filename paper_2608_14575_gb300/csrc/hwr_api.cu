@@ -728,9 +728,9 @@ static hwr_status run_kernels(hwr_ctx *c, const Queries &q, uint32_t flags, bool
     if (tensor) {
         const TcModel t = tc_view(c);
         TRY(grow(c, &c->qual, &c->qual_cap, (size_t)q.Q * c->Mpad));
-        const int ns = tc_mlp_split(t, q.Q);
-        if (ns > 1) {
-            TRY(grow(c, &c->part, &c->part_cap, (size_t)ns * q.Q * 16));
+        const MlpSplit sp = tc_mlp_split(t, q.Q);
+        if (sp.nsplit > 1) {
+            TRY(grow(c, &c->part, &c->part_cap, (size_t)sp.nsplit * q.Q * 16));
             if (c->count_cap < (size_t)q.Q) {
                 TRY(grow(c, &c->count, &c->count_cap, (size_t)q.Q));
                 CK(c, cudaMemsetAsync(c->count, 0, c->count_cap * 4, c->stream), "zero counters");
@@ -740,7 +740,7 @@ static hwr_status run_kernels(hwr_ctx *c, const Queries &q, uint32_t flags, bool
         CK(c, launch_qual_tc(t, q, c->qual, c->status_d, c->stream), "quality kernel");
         a.done();
         LaunchScope b(c, HWR_K_MLP_TC, prof);
-        CK(c, launch_mlp_tc(t, q, c->qual, ns, c->part, c->count, c->status_d, c->stream),
+        CK(c, launch_mlp_tc(t, q, c->qual, sp, c->part, c->count, c->status_d, c->stream),
            "predictor kernel");
         b.done();
         return HWR_OK;
@@ -1176,14 +1176,13 @@ hwr_status hwr_internal_route_tensor_scratch(hwr_ctx *c, int32_t Q, const float 
     q.lat = pred_latency;
     q.util = utility;
     const TcModel t = tc_view(c);
-    int ns = tc_mlp_split(t, Q);
-    if (ns > max_split) ns = max_split;
-    if (ns > 1)
+    const MlpSplit sp = tc_mlp_split(t, Q, max_split);
+    if (sp.nsplit > 1)
         CK(c, cudaMemsetAsync(count, 0, (size_t)Q * sizeof(int32_t), c->stream), "clear counters");
     CK(c, launch_qual_tc(t, q, qual, c->status_d, c->stream), "quality kernel");
     c->stats.kernel_launches++;
     c->stats.launches[HWR_K_QUAL_TC]++;
-    CK(c, launch_mlp_tc(t, q, qual, ns, part, count, c->status_d, c->stream), "predictor kernel");
+    CK(c, launch_mlp_tc(t, q, qual, sp, part, count, c->status_d, c->stream), "predictor kernel");
     c->stats.kernel_launches++;
     c->stats.launches[HWR_K_MLP_TC]++;
     c->stats.queries_routed += Q;

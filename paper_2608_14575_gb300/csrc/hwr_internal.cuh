@@ -183,12 +183,16 @@ void tc_build_membimg(const uint16_t *memb_EM, int E, int M, int Mpad, int Epad,
 // qual: scratch [Q][Mpad] fp32.  status: device int32 word.
 cudaError_t launch_qual_tc(const TcModel &m, const Queries &q, float *qual,
                            int32_t *status, cudaStream_t s);
-// Deployments of a tile may be split over `nsplit` units; then `part`
+// The first nwhole query tiles are processed whole; the deployments of each
+// remaining tile are split over nsplit units.  With nsplit > 1, `part`
 // (nsplit * Q records of 16 bytes) and `count` (Q int32, zero, self-resetting)
 // are scratch.
-int tc_mlp_split(const TcModel &m, int Q);
+struct MlpSplit {
+    int nwhole, nsplit;
+};
+MlpSplit tc_mlp_split(const TcModel &m, int Q, int max_split = 8);
 cudaError_t launch_mlp_tc(const TcModel &m, const Queries &q, const float *qual,
-                          int nsplit, void *part, int32_t *count, int32_t *status,
+                          const MlpSplit &sp, void *part, int32_t *count, int32_t *status,
                           cudaStream_t s);
 cudaError_t tc_prepare();
 // Costs of every (query, deployment) pair of at most 128 queries into

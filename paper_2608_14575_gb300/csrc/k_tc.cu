@@ -319,20 +319,34 @@ k_qual_tc(const __grid_constant__ CUtensorMap tmap, TcModel m, int Q, float *qua
 // ---------------------------------------------------------------------------
 // K_mlp_tc
 //
-// Work unit = (query tile, part of the deployment range).  With more than one
-// part per tile, each unit leaves its per-row best candidate in `part` and the
-// last of a row's units to arrive (per-row atomic counter) merges them.
+// Work unit = (query tile, part of the deployment range).  The first nwhole
+// tiles are units of all D deployments; each remaining tile is split into
+// nsplit parts, dealt after them (so the split tiles even out the last,
+// partial round over the CTAs).  A part leaves its per-row best candidate in
+// `part` and the last of a row's parts to arrive (per-row atomic counter)
+// merges them; whole tiles write their decisions directly.
 
 struct Unit {
-    int tile, part, d0, d1;
+    int tile, d0, d1;
 };
 
-__device__ __forceinline__ Unit unit_of(int u, int ntiles, int nsplit, int D) {
+__host__ __device__ __forceinline__ int unit_part(int u, int ntiles, int nwhole) {
+    return u < nwhole ? 0 : (u - nwhole) / (ntiles - nwhole);
+}
+
+__host__ __device__ __forceinline__ Unit unit_of(int u, int ntiles, int nwhole, int nsplit,
+                                                 int D) {
     Unit x;
-    x.tile = u % ntiles;
-    x.part = u / ntiles;
-    x.d0 = x.part * D / nsplit;
-    x.d1 = (x.part + 1) * D / nsplit;
+    if (u < nwhole) {
+        x.tile = u;
+        x.d0 = 0;
+        x.d1 = D;
+        return x;
+    }
+    const int v = u - nwhole, ntail = ntiles - nwhole, part = v / ntail;
+    x.tile = nwhole + (v - part * ntail);
+    x.d0 = part * D / nsplit;
+    x.d1 = (part + 1) * D / nsplit;
     return x;
 }
 
@@ -395,7 +409,8 @@ struct HeadConsts {
 template <int H2T, int NH>
 __global__ void __launch_bounds__(MLP_THREADS, 1)
 k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
-         const float *__restrict__ qual, int nsplit, int4 *part, int32_t *count, int32_t *status) {
+         const float *__restrict__ qual, int nwhole, int nsplit, int4 *part, int32_t *count,
+         int32_t *status) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *sm = align1024(smem_raw);
     constexpr bool FIXED = H2T > 0;
@@ -417,7 +432,7 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
     uint32_t *tslot = (uint32_t *)(sm + L.misc);
     volatile int *abort_f = (volatile int *)(tslot + 1);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int nch = H1 / KCH, ntiles = (q.Q + BM - 1) / BM, nunits = ntiles * nsplit;
+    const int nch = H1 / KCH, ntiles = (q.Q + BM - 1) / BM, nunits = nwhole + (ntiles - nwhole) * nsplit;
     const uint32_t tcols = 2 * H2 <= 32 ? 32 : 2 * H2 <= 64 ? 64 : 2 * H2 <= 128 ? 128
                                                 : 2 * H2 <= 256 ? 256 : 512;
 
@@ -479,7 +494,7 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
         uint32_t g = 0, ph = 0;
         int s = 0;
         for (int u = blockIdx.x; ok && u < nunits; u += gridDim.x) {
-            const Unit un = unit_of(u, ntiles, nsplit, D);
+            const Unit un = unit_of(u, ntiles, nwhole, nsplit, D);
             for (int d = un.d0; d < un.d1; ++d, ++g) {
                 const int b = g & 1;
                 ok = mbar_wait(&acce[b], ((g >> 1) & 1) ^ 1, abort_f, status);
@@ -524,20 +539,20 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
         // row per thread), one unit ahead: the local unit k uses buffer k & 1,
         // refilled once the producers have read it for unit k - 2.
         if (blockIdx.x < nunits)   // the lengths are inputs: no wait for the kernel before
-            put_slots(m, q, unit_of(blockIdx.x, ntiles, nsplit, D).tile * BM + r, r, uvs,
+            put_slots(m, q, unit_of(blockIdx.x, ntiles, nwhole, nsplit, D).tile * BM + r, r, uvs,
                       &uvfull[0]);
         // the quality matrix comes from the kernel before (a dependent launch
         // may start this grid before that one has finished)
         grid_dependency_wait();
         int lk = 0;
         for (int u = blockIdx.x; ok && u < nunits; u += gridDim.x, ++lk) {
-            const Unit un = unit_of(u, ntiles, nsplit, D);
+            const Unit un = unit_of(u, ntiles, nwhole, nsplit, D);
             if (u + (int)gridDim.x < nunits) {
                 const int k = lk + 1, b = k & 1;
                 if (k >= 2) ok = mbar_wait(&uvfree[b], ((k >> 1) & 1) ^ 1, abort_f, status);
                 ok = __all_sync(0xffffffffu, ok);
                 if (!ok) break;
-                put_slots(m, q, unit_of(u + gridDim.x, ntiles, nsplit, D).tile * BM + r, r,
+                put_slots(m, q, unit_of(u + gridDim.x, ntiles, nwhole, nsplit, D).tile * BM + r, r,
                           uvs + 2 * b * BM, &uvfull[b]);
             }
             const int row = un.tile * BM + r;
@@ -622,22 +637,28 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
                 if (better(cd, best)) best = cd;
             }
             if (!ok || !valid || q.no_select) continue;
-            if (nsplit == 1) {
+            const int nparts = u < nwhole ? 1 : nsplit;
+            if (nparts == 1) {
                 const bool sel = best.cls > 0;
                 q.chosen[row] = sel ? best.d : -1;
                 q.lat[row] = sel ? best.C : __int_as_float(0x7fc00000);
                 q.util[row] = sel ? best.U : __int_as_float(0x7fc00000);
                 continue;
             }
-            part[(size_t)un.part * q.Q + row] =
+            part[(size_t)unit_part(u, ntiles, nwhole) * q.Q + row] =
                 make_int4(best.cls, best.d, __float_as_int(best.C), __float_as_int(best.U));
-            __threadfence();
-            if (atomicAdd(&count[row], 1) == nsplit - 1) {
+            // release: the record above is visible to whoever increments the
+            // counter later; acquire: the last arrival sees every record
+            int seen;
+            asm volatile("atom.acq_rel.gpu.global.add.s32 %0, [%1], 1;"
+                         : "=r"(seen)
+                         : "l"(count + row)
+                         : "memory");
+            if (seen == nparts - 1) {
                 // last of this row's units: merge the parts (any order gives the
                 // same result: the candidate order is total)
-                __threadfence();
                 Cand acc = no_cand();
-                for (int pp = 0; pp < nsplit; ++pp) {
+                for (int pp = 0; pp < nparts; ++pp) {
                     const int4 x = __ldcg(&part[(size_t)pp * q.Q + row]);
                     Cand c;
                     c.cls = x.x;
@@ -661,13 +682,10 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
         // built once per unit in registers (bf16 pairs) and every step then
         // needs one fused add + ReLU per pair: relu(1 * B + A_d).
         const int p = tid - 160, gi = p & 7, rb = p >> 3;
-        uint32_t offs[4];
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            const int r = rb + 32 * i;
-            offs[i] = (uint32_t)(r >> 3) * 1024 + (uint32_t)(r & 7) * 128 +
-                      (uint32_t)((gi ^ (r & 7)) << 4);
-        }
+        // shared-memory offset of granule gi of row rb in a stage (K-major,
+        // 128-byte swizzle); row rb + 32 i sits 4 atoms (4096 bytes) further
+        const uint32_t offs0 = (uint32_t)(rb >> 3) * 1024 + (uint32_t)(rb & 7) * 128 +
+                               (uint32_t)((gi ^ (rb & 7)) << 4);
         const uint32_t one2 = 0x3F803F80u;  // (1.0, 1.0) in bf16
         uint32_t Bq[4][4][4];
         uint32_t ph = 0;
@@ -680,7 +698,7 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
         uint32_t dn = 0;
         int lk = 0;
         for (int u = blockIdx.x; ok && u < nunits; u += gridDim.x, ++lk) {
-            const Unit un = unit_of(u, ntiles, nsplit, D);
+            const Unit un = unit_of(u, ntiles, nwhole, nsplit, D);
             // standardised query slots of this thread's four rows, prepared by
             // the epilogue warps
             const int ub = lk & 1;
@@ -714,21 +732,21 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
                 }
             }
 
-            uint4 a[4];
             for (int d = un.d0; ok && d < un.d1; ++d, ++dn) {
                 const int j = dn & (APRE_SLOTS - 1);
                 ok = ok && mbar_wait(&afull[j], (dn / APRE_SLOTS) & 1, abort_f, status);
                 if (!ok) break;
                 const uint4 *As = (const uint4 *)(apre + j * abytes);
-#pragma unroll
-                for (int c = 0; c < 4; ++c)
-                    if (c < nch) a[c] = As[c * 8 + gi];
                 // two chunks per round: one wait / fence / arrive cycle covers
                 // both, halving the serial latency each producer warp pays
 #pragma unroll
                 for (int c = 0; c < 4; c += 2) {
                     if (c < nch && ok) {
                         const bool two = c + 1 < nch;
+                        // this round's prefix granules (loaded before the waits)
+                        uint4 a[2];
+                        a[0] = As[c * 8 + gi];
+                        if (two) a[1] = As[(c + 1) * 8 + gi];
                         const int s1 = s + 1 == NS ? 0 : s + 1;
                         const uint32_t ph1 = s + 1 == NS ? ph ^ 1 : ph;
                         ok = mbar_wait(&empty[s], ph ^ 1, abort_f, status);
@@ -737,7 +755,7 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
 #pragma unroll
                             for (int cc = 0; cc < 2; ++cc) {
                                 if (cc == 0 || two) {
-                                    const uint4 av = a[c + cc];
+                                    const uint4 av = a[cc];
                                     const uint32_t st = smem_u32(ring + (cc ? s1 : s) * CHUNK_BYTES);
 #pragma unroll
                                     for (int i = 0; i < 4; ++i) {
@@ -746,7 +764,7 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
                                         const uint32_t h2 = hfma2_relu(Bq[i][c + cc][2], one2, av.z);
                                         const uint32_t h3 = hfma2_relu(Bq[i][c + cc][3], one2, av.w);
                                         asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(
-                                                         st + offs[i]),
+                                                         st + offs0 + 4096u * i),
                                                      "r"(h0), "r"(h1), "r"(h2), "r"(h3)
                                                      : "memory");
                                     }
@@ -781,7 +799,7 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
         uint32_t issued = 0;
         bool ok = true;
         for (int u = blockIdx.x; ok && u < nunits; u += gridDim.x) {
-            const Unit un = unit_of(u, ntiles, nsplit, D);
+            const Unit un = unit_of(u, ntiles, nwhole, nsplit, D);
             for (int d = un.d0; d < un.d1; ++d, ++issued) {
                 const int j = issued & (APRE_SLOTS - 1);
                 if (issued >= APRE_SLOTS)
@@ -874,31 +892,47 @@ cudaError_t launch_mlp_tc_scores(const TcModel &m, const Queries &q, const float
     if (q.seq_n && (q.seq_n != q.Q || m.D % (q.seq_n + 1))) return cudaErrorInvalidValue;
     // one tile: split its deployments into one part per SM
     const int sms = g_num_sms > 0 ? g_num_sms : 1;
-    const int ns = m.D < sms ? m.D : sms;
-    return launch_mlp_tc(m, q, qual, ns, nullptr, nullptr, status, s);
+    const MlpSplit sp{0, m.D < sms ? m.D : sms};
+    return launch_mlp_tc(m, q, qual, sp, nullptr, nullptr, status, s);
 }
 
-// Deployment split per tile that minimises the busiest CTA's step count
-// (each unit also pays about half a step of per-unit setup).
-int tc_mlp_split(const TcModel &m, int Q) {
-    const int ntiles = (Q + BM - 1) / BM, sms = g_num_sms > 0 ? g_num_sms : 1;
-    int best = 1;
+// Unit decomposition that minimises the busiest CTA's cost in deployment
+// steps: R rounds of whole tiles (one per SM each), then the remaining tiles
+// in ns parts, dealt round-robin.  A unit also pays a fixed setup cost, larger
+// for split tiles (the part record and the merge), from per-unit timings of
+// the kernel on GB300.
+MlpSplit tc_mlp_split(const TcModel &m, int Q, int max_split) {
+    constexpr double SETUP_WHOLE = 0.7, SETUP_SPLIT = 2.5;   // in deployment steps
+    const int ntiles = (Q + BM - 1) / BM, sms = g_num_sms > 0 ? g_num_sms : 1, D = m.D;
+    MlpSplit best{0, 1};
     double best_cost = 1e300;
-    for (int ns = 1; ns <= 8 && ns <= m.D; ++ns) {
-        const long units = (long)ntiles * ns;
-        const double cost = (double)((units + sms - 1) / sms) * ((m.D + ns - 1) / ns + 0.5);
-        if (cost < best_cost - 1e-9) {
-            best_cost = cost;
-            best = ns;
+    long best_units = 0;
+    for (int R = 0; R * sms <= ntiles; ++R) {
+        const int nwhole = R * sms, ntail = ntiles - nwhole;
+        for (int ns = 1; ns <= max_split && ns <= D; ++ns) {
+            if (ntail == 0 && ns > 1) break;
+            const long tail_units = (long)ntail * ns, units = nwhole + tail_units;
+            if (units == 0) continue;
+            const long grid = units < sms ? units : sms;
+            const double per = ns > 1 ? (double)((D + ns - 1) / ns) + SETUP_SPLIT : D + SETUP_WHOLE;
+            const double cost = R * (D + SETUP_WHOLE) + (double)((tail_units + grid - 1) / grid) * per;
+            if (cost < best_cost - 1e-9 || (cost < best_cost + 1e-9 && units < best_units)) {
+                best_cost = cost;
+                best = MlpSplit{nwhole, ns};
+                best_units = units;
+            }
         }
     }
     return best;
 }
 
-cudaError_t launch_mlp_tc(const TcModel &m, const Queries &q, const float *qual, int nsplit,
-                          void *part, int32_t *count, int32_t *status, cudaStream_t s) {
+cudaError_t launch_mlp_tc(const TcModel &m, const Queries &q, const float *qual,
+                          const MlpSplit &sp, void *part, int32_t *count, int32_t *status,
+                          cudaStream_t s) {
     if (q.Q <= 0) return cudaSuccess;
-    const long units = (long)((q.Q + BM - 1) / BM) * nsplit;
+    const int ntiles = (q.Q + BM - 1) / BM;
+    if (sp.nwhole < 0 || sp.nwhole > ntiles || sp.nsplit < 1) return cudaErrorInvalidValue;
+    const long units = sp.nwhole + (long)(ntiles - sp.nwhole) * sp.nsplit;
     const int grid = units < g_num_sms ? (int)units : g_num_sms;
     const MlpLayout L = mlp_layout(m.H1, m.H2, m.Mpad, m.D, !mlp_fixed_h2(m.H2));
     const HeadConsts &hc = *m.head;
@@ -916,7 +950,8 @@ cudaError_t launch_mlp_tc(const TcModel &m, const Queries &q, const float *qual,
     cfg.attrs = at;
     cfg.numAttrs = 1;
 #define HWR_MLP(H2T, NHT) \
-    return cudaLaunchKernelEx(&cfg, k_mlp_tc<H2T, NHT>, m, q, hc, qual, nsplit, pt, count, status)
+    return cudaLaunchKernelEx(&cfg, k_mlp_tc<H2T, NHT>, m, q, hc, qual, sp.nwhole, sp.nsplit, pt, \
+                              count, status)
     if (m.NH == 3) {
         if (m.H2 == 256) HWR_MLP(256, 3);
         if (m.H2 == 128) HWR_MLP(128, 3);
