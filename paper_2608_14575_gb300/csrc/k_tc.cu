@@ -191,9 +191,6 @@ k_qual_tc(const __grid_constant__ CUtensorMap tmap, TcModel m, int Q, float *qua
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int nch = m.Epad / KCH, ntiles = (Q + BM - 1) / BM, Mpad = m.Mpad;
     const uint32_t membytes = (uint32_t)Mpad * m.Epad * 2;
-    // the predictor kernel that follows may start now: only its epilogue reads
-    // this kernel's output, and it waits for this grid's completion first
-    grid_launch_dependents();
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < QUAL_STAGES; ++s) {
@@ -217,6 +214,12 @@ k_qual_tc(const __grid_constant__ CUtensorMap tmap, TcModel m, int Q, float *qua
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tslot;
+    // Launched as a programmatic dependent of the kernel before it on the
+    // stream: the set-up above may overlap that kernel's last CTAs, nothing
+    // below may.  Only then may the predictor kernel that follows start (it
+    // reads inputs early, and only its epilogue waits for this grid).
+    grid_dependency_wait();
+    grid_launch_dependents();
 
     if (warp == 0 && lane == 0) {
         // producer: model embeddings once, then query tiles chunk by chunk
@@ -477,6 +480,9 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
         tmem_alloc(tslot, tcols);
         tmem_relinquish();
     }
+    // the next route's quality kernel may be scheduled now: it waits for this
+    // grid's completion before it touches memory
+    grid_launch_dependents();
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -881,8 +887,19 @@ cudaError_t launch_qual_tc(const TcModel &m, const Queries &q, float *qual, int3
     const int ntiles = (q.Q + BM - 1) / BM;
     const int grid = ntiles < g_num_sms ? ntiles : g_num_sms;
     const QualLayout L = qual_layout(m.Mpad, m.Epad);
-    k_qual_tc<<<grid, QUAL_THREADS, L.total, s>>>(map, m, q.Q, qual, status);
-    return cudaGetLastError();
+    // programmatic dependent launch: CTAs are set up while the kernel before
+    // finishes, then wait for it (griddepcontrol.wait) before any memory access
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.gridDim = dim3((unsigned)grid);
+    cfg.blockDim = dim3(QUAL_THREADS);
+    cfg.dynamicSmemBytes = L.total;
+    cfg.stream = s;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, k_qual_tc, map, m, q.Q, qual, status);
 }
 
 cudaError_t launch_mlp_tc_scores(const TcModel &m, const Queries &q, const float *qual,
