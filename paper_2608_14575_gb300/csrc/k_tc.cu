@@ -884,8 +884,11 @@ cudaError_t launch_qual_tc(const TcModel &m, const Queries &q, float *qual, int3
                           CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                           CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
+    // as many CTAs as give every CTA the same number of tiles (512 tiles on
+    // 152 SMs: 128 CTAs of 4 tiles, not 152 with a last round on 56)
     const int ntiles = (q.Q + BM - 1) / BM;
-    const int grid = ntiles < g_num_sms ? ntiles : g_num_sms;
+    const int rounds = (ntiles + g_num_sms - 1) / g_num_sms;
+    const int grid = (ntiles + rounds - 1) / rounds;
     const QualLayout L = qual_layout(m.Mpad, m.Epad);
     // programmatic dependent launch: CTAs are set up while the kernel before
     // finishes, then wait for it (griddepcontrol.wait) before any memory access
