@@ -31,7 +31,7 @@ Printed (one JSON line, rank 0):
             p50 of calls queued back to back, queries/s at that median, and the
             fraction of the bf16 tensor roofline.
 --impl reference times the CPU oracle (the reference arm for this build).
---online prints the online evaluation metrics of Sec. 4.3 (SLO attainment,
+--online prints the online evaluation metrics of Sec. 4.4 (SLO attainment,
 queue composition, load/running/waiting skew) for the online sequential
 workload's shapes under each arrival pattern, for the hardware-aware router
 and for the frozen-snapshot static-cost mode, one JSON line each, with the

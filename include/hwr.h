@@ -205,7 +205,7 @@ hwr_status hwr_route_batch(hwr_ctx *ctx, int32_t Q, const float *in_len,
                            float *pred_latency, float *utility);
 
 /*
- * Per-query latency budgets (HW-Router Sec. 4.3, Eq. 4-5).  The paper's SLO
+ * Per-query latency budgets (HW-Router Sec. 4.4, Eq. 4-5).  The paper's SLO
  * for a request with p input tokens and d output tokens is
  * TTFT_SLO(p) + d * TPOT_SLO with TTFT_SLO(p) = slack * (a + b p); routing
  * uses the query's expected output length for d.

@@ -272,7 +272,7 @@ int orc_select(int D, const double *C, const double *U, double slo, int mode)
     return best;
 }
 
-/* ---- per-query latency budget (Sec. 4.3, Eq. 4-5) ---------------------- */
+/* ---- per-query latency budget (Sec. 4.4, Eq. 4-5) ---------------------- */
 
 /* SLO budget of a query with p input tokens and d expected output tokens:
  * TTFT_SLO(p) = slack * (a + b p) and the request meets the SLO when its

@@ -96,7 +96,7 @@ struct Lambdas {
 };
 
 #ifdef __CUDACC__
-// Budget B of query `row` (Sec. 4.3, Eq. 4-5 for the model form):
+// Budget B of query `row` (Sec. 4.4, Eq. 4-5 for the model form):
 // t = fma(b, p, a); s = slack * t; B = fma(tpot_slo, d, s).
 __device__ __forceinline__ float query_budget(const Queries &q, int row) {
     if (q.slo_mode == 1) return q.slo_q[row];

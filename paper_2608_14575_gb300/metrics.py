@@ -1,4 +1,4 @@
-"""Online routing metrics of HW-Router's evaluation (Sec. 4.3, Eq. 6).
+"""Online routing metrics of HW-Router's evaluation (Sec. 4.4, Eq. 6).
 
 Host-side reductions over a trace of routed requests and of queue snapshots
 sampled at each micro-batch (the monitor's view when decisions are made):

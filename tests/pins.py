@@ -520,7 +520,7 @@ def check_three_heads(lib):
 
 
 # ---------------------------------------------------------------------------
-# per-query SLO budgets (Sec. 4.3, Eq. 4-5)
+# per-query SLO budgets (Sec. 4.4, Eq. 4-5)
 
 def check_slo_budget(lib):
     # TTFT_SLO(p) = slack (a + b p); budget = TTFT_SLO(p) + d TPOT_SLO

@@ -1,4 +1,4 @@
-"""Online routing on the GPU against the oracle (Sec. 4.3 evaluation metrics).
+"""Online routing on the GPU against the oracle (Sec. 4.4 evaluation metrics).
 
 The serving world (workload/serve.py) is driven once by the library (routing
 and hwr_score_batch through the C ABI) and once by the oracle in canonical

@@ -1,5 +1,5 @@
 """Online evaluation on the CPU: arrival patterns, micro-batching, the serving
-world's dynamics and the paper's online metrics (Sec. 4.3, Eq. 6).
+world's dynamics and the paper's online metrics (Sec. 4.4, Eq. 6).
 
 Metrics are pinned by hand-computed examples; arrival patterns by their
 defining statistics and by reductions to one another; the world by

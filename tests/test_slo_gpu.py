@@ -1,4 +1,4 @@
-"""Per-query SLO budgets (HW-Router Sec. 4.3, Eq. 4-5) on the GPU.
+"""Per-query SLO budgets (HW-Router Sec. 4.4, Eq. 4-5) on the GPU.
 
 hwr_route_batch_slo takes one budget per query, or the paper's SLO model
 B_q = slack * (a + b * p_q) + d_q * TPOT_SLO evaluated on the device.  The

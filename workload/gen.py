@@ -7,7 +7,7 @@ arrival/drain process.  It holds none of the routing method's arithmetic
 CPU oracle and the CUDA library can both be fed from it without sharing code.
 
 The paper's workloads (MixInstruct short prompts mixed with LongBench long
-contexts, Sec. 4 "Dataset"; vLLM-observed runtime signals, Table 2) are not
+contexts, Sec. 4.3 "Dataset"; vLLM-observed runtime signals, Table 2) are not
 available here; the distributions below stand in for them.
 
 Conventions

@@ -1,13 +1,13 @@
 """Synthetic serving world for online routing experiments.
 
-The paper evaluates routers on live vLLM servers (Sec. 4.3, Sec. 5); here the
+The paper evaluates routers on live vLLM servers (Sec. 4.4, Sec. 5); here the
 servers are replaced by a seeded stand-in that evolves the per-deployment
 hardware snapshot between micro-batches.  Nothing in this module computes any
 part of the routing method: it draws arrivals, groups them into micro-batches,
 hands each batch to caller-supplied routing and scoring functions and moves
 the world on with their choices.
 
-Arrival patterns (Sec. 4.3 load generator):
+Arrival patterns (Sec. 4.5 load generator):
   * "poisson"            exponential gaps with mean 1/rate;
   * "micro_burst"        Poisson whose rate is burst_factor x higher during
                          the first burst_len seconds of every period;
