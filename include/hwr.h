@@ -183,7 +183,12 @@ hwr_status hwr_get_snapshot(hwr_ctx *ctx, int32_t *running_out);
  * next call on the context or by hwr_synchronize.  When earlier work is still
  * queued on the stream -- after an HWR_ASYNC call, or the caller's own work on
  * a stream it passed to hwr_create -- the call synchronises the stream
- * instead of waiting on the outputs).  Pinned host memory gives the full
+ * instead of waiting on the outputs).  Where the GPU can read and write
+ * pageable host memory (cudaDevAttrPageableMemoryAccess, e.g. Grace + GB300
+ * over the coherent CPU-GPU link), such small synchronous calls use the
+ * caller's arrays directly: the kernels read the inputs and write the outputs
+ * there, so the arrays must stay untouched until the call returns.  Pinned
+ * host memory gives the full
  * link bandwidth.  With HWR_DEVICE_PTRS they are device pointers read and
  * written in stream order.  With HWR_ASYNC the call returns after enqueueing;
  * host arrays must then stay valid until hwr_synchronize().

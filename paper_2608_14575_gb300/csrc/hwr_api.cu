@@ -67,6 +67,10 @@ struct hwr_ctx {
     int device = -1;             // the CUDA device current at hwr_create
     long poll_us = 1000000;      // small-batch output poll limit (HWR_TEST_POLL_US)
     bool async_pending = false;  // an HWR_ASYNC call may still have work queued
+    // the GPU reads and writes pageable host memory coherently (address
+    // translation services over the CPU-GPU link, as on Grace + GB300):
+    // small synchronous calls then use the caller's arrays directly
+    bool ats = false;
     std::vector<uint8_t> xform_h;   // feature transforms (host copy, snapshot checks)
     std::string err;
     AllocHook hook;
@@ -574,6 +578,16 @@ extern "C" hwr_status hwr_create(const hwr_deployment_table *table, const hwr_pr
     }
     if (const char *h = getenv("HWR_TEST_FAIL_ALLOC")) c->hook.fail_at = atol(h);
     if (const char *h = getenv("HWR_TEST_POLL_US")) c->poll_us = atol(h) < 0 ? 0 : atol(h);
+    {
+        int pageable = 0;
+        if (cudaDeviceGetAttribute(&pageable, cudaDevAttrPageableMemoryAccess, c->device) !=
+            cudaSuccess) {
+            cudaGetLastError();
+            pageable = 0;
+        }
+        const char *h = getenv("HWR_TEST_NO_ATS");   // test hook: force the staging copies
+        c->ats = pageable == 1 && !(h && atoi(h) != 0);
+    }
     if (const char *h = getenv("HWR_TEST_STALL")) c->test_stall = atoi(h) != 0;
     if (const char *h = getenv("HWR_TC_MIN_PAIRS")) c->tc_min_pairs = atoi(h) > 1 ? atoi(h) : 1;
     if (const char *h = getenv("HWR_PAIRS_MAX_PAIRS"))
@@ -856,13 +870,17 @@ static hwr_status route_impl(hwr_ctx *c, int32_t Q, const float *in_len, const f
     // a small synchronous call for the small-batch kernel or the SIMT
     // sequential kernels: they read the inputs from the mapped staging itself
     // with plain loads (no host-to-device copy)
-    const bool zero_copy = packed && !tensor && !ml && !so && c->pin_d &&
+    const bool zero_copy = packed && !tensor && !ml && !so && (c->pin_d || c->ats) &&
                            (seq ? !(flags & HWR_PATH_TENSOR) : (long)Q * c->D <= c->pairs_max);
     // ... and on the small-batch kernel the host waits for the outputs
     // themselves instead of synchronising the stream
     // ... unless work queued earlier on the stream (an HWR_ASYNC call, or the
     // caller's own work on a stream it passed in) is still running: then
     // the kernel starts late and the host synchronises instead of spinning
+    // ... and where the GPU reaches pageable host memory, from the caller's
+    // own arrays: the kernels read the inputs and write the outputs there
+    // (plain element loads and stores), with no staging copy either way
+    const bool direct = zero_copy && c->ats;
     bool poll = zero_copy && !seq && c->poll_us > 0;
     if (poll && (c->async_pending || !c->own_stream)) {
         const cudaError_t e = cudaStreamQuery(c->stream);
@@ -884,6 +902,17 @@ static hwr_status route_impl(hwr_ctx *c, int32_t Q, const float *in_len, const f
             q.lat = (float *)(c->out_d + o_lat);
             q.util = (float *)(c->out_d + o_util);
         }
+    } else if (direct) {
+        q.inputs_host = 1;
+        q.emb = q_emb;
+        q.in_len = in_len;
+        q.out_len = out_len;
+        if (budgets) q.slo_q = spec->budget;
+        q.chosen = chosen;
+        q.lat = pred_latency;
+        q.util = utility;
+        if (poll)
+            for (int i = 0; i < Q; ++i) chosen[i] = OUT_PENDING;
     } else {
         TRY(grow(c, &c->io_d, &c->io_cap, in_total));
         TRY(grow(c, &c->out_d, &c->out_cap, out_total));
@@ -1020,7 +1049,12 @@ static hwr_status route_impl(hwr_ctx *c, int32_t Q, const float *in_len, const f
             CK(c, cudaMemcpyAsync(so->quality, SQ, (size_t)Q * rowQ, cudaMemcpyDeviceToHost,
                                   c->stream), "copy quality");
     } else if (!dev) {
-        if (packed) {
+        if (direct) {
+            // outputs are already in the caller's arrays once the kernel wrote them
+            if (!(poll && wait_chosen(chosen, Q, c->poll_us)))
+                CK(c, cudaStreamSynchronize(c->stream), "synchronize");
+            synced = true;
+        } else if (packed) {
             const char *ob = c->pin_h + align_up(in_total, 256);
             CK(c, cudaEventRecord(c->pin_ev, c->stream), "record");
             if (!(poll && wait_chosen((const int32_t *)ob, Q, c->poll_us)))

@@ -55,3 +55,24 @@ def test_small_call_queued_behind_an_async_route():
     # with the stream idle again, the next small call takes the fast path
     _exact(r.route(p["in_len"][:4], p["out_len"][:4], p["emb"][:4]), W.query_slice(p, 0, 4))
     r.close()
+
+
+@pytest.mark.parametrize("no_ats", ["0", "1"])
+def test_staged_and_direct_host_paths_agree(monkeypatch, no_ats):
+    """Where the GPU reaches pageable host memory (address translation over the
+    CPU-GPU link), small synchronous calls read the caller's arrays and write
+    its outputs directly; HWR_TEST_NO_ATS=1 forces the pinned staging copies.
+    Both give the oracle's canonical results, batch and sequential."""
+    monkeypatch.setenv("HWR_TEST_NO_ATS", no_ats)
+    p = W.make_config(4, Q=8)
+    r = H.Router(p)
+    _exact(r.route(), p)
+    r.close()
+    p = W.make_config(2, Q=64)
+    r = H.Router(p)
+    got = r.route(flags=H.HWR_SEQUENTIAL)
+    want = O.Problem(p).route(mode=O.F32, sequential=True)
+    assert np.array_equal(got[0], want[0])
+    assert np.array_equal(got[1], want[1].astype(np.float32))
+    assert np.array_equal(r.get_snapshot(), want[3])
+    r.close()
