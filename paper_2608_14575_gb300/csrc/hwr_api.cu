@@ -106,7 +106,9 @@ struct hwr_ctx {
     cudaEvent_t snap_ev = nullptr;
 
     // grow-only scratch
-    float *qual = nullptr;   size_t qual_cap = 0;     // [Q][Mpad]
+    float *qual = nullptr;   size_t qual_cap = 0;     // 2 x [Q][Mpad], alternating per call
+    float *qual_last = nullptr;                       // the buffer the last quality kernel wrote
+    int qual_flip = 0;
     char *part = nullptr;    size_t part_cap = 0;     // split-deployment partials
     int32_t *count = nullptr; size_t count_cap = 0;   // per-row arrivals (self-resetting)
     float *pairC = nullptr;  float *pairQ = nullptr;  int32_t *pairN = nullptr;  // small batches
@@ -679,7 +681,7 @@ static hwr_status run_kernels(hwr_ctx *c, const Queries &q, uint32_t flags, bool
             const size_t Dv = (size_t)c->D * (Qs + 1);
             TRY(grow(c, &c->prebf, &c->prebf_cap, Dv * c->H1));
             TRY(grow(c, &c->dmv, &c->dmv_cap, Dv));
-            TRY(grow(c, &c->qual, &c->qual_cap, (size_t)Qs * c->Mpad));
+            TRY(grow(c, &c->qual, &c->qual_cap, 2 * (size_t)Qs * c->Mpad));
         }
         TRY(grow(c, &c->ctab, &c->ctab_cap, seq_table_floats(c->D, Qs)));
         TRY(grow(c, &c->qseq, &c->qseq_cap, seq_aux_floats(c->D, c->M, c->H1, Qs)));
@@ -717,11 +719,15 @@ static hwr_status run_kernels(hwr_ctx *c, const Queries &q, uint32_t flags, bool
                 LaunchScope a(c, HWR_K_SEQ_TABLE, prof);
                 CK(c, launch_seq_prep_tc(m, k, n, c->qseq, c->prebf, c->dmv, c->stream),
                    "sequential preparation");
-                CK(c, launch_qual_tc(t, k, c->qual, c->status_d, c->stream), "quality kernel");
-                CK(c, launch_mlp_tc_scores(tv, kt, c->qual, c->status_d, c->stream),
+                // fixed halves of the buffer (calls of different sizes must not
+                // overlap the half the previous call's kernels still read)
+                float *qb = c->qual + (c->qual_flip ? c->qual_cap / 2 : 0);
+                c->qual_flip ^= 1;
+                CK(c, launch_qual_tc(t, k, qb, c->status_d, c->stream, true), "quality kernel");
+                CK(c, launch_mlp_tc_scores(tv, kt, qb, c->status_d, c->stream),
                    "sequential table (tensor cores)");
                 a.done();
-                CK(c, launch_seq_chain_tc(m, k, n, c->ctab, c->qseq, c->qual, c->Mpad, c->stream),
+                CK(c, launch_seq_chain_tc(m, k, n, c->ctab, c->qseq, qb, c->Mpad, c->stream),
                    "sequential chain");
                 // preparation, quality and chain beside the scope's table kernel
                 c->stats.kernel_launches += 3;
@@ -741,7 +747,12 @@ static hwr_status run_kernels(hwr_ctx *c, const Queries &q, uint32_t flags, bool
     }
     if (tensor) {
         const TcModel t = tc_view(c);
-        TRY(grow(c, &c->qual, &c->qual_cap, (size_t)q.Q * c->Mpad));
+        TRY(grow(c, &c->qual, &c->qual_cap, 2 * (size_t)q.Q * c->Mpad));
+        // the two halves alternate, so this call's quality kernel may run
+        // alongside the previous call's predictor, which reads the other
+        float *qb = c->qual + (c->qual_flip ? c->qual_cap / 2 : 0);
+        c->qual_flip ^= 1;
+        c->qual_last = qb;
         const MlpSplit sp = tc_mlp_split(t, q.Q);
         if (sp.nsplit > 1) {
             TRY(grow(c, &c->part, &c->part_cap, (size_t)sp.nsplit * q.Q * 16));
@@ -751,10 +762,10 @@ static hwr_status run_kernels(hwr_ctx *c, const Queries &q, uint32_t flags, bool
             }
         }
         LaunchScope a(c, HWR_K_QUAL_TC, prof);
-        CK(c, launch_qual_tc(t, q, c->qual, c->status_d, c->stream), "quality kernel");
+        CK(c, launch_qual_tc(t, q, qb, c->status_d, c->stream, true), "quality kernel");
         a.done();
         LaunchScope b(c, HWR_K_MLP_TC, prof);
-        CK(c, launch_mlp_tc(t, q, c->qual, sp, c->part, c->count, c->status_d, c->stream),
+        CK(c, launch_mlp_tc(t, q, qb, sp, c->part, c->count, c->status_d, c->stream),
            "predictor kernel");
         b.done();
         return HWR_OK;
@@ -987,7 +998,7 @@ static hwr_status route_impl(hwr_ctx *c, int32_t Q, const float *in_len, const f
             CK(c, cudaMemcpyAsync(SQ + (size_t)lo * c->M, c->pairQ, n * rowQ,
                                   cudaMemcpyDeviceToDevice, c->stream), "copy quality");
         if (tensor && SQ)
-            CK(c, cudaMemcpy2DAsync(SQ + (size_t)lo * c->M, rowQ, c->qual, (size_t)c->Mpad * 4,
+            CK(c, cudaMemcpy2DAsync(SQ + (size_t)lo * c->M, rowQ, c->qual_last, (size_t)c->Mpad * 4,
                                     rowQ, n, cudaMemcpyDeviceToDevice, c->stream),
                "copy quality");
         if (!ml) return HWR_OK;
@@ -1213,7 +1224,8 @@ hwr_status hwr_internal_route_tensor_scratch(hwr_ctx *c, int32_t Q, const float 
     const MlpSplit sp = tc_mlp_split(t, Q, max_split);
     if (sp.nsplit > 1)
         CK(c, cudaMemsetAsync(count, 0, (size_t)Q * sizeof(int32_t), c->stream), "clear counters");
-    CK(c, launch_qual_tc(t, q, qual, c->status_d, c->stream), "quality kernel");
+    // one static quality buffer: a plain launch, ordered after the kernel before
+    CK(c, launch_qual_tc(t, q, qual, c->status_d, c->stream, false), "quality kernel");
     c->stats.kernel_launches++;
     c->stats.launches[HWR_K_QUAL_TC]++;
     CK(c, launch_mlp_tc(t, q, qual, sp, part, count, c->status_d, c->stream), "predictor kernel");

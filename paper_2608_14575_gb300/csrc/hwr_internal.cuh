@@ -181,8 +181,11 @@ void tc_build_w2img(const uint16_t *W2, int H1, int H2, uint16_t *img);
 void tc_build_membimg(const uint16_t *memb_EM, int E, int M, int Mpad, int Epad,
                       uint16_t *img);
 // qual: scratch [Q][Mpad] fp32.  status: device int32 word.
+// dependent: launched as a programmatic dependent of the kernel before it on
+// the stream, running alongside it -- only when that kernel does not read
+// `qual` (the context alternates two quality buffers between calls).
 cudaError_t launch_qual_tc(const TcModel &m, const Queries &q, float *qual,
-                           int32_t *status, cudaStream_t s);
+                           int32_t *status, cudaStream_t s, bool dependent);
 // The first nwhole query tiles are processed whole; the deployments of each
 // remaining tile are split over nsplit units.  With nsplit > 1, `part`
 // (nsplit * Q records of 16 bytes) and `count` (Q int32, zero, self-resetting)

@@ -215,11 +215,12 @@ k_qual_tc(const __grid_constant__ CUtensorMap tmap, TcModel m, int Q, float *qua
     tc_fence_after();
     const uint32_t tmem = *tslot;
     // Launched as a programmatic dependent of the kernel before it on the
-    // stream: the set-up above may overlap that kernel's last CTAs, nothing
-    // below may.  Only then may the predictor kernel that follows start (it
-    // reads inputs early, and only its epilogue waits for this grid).
-    grid_dependency_wait();
-    grid_launch_dependents();
+    // stream (normally the previous route's predictor): this grid reads only
+    // the query embeddings, which were complete before that kernel began, and
+    // writes its own quality buffer (two alternate between calls), so it runs
+    // alongside that kernel.  It waits for that kernel's completion only at
+    // the end, before it lets the predictor of its own call start: that
+    // predictor's outputs and scratch are then ordered after the previous one.
 
     if (warp == 0 && lane == 0) {
         // producer: model embeddings once, then query tiles chunk by chunk
@@ -312,6 +313,8 @@ k_qual_tc(const __grid_constant__ CUtensorMap tmap, TcModel m, int Q, float *qua
     }
     tc_fence_before();
     __syncthreads();
+    grid_dependency_wait();
+    grid_launch_dependents();
     if (warp == 1) {
         __syncwarp();
         tc_fence_after();
@@ -872,7 +875,7 @@ cudaError_t tc_prepare() {
 }
 
 cudaError_t launch_qual_tc(const TcModel &m, const Queries &q, float *qual, int32_t *status,
-                           cudaStream_t s) {
+                           cudaStream_t s, bool dependent) {
     if (q.Q <= 0) return cudaSuccess;
     CUtensorMap map;
     const cuuint64_t dims[2] = {(cuuint64_t)m.E, (cuuint64_t)q.Q};
@@ -890,8 +893,9 @@ cudaError_t launch_qual_tc(const TcModel &m, const Queries &q, float *qual, int3
     const int rounds = (ntiles + g_num_sms - 1) / g_num_sms;
     const int grid = (ntiles + rounds - 1) / rounds;
     const QualLayout L = qual_layout(m.Mpad, m.Epad);
-    // programmatic dependent launch: CTAs are set up while the kernel before
-    // finishes, then wait for it (griddepcontrol.wait) before any memory access
+    // programmatic dependent launch (when `qual` is not read by the kernel
+    // before it): the grid runs alongside that kernel and waits for it at
+    // its end
     cudaLaunchConfig_t cfg = {};
     cudaLaunchAttribute at[1];
     at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -901,7 +905,7 @@ cudaError_t launch_qual_tc(const TcModel &m, const Queries &q, float *qual, int3
     cfg.dynamicSmemBytes = L.total;
     cfg.stream = s;
     cfg.attrs = at;
-    cfg.numAttrs = 1;
+    cfg.numAttrs = dependent ? 1 : 0;
     return cudaLaunchKernelEx(&cfg, k_qual_tc, map, m, q.Q, qual, status);
 }
 
