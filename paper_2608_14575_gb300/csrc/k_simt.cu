@@ -735,6 +735,9 @@ __device__ __forceinline__ uint64_t cand_key(float C, float U, int d, float slo)
     return ((uint64_t)cls << 38) | ((uint64_t)key << 6) | (uint64_t)(63 - d);
 }
 
+// HI: deployments 32 .. 63 exist (D > 32); without them every lane of the
+// walk carries one deployment and the second half of the step is compiled out.
+template <bool HI>
 __global__ void __launch_bounds__(CHAIN_THREADS)
 k_seq_chain(Model m, Queries q, int Qs, const float *ctab, float *aux, const float *qsrc,
             int qstride) {
@@ -781,7 +784,7 @@ k_seq_chain(Model m, Queries q, int Qs, const float *ctab, float *aux, const flo
         // (two reductions) and the winner's index from the low bits.
         const unsigned full = 0xffffffffu;
         const int d0 = lane, d1 = lane + 32;
-        const bool h0 = d0 < D, h1 = d1 < D;
+        const bool h0 = d0 < D, h1 = HI && d1 < D;
         const int m0 = h0 ? dm[d0] : 0, m1 = h1 ? dm[d1] : 0;
         const float lam = q.lam, wq = q.wq;
         int c0 = 0, c1 = 0;
@@ -832,7 +835,7 @@ k_seq_chain(Model m, Queries q, int Qs, const float *ctab, float *aux, const flo
                 }
             }
             // step i: the warp's largest key
-            const uint64_t kl = K0 > K1 ? K0 : K1;
+            const uint64_t kl = HI && K1 > K0 ? K1 : K0;
             const uint32_t hi = __reduce_max_sync(full, (uint32_t)(kl >> 32));
             const uint32_t lo =
                 __reduce_max_sync(full, (uint32_t)(kl >> 32) == hi ? (uint32_t)kl : 0u);
@@ -1248,7 +1251,8 @@ cudaError_t simt_prepare() {
     if (e == cudaSuccess) e = opt_in(k_seq_table<2>, big);
     if (e == cudaSuccess) e = opt_in(k_seq_table<4>, big);
     if (e == cudaSuccess) e = opt_in(k_seq_table<8>, big);
-    if (e == cudaSuccess) e = opt_in(k_seq_chain, SEQ_CHAIN_SMEM + 1024);
+    if (e == cudaSuccess) e = opt_in(k_seq_chain<false>, SEQ_CHAIN_SMEM + 1024);
+    if (e == cudaSuccess) e = opt_in(k_seq_chain<true>, SEQ_CHAIN_SMEM + 1024);
     if (e == cudaSuccess) e = opt_in(k_route_pairs, big);
     return e;
 }
@@ -1350,7 +1354,9 @@ cudaError_t launch_seq_chain(const Model &m, const Queries &q, int Qs, const flo
                              float *aux, cudaStream_t s) {
     cudaLaunchConfig_t cfg = dependent_launch(1, CHAIN_THREADS, chain_smem(m.D, m.M, Qs), s);
     const SeqAux A = seq_aux(aux, m.D, m.M, Qs);
-    return cudaLaunchKernelEx(&cfg, k_seq_chain, m, q, Qs, ctab, aux, (const float *)A.qual, m.M);
+    if (m.D > 32)
+        return cudaLaunchKernelEx(&cfg, k_seq_chain<true>, m, q, Qs, ctab, aux, (const float *)A.qual, m.M);
+    return cudaLaunchKernelEx(&cfg, k_seq_chain<false>, m, q, Qs, ctab, aux, (const float *)A.qual, m.M);
 }
 
 cudaError_t launch_seq_prep_tc(const Model &m, const Queries &q, int Qs, float *aux,
@@ -1363,7 +1369,8 @@ cudaError_t launch_seq_prep_tc(const Model &m, const Queries &q, int Qs, float *
 cudaError_t launch_seq_chain_tc(const Model &m, const Queries &q, int Qs, const float *ctab,
                                 float *aux, const float *qual, int qstride, cudaStream_t s) {
     cudaLaunchConfig_t cfg = dependent_launch(1, CHAIN_THREADS, chain_smem(m.D, m.M, Qs), s);
-    return cudaLaunchKernelEx(&cfg, k_seq_chain, m, q, Qs, ctab, aux, qual, qstride);
+    if (m.D > 32) return cudaLaunchKernelEx(&cfg, k_seq_chain<true>, m, q, Qs, ctab, aux, qual, qstride);
+    return cudaLaunchKernelEx(&cfg, k_seq_chain<false>, m, q, Qs, ctab, aux, qual, qstride);
 }
 
 }  // namespace hwr
