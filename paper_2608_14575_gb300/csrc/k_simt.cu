@@ -781,28 +781,31 @@ k_seq_chain(Model m, Queries q, int Qs, const float *ctab, float *aux, const flo
         // While step i is decided, step i + 1's entries at the current count
         // and at one more pick are loaded and turned into candidate keys, so a
         // step is a choice between two ready keys, a 64-bit max over the warp
-        // (two reductions) and the winner's index from the low bits.
+        // (two reductions) and the winner's index from the low bits.  Lanes
+        // without a deployment shadow deployment D - 1 (valid addresses, no
+        // divergent branches) and keep key 0, below every candidate; the row
+        // of one more pick advances by D (Qs - c) - d - 1 after a pick.
         const unsigned full = 0xffffffffu;
         const int d0 = lane, d1 = lane + 32;
         const bool h0 = d0 < D, h1 = HI && d1 < D;
-        const int m0 = h0 ? dm[d0] : 0, m1 = h1 ? dm[d1] : 0;
+        const int e0 = h0 ? d0 : D - 1, e1 = h1 ? d1 : D - 1;
+        const int m0 = dm[e0], m1 = HI ? dm[e1] : 0;
         const float lam = q.lam, wq = q.wq;
         int c0 = 0, c1 = 0;
-        int r0 = h0 ? tab_row(D, Qs, 0, d0) : 0, r1 = h1 ? tab_row(D, Qs, 0, d1) : 0;
+        int r0 = tab_row(D, Qs, 0, e0), r1 = HI ? tab_row(D, Qs, 0, e1) : 0;
+        int r0p = r0 + D * Qs - e0 - 1, r1p = HI ? r1 + D * Qs - e1 - 1 : 0;
         // this step's candidate of each deployment: cost, utility, key
-        float C0 = 0.f, U0 = 0.f, C1 = 0.f, U1 = 0.f;
-        uint64_t K0 = 0, K1 = 0;
+        float C0, U0, C1 = 0.f, U1 = 0.f;
+        uint64_t K0, K1 = 0;
         {
             const float b = slo[0];
-            if (h0) {
-                C0 = tab[r0];
-                U0 = __fmaf_rn(-lam, C0, __fmul_rn(wq, qs[m0]));
-                K0 = cand_key(C0, U0, d0, b);
-            }
-            if (h1) {
+            C0 = tab[r0];
+            U0 = __fmaf_rn(-lam, C0, __fmul_rn(wq, qs[m0]));
+            K0 = h0 ? cand_key(C0, U0, d0, b) : 0;
+            if (HI) {
                 C1 = tab[r1];
                 U1 = __fmaf_rn(-lam, C1, __fmul_rn(wq, qs[m1]));
-                K1 = cand_key(C1, U1, d1, b);
+                K1 = h1 ? cand_key(C1, U1, d1, b) : 0;
             }
         }
         for (int i = 0; i < Qs; ++i) {
@@ -810,28 +813,23 @@ k_seq_chain(Model m, Queries q, int Qs, const float *ctab, float *aux, const flo
             float C0s = 0.f, U0s = 0.f, C0p = 0.f, U0p = 0.f;
             float C1s = 0.f, U1s = 0.f, C1p = 0.f, U1p = 0.f;
             uint64_t K0s = 0, K0p = 0, K1s = 0, K1p = 0;
-            int r0p = 0, r1p = 0;
             if (i + 1 < Qs) {
                 const float b = slo[i + 1];
-                if (h0) {
-                    const float wQ = __fmul_rn(wq, qs[(i + 1) * M + m0]);
-                    r0p = tab_row(D, Qs, c0 + 1, d0);
-                    C0s = tab[r0 + i + 1];
-                    C0p = tab[r0p + i + 1];
-                    U0s = __fmaf_rn(-lam, C0s, wQ);
-                    U0p = __fmaf_rn(-lam, C0p, wQ);
-                    K0s = cand_key(C0s, U0s, d0, b);
-                    K0p = cand_key(C0p, U0p, d0, b);
-                }
-                if (h1) {
-                    const float wQ = __fmul_rn(wq, qs[(i + 1) * M + m1]);
-                    r1p = tab_row(D, Qs, c1 + 1, d1);
+                const float wQ0 = __fmul_rn(wq, qs[(i + 1) * M + m0]);
+                C0s = tab[r0 + i + 1];
+                C0p = tab[r0p + i + 1];
+                U0s = __fmaf_rn(-lam, C0s, wQ0);
+                U0p = __fmaf_rn(-lam, C0p, wQ0);
+                K0s = h0 ? cand_key(C0s, U0s, d0, b) : 0;
+                K0p = h0 ? cand_key(C0p, U0p, d0, b) : 0;
+                if (HI) {
+                    const float wQ1 = __fmul_rn(wq, qs[(i + 1) * M + m1]);
                     C1s = tab[r1 + i + 1];
                     C1p = tab[r1p + i + 1];
-                    U1s = __fmaf_rn(-lam, C1s, wQ);
-                    U1p = __fmaf_rn(-lam, C1p, wQ);
-                    K1s = cand_key(C1s, U1s, d1, b);
-                    K1p = cand_key(C1p, U1p, d1, b);
+                    U1s = __fmaf_rn(-lam, C1s, wQ1);
+                    U1p = __fmaf_rn(-lam, C1p, wQ1);
+                    K1s = h1 ? cand_key(C1s, U1s, d1, b) : 0;
+                    K1p = h1 ? cand_key(C1p, U1p, d1, b) : 0;
                 }
             }
             // step i: the warp's largest key
@@ -841,30 +839,34 @@ k_seq_chain(Model m, Queries q, int Qs, const float *ctab, float *aux, const flo
                 __reduce_max_sync(full, (uint32_t)(kl >> 32) == hi ? (uint32_t)kl : 0u);
             const int wd = 63 - (int)(lo & 63u);
             const bool ok = (hi >> 6) >= 2u;    // class feasible or infeasible, not NaN
-            const bool p0 = ok && wd == d0, p1 = ok && wd == d1;
+            const bool p0 = ok && wd == d0, p1 = HI && ok && wd == d1;
+            if (lane == 0) o_ch[i] = ok ? wd : -1;
             if (p0 || p1) {
-                o_ch[i] = wd;
                 o_lat[i] = p0 ? C0 : C1;
                 o_util[i] = p0 ? U0 : U1;
-            } else if (!ok && lane == 0) {
-                o_ch[i] = -1;
+            }
+            if (!ok && lane == 0) {
                 o_lat[i] = __int_as_float(0x7fc00000);
                 o_util[i] = __int_as_float(0x7fc00000);
             }
             if (p0) {
                 ++c0;
                 r0 = r0p;
+                r0p += D * (Qs - c0) - e0 - 1;
             }
-            if (p1) {
+            if (HI && p1) {
                 ++c1;
                 r1 = r1p;
+                r1p += D * (Qs - c1) - e1 - 1;
             }
             C0 = p0 ? C0p : C0s;
             U0 = p0 ? U0p : U0s;
             K0 = p0 ? K0p : K0s;
-            C1 = p1 ? C1p : C1s;
-            U1 = p1 ? U1p : U1s;
-            K1 = p1 ? K1p : K1s;
+            if (HI) {
+                C1 = p1 ? C1p : C1s;
+                U1 = p1 ? U1p : U1s;
+                K1 = p1 ? K1p : K1s;
+            }
         }
         if (h0) cnt[d0] = c0;
         if (h1) cnt[d1] = c1;
