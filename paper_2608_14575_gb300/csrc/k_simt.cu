@@ -720,19 +720,17 @@ __host__ __device__ inline size_t chain_tab_floats(int D, int Qs) {
 // feasible candidate, smaller C for an infeasible one, as order-preserving
 // integers) and 63 - d (bits 0-5), so that the largest value is the best
 // candidate and ties go to the lowest deployment.  Same classes as make_cand.
+// Written with selects only: the walk is one warp's dependent chain, and a
+// divergent branch there costs more than the few extra instructions.
 __device__ __forceinline__ uint64_t cand_key(float C, float U, int d, float slo) {
-    uint32_t cls, key;
-    if (C != C) {
-        cls = 1u;
-        key = 1u;
-    } else if (C <= slo && U == U) {
-        cls = 3u;
-        key = order_key(U);
-    } else {
-        cls = 2u;
-        key = ~order_key(C);
-    }
-    return ((uint64_t)cls << 38) | ((uint64_t)key << 6) | (uint64_t)(63 - d);
+    const bool nan = C != C;
+    const bool feas = C <= slo && U == U;       // false for a NaN cost
+    const uint32_t kU = order_key(U), kC = ~order_key(C);
+    uint32_t key = feas ? kU : kC, cls = feas ? 3u : 2u;
+    key = nan ? 1u : key;
+    cls = nan ? 1u : cls;
+    const uint32_t hi = (cls << 6) | (key >> 26), lo = (key << 6) | (uint32_t)(63 - d);
+    return ((uint64_t)hi << 32) | lo;
 }
 
 // HI: deployments 32 .. 63 exist (D > 32); without them every lane of the
@@ -782,9 +780,11 @@ k_seq_chain(Model m, Queries q, int Qs, const float *ctab, float *aux, const flo
         // and at one more pick are loaded and turned into candidate keys, so a
         // step is a choice between two ready keys, a 64-bit max over the warp
         // (two reductions) and the winner's index from the low bits.  Lanes
-        // without a deployment shadow deployment D - 1 (valid addresses, no
-        // divergent branches) and keep key 0, below every candidate; the row
-        // of one more pick advances by D (Qs - c) - d - 1 after a pick.
+        // without a deployment shadow deployment D - 1 (valid addresses) and
+        // keep key 0, below every candidate; the row of one more pick advances
+        // by D (Qs - c) - d - 1 after a pick.  The step has no branch: the last
+        // step loads its own column again (valid entries, unused), and a pick
+        // moves the rows by selects.
         const unsigned full = 0xffffffffu;
         const int d0 = lane, d1 = lane + 32;
         const bool h0 = d0 < D, h1 = HI && d1 < D;
@@ -801,36 +801,39 @@ k_seq_chain(Model m, Queries q, int Qs, const float *ctab, float *aux, const flo
             const float b = slo[0];
             C0 = tab[r0];
             U0 = __fmaf_rn(-lam, C0, __fmul_rn(wq, qs[m0]));
-            K0 = h0 ? cand_key(C0, U0, d0, b) : 0;
+            K0 = cand_key(C0, U0, d0, b);
+            K0 = h0 ? K0 : 0;
             if (HI) {
                 C1 = tab[r1];
                 U1 = __fmaf_rn(-lam, C1, __fmul_rn(wq, qs[m1]));
-                K1 = h1 ? cand_key(C1, U1, d1, b) : 0;
+                K1 = cand_key(C1, U1, d1, b);
+                K1 = h1 ? K1 : 0;
             }
         }
         for (int i = 0; i < Qs; ++i) {
-            // step i + 1's candidates: s = same count, p = after one more pick
-            float C0s = 0.f, U0s = 0.f, C0p = 0.f, U0p = 0.f;
+            // step j = i + 1's candidates: s = same count, p = after one more
+            // pick (at the last step, j = i: this step's entries again)
+            const bool more = i + 1 < Qs;
+            const int j = more ? i + 1 : i;
+            const float b = slo[j];
+            const float wQ0 = __fmul_rn(wq, qs[j * M + m0]);
+            const float C0s = tab[r0 + j], C0p = tab[(more ? r0p : r0) + j];
+            const float U0s = __fmaf_rn(-lam, C0s, wQ0), U0p = __fmaf_rn(-lam, C0p, wQ0);
+            uint64_t K0s = cand_key(C0s, U0s, d0, b), K0p = cand_key(C0p, U0p, d0, b);
+            K0s = h0 ? K0s : 0;
+            K0p = h0 ? K0p : 0;
             float C1s = 0.f, U1s = 0.f, C1p = 0.f, U1p = 0.f;
-            uint64_t K0s = 0, K0p = 0, K1s = 0, K1p = 0;
-            if (i + 1 < Qs) {
-                const float b = slo[i + 1];
-                const float wQ0 = __fmul_rn(wq, qs[(i + 1) * M + m0]);
-                C0s = tab[r0 + i + 1];
-                C0p = tab[r0p + i + 1];
-                U0s = __fmaf_rn(-lam, C0s, wQ0);
-                U0p = __fmaf_rn(-lam, C0p, wQ0);
-                K0s = h0 ? cand_key(C0s, U0s, d0, b) : 0;
-                K0p = h0 ? cand_key(C0p, U0p, d0, b) : 0;
-                if (HI) {
-                    const float wQ1 = __fmul_rn(wq, qs[(i + 1) * M + m1]);
-                    C1s = tab[r1 + i + 1];
-                    C1p = tab[r1p + i + 1];
-                    U1s = __fmaf_rn(-lam, C1s, wQ1);
-                    U1p = __fmaf_rn(-lam, C1p, wQ1);
-                    K1s = h1 ? cand_key(C1s, U1s, d1, b) : 0;
-                    K1p = h1 ? cand_key(C1p, U1p, d1, b) : 0;
-                }
+            uint64_t K1s = 0, K1p = 0;
+            if (HI) {
+                const float wQ1 = __fmul_rn(wq, qs[j * M + m1]);
+                C1s = tab[r1 + j];
+                C1p = tab[(more ? r1p : r1) + j];
+                U1s = __fmaf_rn(-lam, C1s, wQ1);
+                U1p = __fmaf_rn(-lam, C1p, wQ1);
+                K1s = cand_key(C1s, U1s, d1, b);
+                K1p = cand_key(C1p, U1p, d1, b);
+                K1s = h1 ? K1s : 0;
+                K1p = h1 ? K1p : 0;
             }
             // step i: the warp's largest key
             const uint64_t kl = HI && K1 > K0 ? K1 : K0;
@@ -849,20 +852,18 @@ k_seq_chain(Model m, Queries q, int Qs, const float *ctab, float *aux, const flo
                 o_lat[i] = __int_as_float(0x7fc00000);
                 o_util[i] = __int_as_float(0x7fc00000);
             }
-            if (p0) {
-                ++c0;
-                r0 = r0p;
-                r0p += D * (Qs - c0) - e0 - 1;
-            }
-            if (HI && p1) {
-                ++c1;
-                r1 = r1p;
-                r1p += D * (Qs - c1) - e1 - 1;
-            }
+            c0 += p0 ? 1 : 0;
+            const int n0 = r0p + D * (Qs - c0) - e0 - 1;
+            r0 = p0 ? r0p : r0;
+            r0p = p0 ? n0 : r0p;
             C0 = p0 ? C0p : C0s;
             U0 = p0 ? U0p : U0s;
             K0 = p0 ? K0p : K0s;
             if (HI) {
+                c1 += p1 ? 1 : 0;
+                const int n1 = r1p + D * (Qs - c1) - e1 - 1;
+                r1 = p1 ? r1p : r1;
+                r1p = p1 ? n1 : r1p;
                 C1 = p1 ? C1p : C1s;
                 U1 = p1 ? U1p : U1s;
                 K1 = p1 ? K1p : K1s;

@@ -42,7 +42,7 @@ __device__ __forceinline__ bool better(const Cand &a, const Cand &b) {
 // map to the same key).
 __device__ __forceinline__ uint32_t order_key(float x) {
     uint32_t u = __float_as_uint(x);
-    if ((u << 1) == 0u) u = 0u;
+    u = (u << 1) == 0u ? 0u : u;
     return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
 }
 
