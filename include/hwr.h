@@ -178,9 +178,11 @@ hwr_status hwr_get_snapshot(hwr_ctx *ctx, int32_t *running_out);
  * Without HWR_DEVICE_PTRS all six arrays are host memory; the call copies the
  * inputs host -> device and the outputs back, and (without HWR_ASYNC)
  * returns after the results are in place (small batches on the small-batch
- * kernel return as soon as every output is written, possibly before the
- * kernel's last blocks retire; a failure after that point is reported by the
- * next call on the context or by hwr_synchronize.  When earlier work is still
+ * kernel, and small HWR_SEQUENTIAL batches on the SIMT kernels, return as
+ * soon as every output is written, possibly before the kernel's last blocks
+ * retire -- the sequential chain then still persists the picks, which later
+ * work on the context is ordered after; a failure after that point is
+ * reported by the next call on the context or by hwr_synchronize.  When earlier work is still
  * queued on the stream -- after an HWR_ASYNC call, or the caller's own work on
  * a stream it passed to hwr_create -- the call synchronises the stream
  * instead of waiting on the outputs).  Where the GPU can read and write

@@ -883,8 +883,9 @@ static hwr_status route_impl(hwr_ctx *c, int32_t Q, const float *in_len, const f
     // with plain loads (no host-to-device copy)
     const bool zero_copy = packed && !tensor && !ml && !so && (c->pin_d || c->ats) &&
                            (seq ? !(flags & HWR_PATH_TENSOR) : (long)Q * c->D <= c->pairs_max);
-    // ... and on the small-batch kernel the host waits for the outputs
-    // themselves instead of synchronising the stream
+    // ... and on these kernels (the small-batch kernel, the sequential chain)
+    // the host waits for the outputs themselves instead of synchronising the
+    // stream
     // ... unless work queued earlier on the stream (an HWR_ASYNC call, or the
     // caller's own work on a stream it passed in) is still running: then
     // the kernel starts late and the host synchronises instead of spinning
@@ -892,7 +893,7 @@ static hwr_status route_impl(hwr_ctx *c, int32_t Q, const float *in_len, const f
     // own arrays: the kernels read the inputs and write the outputs there
     // (plain element loads and stores), with no staging copy either way
     const bool direct = zero_copy && c->ats;
-    bool poll = zero_copy && !seq && c->poll_us > 0;
+    bool poll = zero_copy && c->poll_us > 0;
     if (poll && (c->async_pending || !c->own_stream)) {
         const cudaError_t e = cudaStreamQuery(c->stream);
         if (e == cudaSuccess) {

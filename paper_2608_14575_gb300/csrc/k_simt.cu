@@ -874,9 +874,17 @@ k_seq_chain(Model m, Queries q, int Qs, const float *ctab, float *aux, const flo
     }
     __syncthreads();
     for (int i = tid; i < Qs; i += CHAIN_THREADS) {
-        q.chosen[i] = o_ch[i];
         q.lat[i] = o_lat[i];
         q.util[i] = o_util[i];
+        if (q.inputs_host) {
+            // outputs in host memory: the host may poll chosen with acquire
+            // loads, so it is stored last, with release semantics at system
+            // scope
+            asm volatile("st.release.sys.global.b32 [%0], %1;" ::"l"(q.chosen + i), "r"(o_ch[i])
+                         : "memory");
+        } else {
+            q.chosen[i] = o_ch[i];
+        }
     }
     __syncthreads();
 

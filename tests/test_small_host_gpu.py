@@ -1,4 +1,5 @@
-"""Small synchronous calls with host buffers (the small-batch kernel).
+"""Small synchronous calls with host buffers (the small-batch kernel, and
+sequential routes on the SIMT kernels).
 
 Such a call stages its inputs in mapped host memory and, instead of
 synchronising the stream, waits for the kernel to write each query's chosen
@@ -75,4 +76,41 @@ def test_staged_and_direct_host_paths_agree(monkeypatch, no_ats):
     assert np.array_equal(got[0], want[0])
     assert np.array_equal(got[1], want[1].astype(np.float32))
     assert np.array_equal(r.get_snapshot(), want[3])
+    r.close()
+
+
+def _exact_seq(got, r, p):
+    want = O.Problem(p).route(mode=O.F32, sequential=True)
+    assert np.array_equal(got[0], want[0])
+    assert np.array_equal(got[1], want[1].astype(np.float32))
+    assert np.array_equal(got[2], want[2].astype(np.float32))
+    assert np.array_equal(r.get_snapshot(), want[3])
+
+
+@pytest.mark.parametrize("poll_us", [None, "0"])
+@pytest.mark.parametrize("cfg,Q", [(2, 64), (4, 64)])
+def test_sequential_calls_wait_on_outputs_or_synchronise(monkeypatch, poll_us, cfg, Q):
+    """A small sequential call returns once the chain has written every
+    output (the default) or, with the wait limit at 0, after synchronising the
+    stream; both give the canonical results and the persisted counts.  At
+    D = 32 a 64-query call spans two chunks, whose chains write disjoint parts
+    of the outputs."""
+    if poll_us is not None:
+        monkeypatch.setenv("HWR_TEST_POLL_US", poll_us)
+    p = W.make_config(cfg, Q=Q)
+    r = H.Router(p)
+    for _ in range(2):
+        r.update_snapshot(p["snap"])
+        _exact_seq(r.route(flags=H.HWR_SEQUENTIAL), r, p)
+    r.close()
+
+
+def test_sequential_call_queued_behind_an_async_route():
+    p = W.make_config(4, Q=8192)
+    r = H.Router(p)
+    big = r.route(flags=H.HWR_ASYNC)
+    got = r.route(p["in_len"][:16], p["out_len"][:16], p["emb"][:16], flags=H.HWR_SEQUENTIAL)
+    r.synchronize()
+    check_against_oracle(p, big, idx=np.arange(0, p["Q"], 17))
+    _exact_seq(got, r, W.query_slice(p, 0, 16))
     r.close()
