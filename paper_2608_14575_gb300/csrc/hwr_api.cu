@@ -104,6 +104,9 @@ struct hwr_ctx {
     const uint32_t *snap_hd = nullptr;   // device address of the mapped snap_h
     void *snap_d = nullptr;
     cudaEvent_t snap_ev = nullptr;
+    // a snapshot kernel may still read the staging: set at its launch, cleared
+    // once the host has seen later work on the stream complete
+    bool snap_busy = false;
 
     // grow-only scratch
     float *qual = nullptr;   size_t qual_cap = 0;     // 2 x [Q][Mpad], alternating per call
@@ -639,7 +642,7 @@ extern "C" hwr_status hwr_update_snapshot(hwr_ctx *c, const hwr_snapshot *s) {
     }
     const size_t n = (size_t)c->D * 4;
     // the previous snapshot copy must have left the staging buffer
-    CK(c, cudaEventSynchronize(c->snap_ev), "wait for snapshot staging");
+    if (c->snap_busy) CK(c, cudaEventSynchronize(c->snap_ev), "wait for snapshot staging");
     char *h = (char *)c->snap_h;
     memcpy(h + 0 * n, s->running, n);
     memcpy(h + 1 * n, s->waiting, n);
@@ -653,6 +656,7 @@ extern "C" hwr_status hwr_update_snapshot(hwr_ctx *c, const hwr_snapshot *s) {
     CK(c, launch_snapshot(model_view(c), c->snap_hd, c->stream), "snapshot kernel");
     ls.done();
     CK(c, cudaEventRecord(c->snap_ev, c->stream), "record");
+    c->snap_busy = true;
     c->have_snapshot = true;
     return HWR_OK;
 }
@@ -664,6 +668,7 @@ extern "C" hwr_status hwr_get_snapshot(hwr_ctx *c, int32_t *running_out) {
     CK(c, cudaMemcpyAsync(running_out, c->running, (size_t)c->D * 4, cudaMemcpyDeviceToHost,
                           c->stream), "read running counts");
     CK(c, cudaStreamSynchronize(c->stream), "synchronize");
+    c->snap_busy = false;
     return HWR_OK;
 }
 
@@ -1090,7 +1095,9 @@ static hwr_status route_impl(hwr_ctx *c, int32_t Q, const float *in_len, const f
         return HWR_OK;
     }
     if (!synced) CK(c, cudaStreamSynchronize(c->stream), "synchronize");
+    // this call's work is complete, and with it every earlier kernel
     c->async_pending = false;
+    c->snap_busy = false;
     CK(c, cudaGetLastError(), "kernel");
     if (tensor || (seq && (flags & HWR_PATH_TENSOR))) TRY(check_status_word(c));
     return HWR_OK;
@@ -1149,6 +1156,7 @@ extern "C" hwr_status hwr_synchronize(hwr_ctx *c) {
     if (c->broken) return HWR_ERR_STATE;
     CK(c, cudaStreamSynchronize(c->stream), "synchronize");
     c->async_pending = false;
+    c->snap_busy = false;
     return check_status_word(c);
 }
 

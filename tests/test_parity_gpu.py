@@ -170,6 +170,29 @@ def test_sequential_single_call_exact():
     r.close()
 
 
+def test_back_to_back_snapshots_last_one_wins():
+    """Snapshot updates reuse one staging buffer; an update waits for the
+    previous snapshot kernel only while the host has not yet seen later work
+    on the stream complete.  Updates in a row, and an update after an
+    asynchronous route, must each leave exactly their own snapshot in force."""
+    p = W.make_config(0, Q=256)
+    rng = np.random.default_rng(5)
+    snaps = []
+    for _ in range(3):
+        s = {k: np.array(v, copy=True) for k, v in p["snap"].items()}
+        s["running"] = rng.integers(0, 30, p["D"]).astype(np.int32)
+        s["kv"] = rng.uniform(0, 1, p["D"]).astype(np.float32)
+        snaps.append(s)
+    r = H.Router(p)
+    for s in snaps:
+        r.update_snapshot(s)
+    assert_exact(r.route(), O.Problem(p, snap=snaps[2]).route(mode=O.F32, nthreads=8), "last of three")
+    r.route(flags=H.HWR_ASYNC)
+    r.update_snapshot(snaps[0])
+    assert_exact(r.route(), O.Problem(p, snap=snaps[0]).route(mode=O.F32, nthreads=8), "after async")
+    r.close()
+
+
 def _online(p, n):
     """Run the online micro-batch loop through the GPU and through the oracle."""
     r = H.Router(p)
