@@ -355,10 +355,19 @@ __device__ void pair_mlp(const Model &m, int R, const Rows &rows, const float *u
                         b[0] = wr[0];
                     }
                 }
+                // rows 2ip and 2ip + 1 in one packed fp32 FMA (fma.rn.f32x2:
+                // each lane the same single rounding as __fmaf_rn)
 #pragma unroll
-                for (int i = 0; i < 8; ++i)
+                for (int ip = 0; ip < 4; ++ip) {
+                    const float2 a2 = make_float2(a[2 * ip], a[2 * ip + 1]);
 #pragma unroll
-                    for (int j = 0; j < CPT; ++j) acc[i][j] = __fmaf_rn(b[j], a[i], acc[i][j]);
+                    for (int j = 0; j < CPT; ++j) {
+                        const float2 r = __ffma2_rn(make_float2(b[j], b[j]), a2,
+                                                    make_float2(acc[2 * ip][j], acc[2 * ip + 1][j]));
+                        acc[2 * ip][j] = r.x;
+                        acc[2 * ip + 1][j] = r.y;
+                    }
+                }
             }
         }
         tile_sync();
