@@ -91,6 +91,35 @@ def bytes_per_query(p):
     return p["E"] * es + 8 + 12
 
 
+def qual_bytes_per_query(p):
+    # the quality kernel: the embedding row read, Mpad fp32 qualities written
+    return p["E"] * 2 + (16 if p["M"] <= 16 else 32) * 4
+
+
+def same_size_copy(torch, nbytes, stream, dev):
+    """A device-to-device copy moving the same number of bytes (half read,
+    half written), L2 flushed before each: what a transfer of this size
+    reaches here, ramp and drain included (the measured peak is a long copy)."""
+    half = nbytes // 2
+    src = torch.empty(half, dtype=torch.uint8, device=dev)
+    dst = torch.empty_like(src)
+    flush = torch.empty(2 * L2_BYTES, dtype=torch.uint8, device=dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ts = []
+    with torch.cuda.stream(stream):
+        src.fill_(1)
+        for i in range(13):
+            flush.fill_(i & 0xff)
+            e0.record(stream)
+            dst.copy_(src)
+            e1.record(stream)
+            e1.synchronize()
+            if i >= 3:
+                ts.append(e0.elapsed_time(e1))
+    ms = float(sorted(ts)[len(ts) // 2])
+    return {"bytes": 2 * half, "ms": ms, "gbs": 2 * half / (ms * 1e-3) / 1e9}
+
+
 class ClockSampler:
     """SM clock and clock-event (throttle) reasons, sampled during the timed
     region.  Read-only NVML queries from a host thread every ~2 ms (the
@@ -752,7 +781,7 @@ def main():
                 "peak_source": f"{src} bf16 burst (cuBLAS), frac vs sustained "
                                f"{ach / pk.get('bf16_tflops_sustained', pk['bf16_tflops']):.3f}"}
     elif top == "qual_tc":
-        byt = Q * bytes_per_query(p)
+        byt = Q * qual_bytes_per_query(p)
         ach = byt / (kms[top] * 1e-3) / 1e9
         roof = {"bound": "hbm", "achieved": ach, "peak": pk["hbm_gbs"], "unit": "GB/s",
                 "frac": ach / pk["hbm_gbs"], "traffic": profiled_traffic(top), "kernel": top,
@@ -764,6 +793,18 @@ def main():
         roof = {"bound": "alu", "achieved": ach, "peak": peak, "unit": "TFLOP/s",
                 "frac": ach / peak, "traffic": None, "kernel": top, "ms_per_launch": kms[top],
                 "peak_source": "fp32 FMA: 152 SMs x 128 lanes x 2 x max SM clock"}
+
+    # the other roofline-bound kernel of the step, against the measured peak
+    # and against a copy of the same size
+    others = {}
+    if "qual_tc" in kms and top != "qual_tc":
+        byt = Q * qual_bytes_per_query(p)
+        ach = byt / (kms["qual_tc"] * 1e-3) / 1e9
+        cp = same_size_copy(torch, byt, stream, dev)
+        others["qual_tc"] = {"bound": "hbm", "achieved": ach, "peak": pk["hbm_gbs"], "unit": "GB/s",
+                             "frac": ach / pk["hbm_gbs"], "traffic": profiled_traffic("qual_tc"),
+                             "ms_per_launch": kms["qual_tc"], "bytes_per_launch": byt,
+                             "same_size_copy": cp, "frac_of_same_size_copy": ach / cp["gbs"]}
 
     line = {
         "metric": "routed_queries_per_s", "value": value, "unit": "queries/s",
@@ -777,7 +818,7 @@ def main():
                          f"({'inputs > L2' if in_bytes > L2_BYTES else 'rotation > L2'})",
                    "parallelism": f"replicas x{world} (queries sharded, no collective)"},
         "kernel_ms": kms, "ms_per_step_profiled_pass": ms_prof,
-        "gpu_launches": launches, "roofline": roof, "clocks": clk,
+        "gpu_launches": launches, "roofline": roof, "other_kernels": others, "clocks": clk,
     }
 
     if not args.no_e2e:

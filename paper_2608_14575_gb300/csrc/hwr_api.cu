@@ -104,6 +104,15 @@ struct hwr_ctx {
     const uint32_t *snap_hd = nullptr;   // device address of the mapped snap_h
     void *snap_d = nullptr;
     cudaEvent_t snap_ev = nullptr;
+    // completion counter of the tensor-core predictor kernels (device): every
+    // CTA adds one as it finishes; host side, the CTAs launched in all and by
+    // the most recent predictor launch
+    uint32_t *done_d = nullptr;
+    uint32_t pred_ctas = 0, pred_ctas_last = 0;
+    // outputs of the last tensor-core route (its predictor may still run
+    // while the next route's kernels start)
+    const void *prev_out[3] = {nullptr, nullptr, nullptr};
+    size_t prev_out_bytes = 0;
     // a snapshot kernel may still read the staging: set at its launch, cleared
     // once the host has seen later work on the stream complete
     bool snap_busy = false;
@@ -503,6 +512,8 @@ static hwr_status build_ctx(hwr_ctx *c, const hwr_deployment_table *t, const hwr
         std::vector<uint16_t> img(tc_w2img_elems(H1, H2));
         tc_build_w2img((const uint16_t *)p->W2, H1, H2, img.data());
         TRY(dev_alloc(c, &c->W2img, img.size()));
+        TRY(dev_alloc(c, &c->done_d, 1));
+        CK(c, cudaMemset(c->done_d, 0, sizeof(uint32_t)), "zero completion counter");
         TRY(upload(c, c->W2img, img.data(), img.size() * 2, "upload W2 image"));
         std::vector<uint16_t> mimg(tc_membimg_elems(c->Mpad, c->Epad));
         tc_build_membimg((const uint16_t *)memb_in, E, M, c->Mpad, c->Epad, mimg.data());
@@ -675,6 +686,12 @@ extern "C" hwr_status hwr_get_snapshot(hwr_ctx *c, int32_t *running_out) {
 // ---------------------------------------------------------------------------
 // routing
 
+// Whether byte ranges [a, a + na) and [b, b + nb) share a byte.
+static bool overlaps(const void *a, size_t na, const void *b, size_t nb) {
+    const uintptr_t x = (uintptr_t)a, y = (uintptr_t)b;
+    return a && b && na && nb && x < y + nb && y < x + na;
+}
+
 static hwr_status run_kernels(hwr_ctx *c, const Queries &q, uint32_t flags, bool tensor) {
     const bool prof = flags & HWR_PROFILE;
     const Model m = model_view(c);
@@ -728,9 +745,17 @@ static hwr_status run_kernels(hwr_ctx *c, const Queries &q, uint32_t flags, bool
                 // overlap the half the previous call's kernels still read)
                 float *qb = c->qual + (c->qual_flip ? c->qual_cap / 2 : 0);
                 c->qual_flip ^= 1;
-                CK(c, launch_qual_tc(t, k, qb, c->status_d, c->stream, true), "quality kernel");
-                CK(c, launch_mlp_tc_scores(tv, kt, qb, c->status_d, c->stream),
+                // the preparation kernel lets its dependents start early, and
+                // the cost table reads its prefixes before its dependency wait:
+                // the table starts only once this grid has waited for it
+                CK(c, launch_qual_tc(t, k, qb, c->status_d, c->stream, true, false, 0, c->done_d,
+                                     c->pred_ctas - c->pred_ctas_last),
+                   "quality kernel");
+                int ctas = 0;
+                CK(c, launch_mlp_tc_scores(tv, kt, qb, c->status_d, c->stream, c->done_d, &ctas),
                    "sequential table (tensor cores)");
+                c->pred_ctas += (uint32_t)ctas;
+                c->pred_ctas_last = (uint32_t)ctas;
                 a.done();
                 CK(c, launch_seq_chain_tc(m, k, n, c->ctab, c->qseq, qb, c->Mpad, c->stream),
                    "sequential chain");
@@ -766,12 +791,35 @@ static hwr_status run_kernels(hwr_ctx *c, const Queries &q, uint32_t flags, bool
                 CK(c, cudaMemsetAsync(c->count, 0, c->count_cap * 4, c->stream), "zero counters");
             }
         }
+        // The predictor may start as soon as the quality kernel has: before
+        // its dependency wait it reads only weights, the snapshot's prefixes
+        // and this call's inputs -- unless those inputs are outputs of the
+        // previous tensor-core route, whose predictor may still be running.
+        const size_t qb4 = (size_t)q.Q * 4;
+        bool early = true;
+        for (int o = 0; o < 3; ++o)
+            if (overlaps(q.in_len, qb4, c->prev_out[o], c->prev_out_bytes) ||
+                overlaps(q.out_len, qb4, c->prev_out[o], c->prev_out_bytes) ||
+                overlaps(q.emb, (size_t)q.Q * c->E * 2, c->prev_out[o], c->prev_out_bytes) ||
+                (q.slo_q && overlaps(q.slo_q, qb4, c->prev_out[o], c->prev_out_bytes)))
+                early = false;
+        const int free_sms = tc_mlp_free_sms(q.Q, sp);
         LaunchScope a(c, HWR_K_QUAL_TC, prof);
-        CK(c, launch_qual_tc(t, q, qb, c->status_d, c->stream, true), "quality kernel");
+        CK(c, launch_qual_tc(t, q, qb, c->status_d, c->stream, true, early, free_sms, c->done_d,
+                             c->pred_ctas - c->pred_ctas_last),
+           "quality kernel");
         a.done();
+        c->prev_out[0] = q.chosen;
+        c->prev_out[1] = q.lat;
+        c->prev_out[2] = q.util;
+        c->prev_out_bytes = qb4;
         LaunchScope b(c, HWR_K_MLP_TC, prof);
-        CK(c, launch_mlp_tc(t, q, qb, sp, c->part, c->count, c->status_d, c->stream),
+        int ctas = 0;
+        CK(c, launch_mlp_tc(t, q, qb, sp, c->part, c->count, c->status_d, c->stream, c->done_d,
+                            &ctas),
            "predictor kernel");
+        c->pred_ctas += (uint32_t)ctas;
+        c->pred_ctas_last = (uint32_t)ctas;
         b.done();
         return HWR_OK;
     }
@@ -1234,10 +1282,13 @@ hwr_status hwr_internal_route_tensor_scratch(hwr_ctx *c, int32_t Q, const float 
     if (sp.nsplit > 1)
         CK(c, cudaMemsetAsync(count, 0, (size_t)Q * sizeof(int32_t), c->stream), "clear counters");
     // one static quality buffer: a plain launch, ordered after the kernel before
-    CK(c, launch_qual_tc(t, q, qual, c->status_d, c->stream, false), "quality kernel");
+    CK(c, launch_qual_tc(t, q, qual, c->status_d, c->stream, false, false, 0, nullptr, 0),
+       "quality kernel");
     c->stats.kernel_launches++;
     c->stats.launches[HWR_K_QUAL_TC]++;
-    CK(c, launch_mlp_tc(t, q, qual, sp, part, count, c->status_d, c->stream), "predictor kernel");
+    int ctas = 0;
+    CK(c, launch_mlp_tc(t, q, qual, sp, part, count, c->status_d, c->stream, nullptr, &ctas),
+       "predictor kernel");
     c->stats.kernel_launches++;
     c->stats.launches[HWR_K_MLP_TC]++;
     c->stats.queries_routed += Q;

@@ -184,8 +184,16 @@ void tc_build_membimg(const uint16_t *memb_EM, int E, int M, int Mpad, int Epad,
 // dependent: launched as a programmatic dependent of the kernel before it on
 // the stream, running alongside it -- only when that kernel does not read
 // `qual` (the context alternates two quality buffers between calls).
+// early: its dependent may be scheduled as soon as the grid has started (only
+// when the kernel before does not let its own dependents start early with
+// results the predictor reads before its dependency wait, and this call's
+// inputs are not the previous call's outputs); free_sms: SMs the predictor
+// after it leaves free (a small batch is spread over those alone).
+// done, done_target: the predictors' completion counter; before its first
+// store the grid waits for it to reach done_target (nullptr: no wait).
 cudaError_t launch_qual_tc(const TcModel &m, const Queries &q, float *qual,
-                           int32_t *status, cudaStream_t s, bool dependent);
+                           int32_t *status, cudaStream_t s, bool dependent, bool early,
+                           int free_sms, const uint32_t *done, uint32_t done_target);
 // The first nwhole query tiles are processed whole; the deployments of each
 // remaining tile are split over nsplit units.  With nsplit > 1, `part`
 // (nsplit * Q records of 16 bytes) and `count` (Q int32, zero, self-resetting)
@@ -194,14 +202,18 @@ struct MlpSplit {
     int nwhole, nsplit;
 };
 MlpSplit tc_mlp_split(const TcModel &m, int Q, int max_split = 8);
+// SMs the predictor kernel for Q queries split as sp leaves free (0 if none).
+int tc_mlp_free_sms(int Q, const MlpSplit &sp);
+// done: completion counter every CTA increments (release) as it finishes
+// (nullptr: none); *ctas: the CTAs launched (0 on failure).
 cudaError_t launch_mlp_tc(const TcModel &m, const Queries &q, const float *qual,
                           const MlpSplit &sp, void *part, int32_t *count, int32_t *status,
-                          cudaStream_t s);
+                          cudaStream_t s, uint32_t *done, int *ctas);
 cudaError_t tc_prepare();
 // Costs of every (query, deployment) pair of at most 128 queries into
 // q.pair_C [Q][m.D] (q.no_select set), the deployments spread over the SMs.
 cudaError_t launch_mlp_tc_scores(const TcModel &m, const Queries &q, const float *qual,
-                                 int32_t *status, cudaStream_t s);
+                                 int32_t *status, cudaStream_t s, uint32_t *done, int *ctas);
 size_t tc_head_consts_bytes();
 void tc_fill_head_consts(void *dst, const float *b2, const float *W3, const float *b3, int H2,
                          int NH);

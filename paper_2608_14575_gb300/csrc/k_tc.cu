@@ -179,7 +179,7 @@ __device__ __forceinline__ float standardise_fast(uint8_t code, float v, float m
 
 __global__ void __launch_bounds__(QUAL_THREADS, 1)
 k_qual_tc(const __grid_constant__ CUtensorMap tmap, TcModel m, int Q, float *qual,
-          int32_t *status) {
+          int32_t *status, int early, const uint32_t *done, uint32_t done_target) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *sm = align1024(smem_raw);
     const QualLayout L = qual_layout(m.Mpad, m.Epad);
@@ -219,8 +219,14 @@ k_qual_tc(const __grid_constant__ CUtensorMap tmap, TcModel m, int Q, float *qua
     // the query embeddings, which were complete before that kernel began, and
     // writes its own quality buffer (two alternate between calls), so it runs
     // alongside that kernel.  It waits for that kernel's completion only at
-    // the end, before it lets the predictor of its own call start: that
-    // predictor's outputs and scratch are then ordered after the previous one.
+    // the end.  Its own dependent, the predictor of this call, touches memory
+    // that the kernels before may write (outputs, scratch) only after waiting
+    // for this grid's completion, so with `early` it may be scheduled at once:
+    // its set-up, weight load and first layer-2 steps then overlap this grid
+    // and the kernel before.  Without `early` (the kernel before lets its own
+    // dependents start early and writes what the predictor reads first, or
+    // the caller's inputs may alias earlier outputs) only at the end.
+    if (early) grid_launch_dependents();
 
     if (warp == 0 && lane == 0) {
         // producer: model embeddings once, then query tiles chunk by chunk
@@ -276,7 +282,7 @@ k_qual_tc(const __grid_constant__ CUtensorMap tmap, TcModel m, int Q, float *qua
         const int quad = warp & 3, r = quad * 32 + lane;
         const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
         uint32_t lt = 0;
-        bool ok = true;
+        bool ok = true, may_store = done == nullptr;
         for (int t = blockIdx.x; t < ntiles; t += gridDim.x, ++lt) {
             const int b = lt & 1;
             ok = mbar_wait(&accf[b], (lt >> 1) & 1, abort_f, status);
@@ -297,6 +303,17 @@ k_qual_tc(const __grid_constant__ CUtensorMap tmap, TcModel m, int Q, float *qua
             }
             tc_fence_before();
             mbar_arrive(&acce[b]);
+            if (!may_store) {
+                // This buffer was last read by the predictor two routes back
+                // (the buffers alternate), which may still run when this grid
+                // starts: before the first store, every predictor CTA launched
+                // before the most recent predictor has finished.
+                if (lane == 0) ok = count_wait(done, done_target, abort_f, status);
+                ok = __shfl_sync(0xffffffffu, ok, 0);
+                __syncwarp();
+                may_store = true;
+                if (!ok) break;
+            }
             const int row = t * BM + r;
             if (row < Q) {
                 float4 *dst = (float4 *)(qual + (size_t)row * Mpad);
@@ -314,7 +331,7 @@ k_qual_tc(const __grid_constant__ CUtensorMap tmap, TcModel m, int Q, float *qua
     tc_fence_before();
     __syncthreads();
     grid_dependency_wait();
-    grid_launch_dependents();
+    if (!early) grid_launch_dependents();
     if (warp == 1) {
         __syncwarp();
         tc_fence_after();
@@ -416,7 +433,7 @@ template <int H2T, int NH>
 __global__ void __launch_bounds__(MLP_THREADS, 1)
 k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
          const float *__restrict__ qual, int nwhole, int nsplit, int4 *part, int32_t *count,
-         int32_t *status) {
+         int32_t *status, uint32_t *done) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *sm = align1024(smem_raw);
     constexpr bool FIXED = H2T > 0;
@@ -825,6 +842,9 @@ k_mlp_tc(TcModel m, Queries q, const __grid_constant__ HeadConsts hc,
     }
     tc_fence_before();
     __syncthreads();
+    // every global access of this CTA is done: count it for the quality kernel
+    // that will next overwrite the quality buffer this grid read
+    if (done && tid == 0) count_release(done);
     if (warp == 0) {
         __syncwarp();
         tc_fence_after();
@@ -875,7 +895,8 @@ cudaError_t tc_prepare() {
 }
 
 cudaError_t launch_qual_tc(const TcModel &m, const Queries &q, float *qual, int32_t *status,
-                           cudaStream_t s, bool dependent) {
+                           cudaStream_t s, bool dependent, bool early, int free_sms,
+                           const uint32_t *done, uint32_t done_target) {
     if (q.Q <= 0) return cudaSuccess;
     CUtensorMap map;
     const cuuint64_t dims[2] = {(cuuint64_t)m.E, (cuuint64_t)q.Q};
@@ -890,7 +911,14 @@ cudaError_t launch_qual_tc(const TcModel &m, const Queries &q, float *qual, int3
     // as many CTAs as give every CTA the same number of tiles (512 tiles on
     // 152 SMs: 128 CTAs of 4 tiles, not 152 with a last round on 56)
     const int ntiles = (q.Q + BM - 1) / BM;
-    const int rounds = (ntiles + g_num_sms - 1) / g_num_sms;
+    int rounds = (ntiles + g_num_sms - 1) / g_num_sms;
+    // a small batch on the SMs the predictor leaves free, at most two tiles
+    // each: the predictor's CTAs then find their SMs free as the previous
+    // predictor's leave (4,096 queries at D = 32: 16 CTAs of 2 tiles beside
+    // 128 predictor CTAs, 24.8 -> 19.6 us per call back to back; with three or
+    // more tiles per CTA the longer quality kernel costs a lone call more
+    // than the overlap gives)
+    if (early && free_sms >= 8 && ntiles <= 2 * free_sms) rounds = (ntiles + free_sms - 1) / free_sms;
     const int grid = (ntiles + rounds - 1) / rounds;
     const QualLayout L = qual_layout(m.Mpad, m.Epad);
     // programmatic dependent launch (when `qual` is not read by the kernel
@@ -906,18 +934,20 @@ cudaError_t launch_qual_tc(const TcModel &m, const Queries &q, float *qual, int3
     cfg.stream = s;
     cfg.attrs = at;
     cfg.numAttrs = dependent ? 1 : 0;
-    return cudaLaunchKernelEx(&cfg, k_qual_tc, map, m, q.Q, qual, status);
+    return cudaLaunchKernelEx(&cfg, k_qual_tc, map, m, q.Q, qual, status, early ? 1 : 0, done,
+                              done_target);
 }
 
 cudaError_t launch_mlp_tc_scores(const TcModel &m, const Queries &q, const float *qual,
-                                 int32_t *status, cudaStream_t s) {
+                                 int32_t *status, cudaStream_t s, uint32_t *done, int *ctas) {
+    *ctas = 0;
     if (q.Q <= 0) return cudaSuccess;
     if (q.Q > BM || !q.no_select || !q.pair_C) return cudaErrorInvalidValue;
     if (q.seq_n && (q.seq_n != q.Q || m.D % (q.seq_n + 1))) return cudaErrorInvalidValue;
     // one tile: split its deployments into one part per SM
     const int sms = g_num_sms > 0 ? g_num_sms : 1;
     const MlpSplit sp{0, m.D < sms ? m.D : sms};
-    return launch_mlp_tc(m, q, qual, sp, nullptr, nullptr, status, s);
+    return launch_mlp_tc(m, q, qual, sp, nullptr, nullptr, status, s, done, ctas);
 }
 
 // Unit decomposition that minimises the busiest CTA's cost in deployment
@@ -950,9 +980,16 @@ MlpSplit tc_mlp_split(const TcModel &m, int Q, int max_split) {
     return best;
 }
 
+int tc_mlp_free_sms(int Q, const MlpSplit &sp) {
+    const int ntiles = (Q + BM - 1) / BM;
+    const long units = sp.nwhole + (long)(ntiles - sp.nwhole) * sp.nsplit;
+    return units < g_num_sms ? g_num_sms - (int)units : 0;
+}
+
 cudaError_t launch_mlp_tc(const TcModel &m, const Queries &q, const float *qual,
                           const MlpSplit &sp, void *part, int32_t *count, int32_t *status,
-                          cudaStream_t s) {
+                          cudaStream_t s, uint32_t *done, int *ctas) {
+    *ctas = 0;
     if (q.Q <= 0) return cudaSuccess;
     const int ntiles = (q.Q + BM - 1) / BM;
     if (sp.nwhole < 0 || sp.nwhole > ntiles || sp.nsplit < 1) return cudaErrorInvalidValue;
@@ -973,18 +1010,22 @@ cudaError_t launch_mlp_tc(const TcModel &m, const Queries &q, const float *qual,
     cfg.stream = s;
     cfg.attrs = at;
     cfg.numAttrs = 1;
+    cudaError_t e;
 #define HWR_MLP(H2T, NHT) \
-    return cudaLaunchKernelEx(&cfg, k_mlp_tc<H2T, NHT>, m, q, hc, qual, sp.nwhole, sp.nsplit, pt, \
-                              count, status)
+    e = cudaLaunchKernelEx(&cfg, k_mlp_tc<H2T, NHT>, m, q, hc, qual, sp.nwhole, sp.nsplit, pt, \
+                           count, status, done)
     if (m.NH == 3) {
         if (m.H2 == 256) HWR_MLP(256, 3);
-        if (m.H2 == 128) HWR_MLP(128, 3);
-        HWR_MLP(0, 3);
+        else if (m.H2 == 128) HWR_MLP(128, 3);
+        else HWR_MLP(0, 3);
+    } else {
+        if (m.H2 == 256) HWR_MLP(256, 2);
+        else if (m.H2 == 128) HWR_MLP(128, 2);
+        else HWR_MLP(0, 2);
     }
-    if (m.H2 == 256) HWR_MLP(256, 2);
-    if (m.H2 == 128) HWR_MLP(128, 2);
-    HWR_MLP(0, 2);
 #undef HWR_MLP
+    if (e == cudaSuccess) *ctas = grid;
+    return e;
 }
 
 size_t tc_head_consts_bytes() { return sizeof(HeadConsts); }

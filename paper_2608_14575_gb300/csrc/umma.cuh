@@ -121,6 +121,36 @@ __device__ __forceinline__ void grid_dependency_wait() {
     asm volatile("griddepcontrol.wait;" ::: "memory");
 }
 
+// ---- completion counter -----------------------------------------------------
+
+// Count this CTA as finished on `ctr` (release at GPU scope: the CTA's global
+// reads and writes, ordered before this thread by the barrier before the
+// call, happen before whatever acquires the new value).
+__device__ __forceinline__ void count_release(uint32_t *ctr) {
+    asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(ctr) : "memory");
+}
+
+// Wait (bounded) until `ctr` has reached `target` (modulo 2^32: the counter
+// only grows), acquiring what the counted CTAs did.  On timeout: sets the
+// abort flag and the status word and returns false.
+__device__ __forceinline__ bool count_wait(const uint32_t *ctr, uint32_t target,
+                                           volatile int *abort_flag, int32_t *status) {
+    const long long t0 = clock64();
+    while (true) {
+        uint32_t v;
+        asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(ctr) : "memory");
+        if ((int32_t)(v - target) >= 0) return true;
+        if (*abort_flag) return false;
+        if (clock64() - t0 > WAIT_CYCLES) {
+            *abort_flag = 1;
+            *(volatile int32_t *)status = 1;  // ST_TIMEOUT
+            __threadfence_system();
+            return false;
+        }
+        __nanosleep(64);
+    }
+}
+
 // ---- tcgen05 ---------------------------------------------------------------
 
 __device__ __forceinline__ void tmem_alloc(uint32_t *dst_smem, uint32_t ncols) {

@@ -116,6 +116,72 @@ def test_tensor_device_pointers():
     r.close()
 
 
+def _dev_batch(p, lo, hi, dev):
+    import torch
+    return (torch.from_numpy(p["in_len"][lo:hi].copy()).to(dev),
+            torch.from_numpy(p["out_len"][lo:hi].copy()).to(dev),
+            torch.from_numpy(p["emb"][lo:hi].view(np.int16).copy()).to(dev))
+
+
+def _outs(n, dev):
+    import torch
+    return (torch.empty(n, dtype=torch.int32, device=dev), torch.empty(n, device=dev),
+            torch.empty(n, device=dev))
+
+
+@pytest.mark.parametrize("cfg,Q", [(4, 4096), (4, 1024), (3, 8192)])
+def test_back_to_back_routes_keep_stream_order(cfg, Q):
+    """Routes queued back to back overlap (a predictor starts while the
+    quality kernel and the previous predictor still run); each must still
+    equal the same route run alone, and a later route writing the same
+    output arrays must leave its own results there."""
+    import torch
+    dev = torch.device("cuda:0")
+    p = W.make_config(cfg, Q=2 * Q)
+    r = H.Router(p, stream=torch.cuda.current_stream().cuda_stream)
+    A, B = _dev_batch(p, 0, Q, dev), _dev_batch(p, Q, 2 * Q, dev)
+    ref = []
+    for batch in (A, B):
+        o = _outs(Q, dev)
+        r.route_device(*batch, *o, slo=p["slo"], lam=p["lam"], flags=TC)
+        torch.cuda.synchronize()
+        ref.append([t.cpu().numpy() for t in o])
+    X, Y = _outs(Q, dev), _outs(Q, dev)
+    for _ in range(3):
+        r.route_device(*A, *X, slo=p["slo"], lam=p["lam"], flags=TC | H.HWR_ASYNC)
+        r.route_device(*B, *X, slo=p["slo"], lam=p["lam"], flags=TC | H.HWR_ASYNC)
+        r.route_device(*A, *Y, slo=p["slo"], lam=p["lam"], flags=TC | H.HWR_ASYNC)
+    r.synchronize()
+    for got, want in ((X, ref[1]), (Y, ref[0])):
+        for a, b in zip(got, want):
+            assert np.array_equal(a.cpu().numpy(), b, equal_nan=True)
+    r.close()
+
+
+def test_inputs_that_are_the_previous_routes_outputs():
+    """A route queued right behind another whose outputs it reads as inputs
+    (here the first route's latencies as the second's output lengths) must
+    see them complete: the predictor then waits for the previous one before
+    it reads anything."""
+    import torch
+    dev = torch.device("cuda:0")
+    p = W.make_config(4, Q=4096)
+    r = H.Router(p, stream=torch.cuda.current_stream().cuda_stream)
+    il, ol, em = _dev_batch(p, 0, p["Q"], dev)
+    o1, o2 = _outs(p["Q"], dev), _outs(p["Q"], dev)
+    for _ in range(3):
+        r.route_device(il, ol, em, *o1, slo=p["slo"], lam=p["lam"], flags=TC | H.HWR_ASYNC)
+        r.route_device(il, o1[1], em, *o2, slo=p["slo"], lam=p["lam"], flags=TC | H.HWR_ASYNC)
+    r.synchronize()
+    lat1 = o1[1].clone()
+    o3 = _outs(p["Q"], dev)
+    r.route_device(il, lat1, em, *o3, slo=p["slo"], lam=p["lam"], flags=TC)
+    torch.cuda.synchronize()
+    for a, b in zip(o2, o3):
+        assert np.array_equal(a.cpu().numpy(), b.cpu().numpy(), equal_nan=True)
+    r.close()
+
+
 @pytest.mark.parametrize("Q", [1, 16, 256, 4096, 65_536])
 def test_batch_sweep_d32(Q):
     p = W.make_config(4, Q=Q)
