@@ -252,6 +252,7 @@ class Router:
                             b[4 * D:5 * D].view(np.float32), b[5 * D:6 * D].view(np.float32))
         base = b.ctypes.data
         self._snap_struct = hwr_snapshot(*[base + 4 * D * k for k in range(6)])
+        self._snap_ref = ct.byref(self._snap_struct)
         self.update_snapshot(p["snap"])
 
     def _check(self, st):
@@ -259,13 +260,15 @@ class Router:
             raise HwrError(st, self.lib.hwr_last_error(self.ctx).decode())
 
     def update_snapshot(self, snap: dict):
-        v = self._snap_views
-        for k, name in enumerate(("running", "waiting", "kv", "gpu_util", "ttft", "tpot")):
-            a = np.asarray(snap[name])
-            if a.shape != (self.D,):
-                raise ValueError(f"snapshot {name}: shape {a.shape}, want ({self.D},)")
-            v[k][...] = a
-        self._check(self.lib.hwr_update_snapshot(self.ctx, ct.byref(self._snap_struct)))
+        shape = (self.D,)
+        for v, name in zip(self._snap_views, ("running", "waiting", "kv", "gpu_util", "ttft", "tpot")):
+            a = snap[name]
+            if a.__class__ is not np.ndarray:
+                a = np.asarray(a)
+            if a.shape != shape:
+                raise ValueError(f"snapshot {name}: shape {a.shape}, want {shape}")
+            v[...] = a
+        self._check(self.lib.hwr_update_snapshot(self.ctx, self._snap_ref))
 
     def get_snapshot(self) -> np.ndarray:
         out = np.empty(self.D, np.int32)
