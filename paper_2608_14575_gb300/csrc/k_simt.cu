@@ -196,10 +196,22 @@ __global__ void __launch_bounds__(SIMT_THREADS) k_snapshot(Model m, const uint32
     for (int j = threadIdx.x; j < m.H1; j += blockDim.x) {
         const float *w = m.W1T + j;   // slot k at w[k * H1]
         float acc = m.b1[j];
-        int k = 0;
-        for (; k <= m.P; ++k) acc = __fmaf_rn(w[(size_t)k * m.H1], xs[k], acc);
+        // slots k0 .. k1 - 1 in order, their weights loaded eight at a time
+        // ahead of the FMAs (the loads would otherwise wait one by one)
+        auto chain = [&](int k0, int k1) {
+            int k = k0;
+            for (; k + 8 <= k1; k += 8) {
+                float wv[8];
+#pragma unroll
+                for (int t = 0; t < 8; ++t) wv[t] = w[(size_t)(k + t) * m.H1];
+#pragma unroll
+                for (int t = 0; t < 8; ++t) acc = __fmaf_rn(wv[t], xs[k + t], acc);
+            }
+            for (; k < k1; ++k) acc = __fmaf_rn(w[(size_t)k * m.H1], xs[k], acc);
+        };
+        chain(0, m.P + 1);
         m.Spre[(size_t)d * m.H1 + j] = acc;
-        for (; k < m.F - 2; ++k) acc = __fmaf_rn(w[(size_t)k * m.H1], xs[k], acc);
+        chain(m.P + 1, m.F - 2);
         m.A[(size_t)d * m.H1 + j] = acc;
         m.Abf[(size_t)d * m.H1 + j] = __bfloat16_as_ushort(__float2bfloat16_rn(acc));
     }
@@ -600,7 +612,22 @@ k_seq_prep(Model m, Queries q, int Qs, float *aux, uint16_t *pre_bf, int32_t *dm
         float acc[PREP_COUNTS];
 #pragma unroll
         for (int c = 0; c < PREP_COUNTS; ++c) acc[c] = __fmaf_rn(w, xr[c], s0);
-        for (int k = P + 2; k < F - 2; ++k) {
+        // the remaining slots in order, their weights and features loaded
+        // eight at a time ahead of the FMAs
+        int k = P + 2;
+        for (; k + 8 <= F - 2; k += 8) {
+            float wv[8], xv[8];
+#pragma unroll
+            for (int t = 0; t < 8; ++t) {
+                wv[t] = m.W1T[(size_t)(k + t) * H1 + j];
+                xv[t] = x[k + t];
+            }
+#pragma unroll
+            for (int t = 0; t < 8; ++t)
+#pragma unroll
+                for (int c = 0; c < PREP_COUNTS; ++c) acc[c] = __fmaf_rn(wv[t], xv[t], acc[c]);
+        }
+        for (; k < F - 2; ++k) {
             const float wk = m.W1T[(size_t)k * H1 + j], xk = x[k];
 #pragma unroll
             for (int c = 0; c < PREP_COUNTS; ++c) acc[c] = __fmaf_rn(wk, xk, acc[c]);
