@@ -696,7 +696,11 @@ static hwr_status run_kernels(hwr_ctx *c, const Queries &q, uint32_t flags, bool
     const bool prof = flags & HWR_PROFILE;
     const Model m = model_view(c);
     if (flags & HWR_SEQUENTIAL) {
-        const int Qs = c->seq_qs;
+        // chunks of equal size, at most seq_qs: the table grows with the square
+        // of a chunk, so 64 queries under a 55-query limit run as 32 + 32, not
+        // 55 + 9 (the walk, and so every result, is the same either way)
+        const int nchunks = (q.Q + c->seq_qs - 1) / c->seq_qs;
+        const int Qs = (q.Q + nchunks - 1) / nchunks;
         // HWR_PATH_TENSOR: the table on the tensor cores (bf16 contexts)
         const bool tcs = (flags & HWR_PATH_TENSOR) && c->tc_ok;
         if (tcs) {
