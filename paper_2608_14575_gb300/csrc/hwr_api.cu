@@ -111,8 +111,10 @@ struct hwr_ctx {
     uint32_t pred_ctas = 0, pred_ctas_last = 0;
     // outputs of the last tensor-core route (its predictor may still run
     // while the next route's kernels start)
-    const void *prev_out[3] = {nullptr, nullptr, nullptr};
-    size_t prev_out_bytes = 0;
+    struct Range {
+        const void *p = nullptr;
+        size_t n = 0;
+    } prev_out[4];                   // chosen, latency, utility, per-pair costs
     // a snapshot kernel may still read the staging: set at its launch, cleared
     // once the host has seen later work on the stream complete
     bool snap_busy = false;
@@ -801,11 +803,10 @@ static hwr_status run_kernels(hwr_ctx *c, const Queries &q, uint32_t flags, bool
         // previous tensor-core route, whose predictor may still be running.
         const size_t qb4 = (size_t)q.Q * 4;
         bool early = true;
-        for (int o = 0; o < 3; ++o)
-            if (overlaps(q.in_len, qb4, c->prev_out[o], c->prev_out_bytes) ||
-                overlaps(q.out_len, qb4, c->prev_out[o], c->prev_out_bytes) ||
-                overlaps(q.emb, (size_t)q.Q * c->E * 2, c->prev_out[o], c->prev_out_bytes) ||
-                (q.slo_q && overlaps(q.slo_q, qb4, c->prev_out[o], c->prev_out_bytes)))
+        for (const auto &o : c->prev_out)
+            if (overlaps(q.in_len, qb4, o.p, o.n) || overlaps(q.out_len, qb4, o.p, o.n) ||
+                overlaps(q.emb, (size_t)q.Q * c->E * 2, o.p, o.n) ||
+                (q.slo_q && overlaps(q.slo_q, qb4, o.p, o.n)))
                 early = false;
         const int free_sms = tc_mlp_free_sms(q.Q, sp);
         LaunchScope a(c, HWR_K_QUAL_TC, prof);
@@ -813,10 +814,10 @@ static hwr_status run_kernels(hwr_ctx *c, const Queries &q, uint32_t flags, bool
                              c->pred_ctas - c->pred_ctas_last),
            "quality kernel");
         a.done();
-        c->prev_out[0] = q.chosen;
-        c->prev_out[1] = q.lat;
-        c->prev_out[2] = q.util;
-        c->prev_out_bytes = qb4;
+        c->prev_out[0] = {q.chosen, qb4};
+        c->prev_out[1] = {q.lat, qb4};
+        c->prev_out[2] = {q.util, qb4};
+        c->prev_out[3] = {q.pair_C, q.pair_C ? qb4 * c->D : 0};
         LaunchScope b(c, HWR_K_MLP_TC, prof);
         int ctas = 0;
         CK(c, launch_mlp_tc(t, q, qb, sp, c->part, c->count, c->status_d, c->stream, c->done_d,
