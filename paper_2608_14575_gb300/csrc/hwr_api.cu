@@ -698,13 +698,17 @@ static hwr_status run_kernels(hwr_ctx *c, const Queries &q, uint32_t flags, bool
     const bool prof = flags & HWR_PROFILE;
     const Model m = model_view(c);
     if (flags & HWR_SEQUENTIAL) {
-        // chunks of equal size, at most seq_qs: the table grows with the square
-        // of a chunk, so 64 queries under a 55-query limit run as 32 + 32, not
-        // 55 + 9 (the walk, and so every result, is the same either way)
-        const int nchunks = (q.Q + c->seq_qs - 1) / c->seq_qs;
-        const int Qs = (q.Q + nchunks - 1) / nchunks;
         // HWR_PATH_TENSOR: the table on the tensor cores (bf16 contexts)
         const bool tcs = (flags & HWR_PATH_TENSOR) && c->tc_ok;
+        // Chunks of equal size, at most the limit: the SIMT table grows with
+        // the square of a chunk, so 64 queries under a 55-query limit run as
+        // 32 + 32, not 55 + 9 (the walk, and so every result, is the same
+        // either way).  The tensor-core table is cheap per entry and a chunk
+        // costs four dependent kernels: its chunks go up to SEQ_MAX_CHUNK,
+        // the chain reading the rows that do not fit its shared memory from L2.
+        const int limit = tcs ? SEQ_MAX_CHUNK : c->seq_qs;
+        const int nchunks = (q.Q + limit - 1) / limit;
+        const int Qs = (q.Q + nchunks - 1) / nchunks;
         if (tcs) {
             const size_t Dv = (size_t)c->D * (Qs + 1);
             TRY(grow(c, &c->prebf, &c->prebf_cap, Dv * c->H1));

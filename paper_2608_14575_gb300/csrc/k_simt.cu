@@ -771,10 +771,12 @@ __device__ __forceinline__ uint64_t cand_key(float C, float U, int d, float slo)
 
 // HI: deployments 32 .. 63 exist (D > 32); without them every lane of the
 // walk carries one deployment and the second half of the step is compiled out.
-template <bool HI>
+// BIG: only the table's first `tsm` entries (the rows of the first counts)
+// fit in shared memory; the walk reads the rest from global memory (L2).
+template <bool HI, bool BIG>
 __global__ void __launch_bounds__(CHAIN_THREADS)
 k_seq_chain(Model m, Queries q, int Qs, const float *ctab, float *aux, const float *qsrc,
-            int qstride) {
+            int qstride, int tsm) {
     extern __shared__ float4 sm4[];
     float *sm = reinterpret_cast<float *>(sm4);
     const int tid = threadIdx.x, lane = tid & 31;
@@ -783,7 +785,16 @@ k_seq_chain(Model m, Queries q, int Qs, const float *ctab, float *aux, const flo
     const size_t T = tri_off(D, Qs, Qs);
     int *dm = reinterpret_cast<int *>(sm), *cnt = dm + MAX_D;
     float *tab = sm + 2 * MAX_D;
-    float *qs = tab + chain_tab_floats(D, Qs), *slo = qs + (size_t)Qs * M;
+    float *qs = tab + (BIG ? (size_t)tsm : chain_tab_floats(D, Qs)), *slo = qs + (size_t)Qs * M;
+    const size_t Ts = BIG ? (size_t)tsm : T;    // entries staged in shared memory
+    // entry e of the table: shared memory, or (BIG, e >= tsm) global memory
+    auto at = [&](int e) -> float {
+        if constexpr (BIG) {
+            return e < tsm ? tab[e] : __ldcg(ctab + e);
+        } else {
+            return tab[e];
+        }
+    };
     float *o_lat = slo + Qs, *o_util = o_lat + Qs;
     int *o_ch = reinterpret_cast<int *>(o_util + Qs);
 
@@ -796,11 +807,11 @@ k_seq_chain(Model m, Queries q, int Qs, const float *ctab, float *aux, const flo
     const uint32_t tab_s = (uint32_t)__cvta_generic_to_shared(tab);
     // the triangular table, by 16-byte asynchronous copies (both sides
     // 16-byte aligned)
-    for (size_t e = tid; e < T / 4; e += CHAIN_THREADS)
+    for (size_t e = tid; e < Ts / 4; e += CHAIN_THREADS)
         asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(tab_s + (uint32_t)(16 * e)),
                      "l"(__cvta_generic_to_global(ctab + 4 * e))
                      : "memory");
-    for (size_t e = T / 4 * 4 + tid; e < T; e += CHAIN_THREADS) tab[e] = __ldcg(ctab + e);
+    for (size_t e = Ts / 4 * 4 + tid; e < Ts; e += CHAIN_THREADS) tab[e] = __ldcg(ctab + e);
     asm volatile("cp.async.commit_group;" ::: "memory");
     for (int e = tid; e < Qs * M; e += CHAIN_THREADS) {
         const int i = e / M;
@@ -835,12 +846,12 @@ k_seq_chain(Model m, Queries q, int Qs, const float *ctab, float *aux, const flo
         uint64_t K0, K1 = 0;
         {
             const float b = slo[0];
-            C0 = tab[r0];
+            C0 = at(r0);
             U0 = __fmaf_rn(-lam, C0, __fmul_rn(wq, qs[m0]));
             K0 = cand_key(C0, U0, d0, b);
             K0 = h0 ? K0 : 0;
             if (HI) {
-                C1 = tab[r1];
+                C1 = at(r1);
                 U1 = __fmaf_rn(-lam, C1, __fmul_rn(wq, qs[m1]));
                 K1 = cand_key(C1, U1, d1, b);
                 K1 = h1 ? K1 : 0;
@@ -853,7 +864,7 @@ k_seq_chain(Model m, Queries q, int Qs, const float *ctab, float *aux, const flo
             const int j = more ? i + 1 : i;
             const float b = slo[j];
             const float wQ0 = __fmul_rn(wq, qs[j * M + m0]);
-            const float C0s = tab[r0 + j], C0p = tab[(more ? r0p : r0) + j];
+            const float C0s = at(r0 + j), C0p = at((more ? r0p : r0) + j);
             const float U0s = __fmaf_rn(-lam, C0s, wQ0), U0p = __fmaf_rn(-lam, C0p, wQ0);
             uint64_t K0s = cand_key(C0s, U0s, d0, b), K0p = cand_key(C0p, U0p, d0, b);
             K0s = h0 ? K0s : 0;
@@ -862,8 +873,8 @@ k_seq_chain(Model m, Queries q, int Qs, const float *ctab, float *aux, const flo
             uint64_t K1s = 0, K1p = 0;
             if (HI) {
                 const float wQ1 = __fmul_rn(wq, qs[j * M + m1]);
-                C1s = tab[r1 + j];
-                C1p = tab[(more ? r1p : r1) + j];
+                C1s = at(r1 + j);
+                C1p = at((more ? r1p : r1) + j);
                 U1s = __fmaf_rn(-lam, C1s, wQ1);
                 U1p = __fmaf_rn(-lam, C1p, wQ1);
                 K1s = cand_key(C1s, U1s, d1, b);
@@ -1298,8 +1309,10 @@ cudaError_t simt_prepare() {
     if (e == cudaSuccess) e = opt_in(k_seq_table<2>, big);
     if (e == cudaSuccess) e = opt_in(k_seq_table<4>, big);
     if (e == cudaSuccess) e = opt_in(k_seq_table<8>, big);
-    if (e == cudaSuccess) e = opt_in(k_seq_chain<false>, SEQ_CHAIN_SMEM + 1024);
-    if (e == cudaSuccess) e = opt_in(k_seq_chain<true>, SEQ_CHAIN_SMEM + 1024);
+    if (e == cudaSuccess) e = opt_in(k_seq_chain<false, false>, SEQ_CHAIN_SMEM + 1024);
+    if (e == cudaSuccess) e = opt_in(k_seq_chain<true, false>, SEQ_CHAIN_SMEM + 1024);
+    if (e == cudaSuccess) e = opt_in(k_seq_chain<false, true>, SEQ_CHAIN_SMEM + 1024);
+    if (e == cudaSuccess) e = opt_in(k_seq_chain<true, true>, SEQ_CHAIN_SMEM + 1024);
     if (e == cudaSuccess) e = opt_in(k_route_pairs, big);
     return e;
 }
@@ -1402,8 +1415,10 @@ cudaError_t launch_seq_chain(const Model &m, const Queries &q, int Qs, const flo
     cudaLaunchConfig_t cfg = dependent_launch(1, CHAIN_THREADS, chain_smem(m.D, m.M, Qs), s);
     const SeqAux A = seq_aux(aux, m.D, m.M, Qs);
     if (m.D > 32)
-        return cudaLaunchKernelEx(&cfg, k_seq_chain<true>, m, q, Qs, ctab, aux, (const float *)A.qual, m.M);
-    return cudaLaunchKernelEx(&cfg, k_seq_chain<false>, m, q, Qs, ctab, aux, (const float *)A.qual, m.M);
+        return cudaLaunchKernelEx(&cfg, k_seq_chain<true, false>, m, q, Qs, ctab, aux,
+                                  (const float *)A.qual, m.M, 0);
+    return cudaLaunchKernelEx(&cfg, k_seq_chain<false, false>, m, q, Qs, ctab, aux,
+                              (const float *)A.qual, m.M, 0);
 }
 
 cudaError_t launch_seq_prep_tc(const Model &m, const Queries &q, int Qs, float *aux,
@@ -1415,9 +1430,25 @@ cudaError_t launch_seq_prep_tc(const Model &m, const Queries &q, int Qs, float *
 
 cudaError_t launch_seq_chain_tc(const Model &m, const Queries &q, int Qs, const float *ctab,
                                 float *aux, const float *qual, int qstride, cudaStream_t s) {
-    cudaLaunchConfig_t cfg = dependent_launch(1, CHAIN_THREADS, chain_smem(m.D, m.M, Qs), s);
-    if (m.D > 32) return cudaLaunchKernelEx(&cfg, k_seq_chain<true>, m, q, Qs, ctab, aux, qual, qstride);
-    return cudaLaunchKernelEx(&cfg, k_seq_chain<false>, m, q, Qs, ctab, aux, qual, qstride);
+    if (chain_smem(m.D, m.M, Qs) <= (size_t)SEQ_CHAIN_SMEM) {
+        cudaLaunchConfig_t cfg = dependent_launch(1, CHAIN_THREADS, chain_smem(m.D, m.M, Qs), s);
+        if (m.D > 32)
+            return cudaLaunchKernelEx(&cfg, k_seq_chain<true, false>, m, q, Qs, ctab, aux, qual,
+                                      qstride, 0);
+        return cudaLaunchKernelEx(&cfg, k_seq_chain<false, false>, m, q, Qs, ctab, aux, qual,
+                                  qstride, 0);
+    }
+    // the table's first rows in shared memory, the rest read from L2
+    const size_t rest = chain_smem(m.D, m.M, Qs) - chain_tab_floats(m.D, Qs) * sizeof(float);
+    if (rest + 4 * sizeof(float) > (size_t)SEQ_CHAIN_SMEM) return cudaErrorInvalidValue;
+    const int tsm = (int)(((size_t)SEQ_CHAIN_SMEM - rest) / sizeof(float)) & ~3;
+    cudaLaunchConfig_t cfg =
+        dependent_launch(1, CHAIN_THREADS, rest + (size_t)tsm * sizeof(float), s);
+    if (m.D > 32)
+        return cudaLaunchKernelEx(&cfg, k_seq_chain<true, true>, m, q, Qs, ctab, aux, qual,
+                                  qstride, tsm);
+    return cudaLaunchKernelEx(&cfg, k_seq_chain<false, true>, m, q, Qs, ctab, aux, qual, qstride,
+                              tsm);
 }
 
 }  // namespace hwr

@@ -317,7 +317,7 @@ def _replay_check(p, got):
     return float(np.mean(clear))
 
 
-@pytest.mark.parametrize("c,Q", [(1, 150), (4, 70), (3, 45)])
+@pytest.mark.parametrize("c,Q", [(1, 150), (4, 70), (4, 64), (3, 45), (3, 64)])
 def test_sequential_tensor_table_valid(c, Q):
     p = W.make_config(c, Q=Q)
     r = H.Router(p)
