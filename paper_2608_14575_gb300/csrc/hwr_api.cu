@@ -1298,6 +1298,13 @@ hwr_status hwr_internal_route_tensor_scratch(hwr_ctx *c, int32_t Q, const float 
     int ctas = 0;
     CK(c, launch_mlp_tc(t, q, qual, sp, part, count, c->status_d, c->stream, nullptr, &ctas),
        "predictor kernel");
+    // this predictor may still run when the next tensor-core route starts
+    // early: that route checks its inputs against these outputs
+    const size_t qb4 = (size_t)Q * 4;
+    c->prev_out[0] = {chosen, qb4};
+    c->prev_out[1] = {pred_latency, qb4};
+    c->prev_out[2] = {utility, qb4};
+    c->prev_out[3] = {};
     c->stats.kernel_launches++;
     c->stats.launches[HWR_K_MLP_TC]++;
     c->stats.queries_routed += Q;

@@ -67,6 +67,30 @@ def test_noalloc_matches_route_batch_on_two_calls():
     r.close()
 
 
+def test_route_reading_noalloc_outputs_waits_for_them():
+    """A normal route queued right behind an allocation-free one, reading
+    that call's latencies as its output lengths, must see them complete."""
+    import torch
+    H.build()
+    dev = torch.device("cuda:0")
+    p = W.make_config(4, Q=4096)
+    r = H.Router(p, stream=torch.cuda.current_stream().cuda_stream)
+    il, ol, em = _dev(p, 0, p["Q"], dev)
+    o1, o2 = _outs(p["Q"], dev), _outs(p["Q"], dev)
+    for _ in range(3):
+        r.route_device_noalloc(il, ol, em, *o1, slo=p["slo"], lam=p["lam"], flags=H.HWR_ASYNC)
+        r.route_device(il, o1[1], em, *o2, slo=p["slo"], lam=p["lam"],
+                       flags=H.HWR_PATH_TENSOR | H.HWR_ASYNC)
+    r.synchronize()
+    lat1 = o1[1].clone()
+    o3 = _outs(p["Q"], dev)
+    r.route_device(il, lat1, em, *o3, slo=p["slo"], lam=p["lam"], flags=H.HWR_PATH_TENSOR)
+    torch.cuda.synchronize()
+    for a, b in zip(o2, o3):
+        assert np.array_equal(a.cpu().numpy(), b.cpu().numpy(), equal_nan=True)
+    r.close()
+
+
 def test_noalloc_allocates_nothing_and_rejects_oversize():
     import torch
     H.build()
