@@ -137,6 +137,7 @@ struct hwr_ctx {
     uint16_t *prebf = nullptr; size_t prebf_cap = 0;
     int32_t *dmv = nullptr;  size_t dmv_cap = 0;
     int seq_slots = 0;       // sequential-table blocks resident at once
+    int nsm = 1;             // SMs of the context's device
 
     // I/O staging for host pointers: device [emb | in | out] and [chosen | lat | util]
     char *io_d = nullptr;    size_t io_cap = 0;
@@ -544,6 +545,7 @@ static hwr_status build_ctx(hwr_ctx *c, const hwr_deployment_table *t, const hwr
 
     c->seq_qs = seq_chunk(model_view(c));
     c->seq_slots = seq_table_slots(model_view(c));
+    CK(c, cudaDeviceGetAttribute(&c->nsm, cudaDevAttrMultiProcessorCount, c->device), "SM count");
     CK(c, cudaDeviceSynchronize(), "create");
     return HWR_OK;
 }
@@ -834,7 +836,7 @@ static hwr_status run_kernels(hwr_ctx *c, const Queries &q, uint32_t flags, bool
     }
     LaunchScope a(c, HWR_K_ROUTE_SIMT, prof);
     if ((long)q.Q * c->D <= c->pairs_max)
-        CK(c, launch_route_pairs(m, q, c->pairC, c->pairQ, c->pairH, c->pairN, c->stream),
+        CK(c, launch_route_pairs(m, q, c->pairC, c->pairQ, c->pairH, c->pairN, c->nsm, c->stream),
            "route kernel");
     else
         CK(c, launch_route_simt(m, q, c->stream), "route kernel");

@@ -123,7 +123,7 @@ cudaError_t launch_route_simt(const Model &m, const Queries &q, cudaStream_t s);
 // Reads W2 through m.W2T and layer 1's query columns through m.W1T.
 constexpr int PAIRS_MAX_PAIRS = 2048;   // default upper bound on Q * D for this kernel
 cudaError_t launch_route_pairs(const Model &m, const Queries &q, float *pairC, float *qualS,
-                               float *h2, int32_t *count, cudaStream_t s);
+                               float *h2, int32_t *count, int nsm, cudaStream_t s);
 size_t route_pairs_smem(const Model &m);
 // Sequential mode over one chunk of Qs <= seq_chunk(m) queries: the chunk's
 // standardised features and layer-1 prefixes, and the score table (every

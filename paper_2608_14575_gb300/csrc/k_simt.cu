@@ -953,17 +953,22 @@ k_seq_chain(Model m, Queries q, int Qs, const float *ctab, float *aux, const flo
 // ---------------------------------------------------------------------------
 // K_route_pairs: the small-batch (latency) variant.  The (query, deployment)
 // pairs p = qq D + d are taken in groups of PAIR_G consecutive pairs, and a
-// group's layer 2 is split by columns over ncb = ceil(H2 / PAIR_COLS) blocks:
-// each stages its W2 columns (16-byte async copies) and the group's layer-1
-// rows in shared memory, runs its columns' serial chains (warp w: columns
-// 4w .. 4w + 3, lane: pair, so a W2 load is a broadcast) and stores them to a
-// scratch h2 [groups][H2][PAIR_G].  The last column block of a group (arrival
-// counter, self-resetting) copies the group's h2 block back with 16-byte
-// async copies and runs the head chains and the cost of Eq. 2.
+// group's layer 2 is split by columns over ncb column blocks, in one of two
+// shapes.  Split (PAIR_COLS columns per block, when groups are many): each
+// block stages its W2 columns k-major and the group's layer-1 rows in shared
+// memory, runs its columns' serial chains (warp w: columns 4w .. 4w + 3,
+// lane: pair, so a W2 load is a broadcast) and stores them to a scratch h2
+// [groups][H2][PAIR_G].  Fused (PAIR_FUSED_COLS columns per block, when every
+// block of the grid has an SM of its own, e.g. one query): each block stages
+// its W2 rows, the pairs' deployment prefixes and W1's query columns, and
+// rebuilds every layer-1 unit inside the layer-2 chains (warp w: columns 2w,
+// 2w + 1), storing h2 rows [groups][PAIR_G][H2].  The last column block of a
+// group (arrival counter, self-resetting) copies the group's h2 back with
+// 16-byte async copies and runs the head chains and the cost of Eq. 2.
 // Quality blocks run the per-(query, model) chains from shared memory.  A
 // query is decided by the block that completes its count of D pairs and
 // qblocks quality blocks (self-resetting).  Same canonical order as the
-// kernels above: every chain is the same sequence of roundings.
+// kernels above in both shapes: every chain is the same sequence of roundings.
 
 struct PairArgs {
     float *pairC;       // [Q][D] scratch
@@ -973,11 +978,13 @@ struct PairArgs {
     int32_t *gcount;    // [groups] column-block arrivals, zero between calls
     int qblocks;        // quality blocks per query
     int ncb;            // column blocks per group
+    int cols;           // layer-2 columns per column block: PAIR_FUSED_COLS or PAIR_COLS
 };
 
 constexpr int PAIR_MPB = 8;    // models per quality block
 constexpr int PAIR_G = 32;     // pairs per group
-constexpr int PAIR_COLS = 32;  // layer-2 columns per block
+constexpr int PAIR_COLS = 32;  // layer-2 columns per block, split shape
+constexpr int PAIR_FUSED_COLS = 8;   // layer-2 columns per block, fused shape
 
 __device__ void pair_select(const Model &m, const Queries &q, const PairArgs &a, int qq) {
     // one warp: utility, SLO mask, argmax over the query's stored costs
@@ -1012,160 +1019,449 @@ __device__ void pair_select(const Model &m, const Queries &q, const PairArgs &a,
 
 __host__ __device__ inline int pair_groups(int npair) { return (npair + PAIR_G - 1) / PAIR_G; }
 
+// Shared-memory layout of a fused-shape column block (floats; every region
+// 16-byte aligned), and of the group's last block over the same space.  Rows
+// that a warp reads as 16-byte vectors, one row per lane, have a stride of an
+// odd number of 16-byte units, so that the 8 lanes of each wavefront fall in
+// distinct banks.
+struct PairSmem {
+    int ldk, lda, ld2;          // W2 / W1-column row stride; prefix and layer-2 row strides
+    int w2, as, w1;             // column block: W2 rows, prefix rows, W1's query columns
+    int h2, w3;                 // last block: layer-2 rows, W3
+    int total;
+};
+
+__host__ __device__ inline int odd_units(int n) {   // n rounded up to 4, then to an odd multiple of 4
+    const int r = (n + 3) & ~3;
+    return ((r >> 2) & 1) ? r : r + 4;
+}
+
+__host__ __device__ inline PairSmem pair_smem(int H1, int H2) {
+    PairSmem L;
+    L.ldk = (H1 + 3) & ~3;
+    L.lda = (H1 & 3) == 0 ? odd_units(H1) : H1;
+    L.ld2 = odd_units(H2);
+    int o = 3 * PAIR_G;                     // qu, qv, qo
+    L.w2 = o;
+    o += PAIR_FUSED_COLS * L.ldk;
+    L.as = o;
+    o += (PAIR_G * L.lda + 3) & ~3;
+    L.w1 = o;
+    o += 2 * L.ldk;
+    L.h2 = 3 * PAIR_G;
+    L.w3 = L.h2 + PAIR_G * L.ld2;
+    const int fin = L.w3 + 3 * H2;
+    L.total = o > fin ? o : fin;
+    return L;
+}
+
+// Layers 1 and 2 of pair p (deployment prefix row ar, query slots u, v) for
+// the block's columns c0, c0 + 1: each layer-1 unit is rebuilt where
+// layer 2 consumes it (same two FMAs and ReLU as everywhere), and each
+// layer-2 chain is bias, then k ascending.  Shared-memory operands come as
+// 16-byte vectors, eight k at a time ahead of their FMAs: on this GPU a
+// chain step waiting on its own shared loads costs several times its FMA.
+// Stores relu(h2) into the group's scratch rows [PAIR_G][H2].
+__device__ __forceinline__ void pair_layers(const Model &m, const PairArgs &a, const PairSmem &L,
+                                            const float *w2c, const float *ar, const float *w1s,
+                                            float u, float v, int g, int n0, int nb, int c0,
+                                            int p) {
+    constexpr int NC = 2;
+    const int H1 = m.H1, H2 = m.H2;
+    float acc[NC];
+    const float *wr[NC];
+#pragma unroll
+    for (int j = 0; j < NC; ++j) {
+        const int c = c0 + j;
+        acc[j] = c < nb ? m.b2[n0 + c] : 0.f;
+        wr[j] = w2c + (size_t)(c < nb ? c : 0) * L.ldk;
+    }
+    const float *wi = w1s, *wo = w1s + L.ldk;
+    int k = 0;
+    if ((H1 & 3) == 0) {
+        for (; k + 8 <= H1; k += 8) {
+            const float4 a0 = *reinterpret_cast<const float4 *>(ar + k);
+            const float4 a1 = *reinterpret_cast<const float4 *>(ar + k + 4);
+            const float4 i0 = *reinterpret_cast<const float4 *>(wi + k);
+            const float4 i1 = *reinterpret_cast<const float4 *>(wi + k + 4);
+            const float4 o0 = *reinterpret_cast<const float4 *>(wo + k);
+            const float4 o1 = *reinterpret_cast<const float4 *>(wo + k + 4);
+            float4 w0[NC], w1[NC];
+#pragma unroll
+            for (int j = 0; j < NC; ++j) {
+                w0[j] = *reinterpret_cast<const float4 *>(wr[j] + k);
+                w1[j] = *reinterpret_cast<const float4 *>(wr[j] + k + 4);
+            }
+            const float av[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
+            const float iv[8] = {i0.x, i0.y, i0.z, i0.w, i1.x, i1.y, i1.z, i1.w};
+            const float ov[8] = {o0.x, o0.y, o0.z, o0.w, o1.x, o1.y, o1.z, o1.w};
+            float h[8];
+#pragma unroll
+            for (int t = 0; t < 8; ++t) {
+                const float x = __fmaf_rn(ov[t], v, __fmaf_rn(iv[t], u, av[t]));
+                h[t] = x > 0.f ? x : 0.f;
+            }
+#pragma unroll
+            for (int j = 0; j < NC; ++j) {
+                acc[j] = __fmaf_rn(w0[j].x, h[0], acc[j]);
+                acc[j] = __fmaf_rn(w0[j].y, h[1], acc[j]);
+                acc[j] = __fmaf_rn(w0[j].z, h[2], acc[j]);
+                acc[j] = __fmaf_rn(w0[j].w, h[3], acc[j]);
+                acc[j] = __fmaf_rn(w1[j].x, h[4], acc[j]);
+                acc[j] = __fmaf_rn(w1[j].y, h[5], acc[j]);
+                acc[j] = __fmaf_rn(w1[j].z, h[6], acc[j]);
+                acc[j] = __fmaf_rn(w1[j].w, h[7], acc[j]);
+            }
+        }
+    }
+    for (; k < H1; ++k) {
+        const float x = __fmaf_rn(wo[k], v, __fmaf_rn(wi[k], u, ar[k]));
+        const float h = x > 0.f ? x : 0.f;
+#pragma unroll
+        for (int j = 0; j < NC; ++j) acc[j] = __fmaf_rn(wr[j][k], h, acc[j]);
+    }
+    float *dst = a.h2 + ((size_t)g * PAIR_G + p) * H2 + n0;
+#pragma unroll
+    for (int j = 0; j < NC; ++j)
+        if (c0 + j < nb) dst[c0 + j] = acc[j] > 0.f ? acc[j] : 0.f;
+    __threadfence();   // before the group's arrival
+}
+
+// The decision for each query of a group: its pairs arrive; the warp that
+// completes the query's count (pairs and quality blocks) decides it.
+__device__ __forceinline__ void pair_decide(const Model &m, const Queries &q, const PairArgs &a,
+                                            int p0, int np, int q0, int nq) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, D = m.D;
+    for (int ql = warp; ql < nq; ql += SIMT_THREADS / 32) {
+        const int qq = q0 + ql;
+        const int cnt = min(p0 + np, (qq + 1) * D) - max(p0, qq * D);
+        int done = 0;
+        if (lane == 0) done = atomicAdd(&a.count[qq], cnt) + cnt == D + a.qblocks;
+        done = __shfl_sync(0xffffffffu, done, 0);
+        if (done) {
+            __threadfence();
+            pair_select(m, q, a, qq);
+        }
+    }
+}
+
+// Column block, split shape (many groups): W2 columns n0 .. n0 + 31 k-major,
+// layer 1 written once per (pair, unit), layer-2 chains of 4 columns per warp
+// (lane = pair), h2 scratch [groups][H2][PAIR_G]; the group's last column
+// block runs the heads.
+__device__ __forceinline__ void pair_cols_split(const Model &m, const Queries &q, const PairArgs &a,
+                                             float *sm, int *s_last_p) {
+    int &s_last = *s_last_p;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int F = m.F, H1 = m.H1, H2 = m.H2, D = m.D;
+    const int npair = q.Q * D;
+    const int g = blockIdx.x / a.ncb, cb = blockIdx.x - g * a.ncb;
+    const int p0 = g * PAIR_G, np = min(PAIR_G, npair - p0);
+    const int q0 = p0 / D, nq = (p0 + np - 1) / D - q0 + 1;   // queries touched, <= PAIR_G
+    const int n0 = cb * PAIR_COLS, nb = min(PAIR_COLS, H2 - n0);
+    float *qu = sm, *qv = sm + PAIR_G, *qo = sm + 2 * PAIR_G;
+    float *w2s = sm + 3 * PAIR_G;               // [H1][PAIR_COLS]
+    const int ld1 = H1 | 1;                     // odd: rows of 4 pairs in distinct banks
+    float *h1s = w2s + (size_t)H1 * PAIR_COLS;  // [PAIR_G][ld1]
+    // W2 columns n0 .. n0 + 31 of every k (only within the padded row)
+    {
+        const int c4n = min(PAIR_COLS, m.H2p - n0) >> 2;
+        const uint32_t base = (uint32_t)__cvta_generic_to_shared(w2s);
+        for (int e = tid; e < H1 * c4n; e += SIMT_THREADS) {
+            const int k = e / c4n, c4 = e - k * c4n;
+            asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(
+                             base + (uint32_t)(4 * (k * PAIR_COLS + 4 * c4))),
+                         "l"(__cvta_generic_to_global(m.W2T + (size_t)k * m.H2p + n0 + 4 * c4)) : "memory");
+        }
+        asm volatile("cp.async.commit_group;" ::: "memory");
+    }
+    // the query slots of the group's queries (fp64 chains side by side)
+    if (tid < nq) {
+        qu[tid] = standardise(m.xform[F - 2], (double)q.in_len[q0 + tid], m.mu[F - 2], m.sd[F - 2]);
+    } else if (tid >= 32 && tid < 32 + nq) {
+        const float o = q.out_len[q0 + tid - 32];
+        qv[tid - 32] = standardise(m.xform[F - 1], (double)o, m.mu[F - 1], m.sd[F - 1]);
+        qo[tid - 32] = o;
+    }
+    // this thread's unit k of layer 1 for every pair of the group: the
+    // prefix loads first, all in flight together
+    const int k = tid;
+    const bool hk = k < H1;
+    float av[PAIR_G];
+    {
+        int qq = q0, d = p0 - q0 * D;
+#pragma unroll
+        for (int p = 0; p < PAIR_G; ++p) {
+            av[p] = hk && p < np ? m.A[(size_t)d * H1 + k] : 0.f;
+            if (++d == D) {
+                d = 0;
+                ++qq;
+            }
+        }
+    }
+    const float wi = hk ? m.W1T[(size_t)(F - 2) * H1 + k] : 0.f;
+    const float wo = hk ? m.W1T[(size_t)(F - 1) * H1 + k] : 0.f;
+    __syncthreads();
+    if (hk) {
+        int ql = 0, d = p0 - q0 * D;
+#pragma unroll
+        for (int p = 0; p < PAIR_G; ++p) {
+            if (p < np) {
+                float x = __fmaf_rn(wi, qu[ql], av[p]);
+                x = __fmaf_rn(wo, qv[ql], x);
+                h1s[p * ld1 + k] = x > 0.f ? x : 0.f;
+            }
+            if (++d == D) {
+                d = 0;
+                ++ql;
+            }
+        }
+    }
+    asm volatile("cp.async.wait_all;" ::: "memory");
+    __syncthreads();
+    // layer 2: thread (pair p = lane, columns c .. c + 3 of warp w), serial over k
+    {
+        const int p = lane, c = 4 * warp;
+        if (p < np && c < nb) {
+            float acc[4];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) acc[j] = c + j < nb ? m.b2[n0 + c + j] : 0.f;
+            const float *hr = h1s + p * ld1;
+            const float *wr = w2s + c;
+#pragma unroll 8
+            for (int kk = 0; kk < H1; ++kk) {
+                const float4 w = *reinterpret_cast<const float4 *>(wr + kk * PAIR_COLS);
+                const float h = hr[kk];
+                acc[0] = __fmaf_rn(w.x, h, acc[0]);
+                acc[1] = __fmaf_rn(w.y, h, acc[1]);
+                acc[2] = __fmaf_rn(w.z, h, acc[2]);
+                acc[3] = __fmaf_rn(w.w, h, acc[3]);
+            }
+            float *dst = a.h2 + ((size_t)g * H2 + n0 + c) * PAIR_G + p;
+#pragma unroll
+            for (int j = 0; j < 4; ++j)
+                if (c + j < nb) dst[j * PAIR_G] = acc[j] > 0.f ? acc[j] : 0.f;
+            __threadfence();   // before the group's arrival below
+        }
+    }
+    __syncthreads();
+    if (tid == 0) {
+        __threadfence();
+        s_last = atomicAdd(&a.gcount[g], 1) == a.ncb - 1;
+    }
+    __syncthreads();
+    if (!s_last) return;
+    // the group's last column block: heads and cost of every pair
+    __threadfence();
+    float *h2s = w2s;                            // [H2][PAIR_G]
+    float *w3s = h2s + (size_t)H2 * PAIR_G;      // [NH][H2]
+    {
+        // the group's whole block (rows of pairs past np are not read),
+        // L2 to shared memory by 16-byte copies that skip L1
+        const uint32_t base = (uint32_t)__cvta_generic_to_shared(h2s);
+        const float *src = a.h2 + (size_t)g * H2 * PAIR_G;
+        for (int e = tid; e < H2 * PAIR_G / 4; e += SIMT_THREADS)
+            asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(base + 16u * e),
+                         "l"(__cvta_generic_to_global(src + 4 * e)) : "memory");
+        asm volatile("cp.async.commit_group;" ::: "memory");
+    }
+    for (int i = tid; i < m.NH * H2; i += SIMT_THREADS) w3s[i] = m.W3[i];
+    asm volatile("cp.async.wait_all;" ::: "memory");
+    __syncthreads();
+    __shared__ float hd[PAIR_G * 3];
+    if (warp < m.NH) {
+        // head o = warp of pair p = lane: W3 reads are broadcasts, h2
+        // reads consecutive words
+        const int o = warp, p = lane;
+        const float *w3 = w3s + (size_t)o * H2;
+        float z = m.b3[o];
+#pragma unroll 8
+        for (int n = 0; n < H2; ++n) z = __fmaf_rn(w3[n], h2s[n * PAIR_G + p], z);
+        if (p < np) hd[p * m.NH + o] = softplus_c(z);
+    }
+    __syncthreads();
+    for (int p = tid; p < np; p += SIMT_THREADS) {
+        const int qq = (p0 + p) / D, NH = m.NH;
+        a.pairC[p0 + p] =
+            __fmaf_rn(NH == 3 ? hd[p * NH + 2] : qo[qq - q0], hd[p * NH + 1], hd[p * NH]);
+    }
+    if (tid == 0) a.gcount[g] = 0;
+    __threadfence();
+    __syncthreads();
+    pair_decide(m, q, a, p0, np, q0, nq);
+}
+
+// Column block, fused shape (few groups, so that every block has an SM of
+// its own): the block's 8 W2 rows, each pair's deployment prefix row and
+// W1's query columns staged by asynchronous copies behind the query slots'
+// loads; each layer-1 unit rebuilt where layer 2 consumes it (no layer-1
+// pass); h2 scratch [groups][PAIR_G][H2], a row per pair, so that the last
+// block's head chains read it as vectors.
+__device__ __forceinline__ void pair_cols_fused(const Model &m, const Queries &q, const PairArgs &a,
+                                             float *sm, int *s_last_p) {
+    int &s_last = *s_last_p;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int F = m.F, H1 = m.H1, H2 = m.H2, D = m.D;
+    const int npair = q.Q * D;
+    const int g = blockIdx.x / a.ncb, cb = blockIdx.x - g * a.ncb;
+    const int p0 = g * PAIR_G, np = min(PAIR_G, npair - p0);
+    const int q0 = p0 / D, nq = (p0 + np - 1) / D - q0 + 1;   // queries touched, <= PAIR_G
+    const int cols = a.cols, n0 = cb * cols, nb = min(cols, H2 - n0);
+    const PairSmem L = pair_smem(H1, H2);
+    float *qu = sm, *qv = sm + PAIR_G, *qo = sm + 2 * PAIR_G;
+    float *w2c = sm + L.w2;    // [cols][ldk]: W2 rows n0 .. n0 + cols - 1
+    float *as = sm + L.as;     // [PAIR_G][lda]: each pair's deployment prefix
+    float *w1s = sm + L.w1;    // [2][ldk]: W1's two query columns
+    // the query slots' raw lengths first: their double-precision chains below
+    // are this block's longest wait
+    float iv = 0.f, ov = 0.f;
+    if (tid < nq) iv = q.in_len[q0 + tid];
+    else if (tid >= 32 && tid < 32 + nq) ov = q.out_len[q0 + tid - 32];
+    {
+        // pair p of the group is deployment (p0 + p) mod D; 16-byte copies
+        // where the rows allow, else 4-byte ones
+        const uint32_t wb = (uint32_t)__cvta_generic_to_shared(w2c);
+        const uint32_t ab = (uint32_t)__cvta_generic_to_shared(as);
+        const int d0 = p0 - q0 * D;
+        if ((H1 & 3) == 0) {
+            const int r4 = H1 >> 2;
+            for (int e = tid; e < nb * r4; e += SIMT_THREADS) {
+                const int c = e / r4, j = e - c * r4;
+                asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(
+                                 wb + (uint32_t)(4 * (c * L.ldk + 4 * j))),
+                             "l"(__cvta_generic_to_global(m.W2 + (size_t)(n0 + c) * H1 + 4 * j)) : "memory");
+            }
+            for (int e = tid; e < np * r4; e += SIMT_THREADS) {
+                const int p = e / r4, j = e - p * r4;
+                int d = d0 + p;
+                d -= (d / D) * D;
+                asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(
+                                 ab + (uint32_t)(4 * (p * L.lda + 4 * j))),
+                             "l"(__cvta_generic_to_global(m.A + (size_t)d * H1 + 4 * j)) : "memory");
+            }
+        } else {
+            for (int e = tid; e < nb * H1; e += SIMT_THREADS) {
+                const int c = e / H1, j = e - c * H1;
+                asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(
+                                 wb + (uint32_t)(4 * (c * L.ldk + j))),
+                             "l"(__cvta_generic_to_global(m.W2 + (size_t)(n0 + c) * H1 + j)) : "memory");
+            }
+            for (int e = tid; e < np * H1; e += SIMT_THREADS) {
+                const int p = e / H1, j = e - p * H1;
+                int d = d0 + p;
+                d -= (d / D) * D;
+                asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(
+                                 ab + (uint32_t)(4 * (p * L.lda + j))),
+                             "l"(__cvta_generic_to_global(m.A + (size_t)d * H1 + j)) : "memory");
+            }
+        }
+        const uint32_t w1b = (uint32_t)__cvta_generic_to_shared(w1s);
+        for (int e = tid; e < 2 * H1; e += SIMT_THREADS) {
+            const int r = e / H1, j = e - r * H1;
+            asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(
+                             w1b + (uint32_t)(4 * (r * L.ldk + j))),
+                         "l"(__cvta_generic_to_global(m.W1T + (size_t)(F - 2 + r) * H1 + j)) : "memory");
+        }
+        asm volatile("cp.async.commit_group;" ::: "memory");
+    }
+    // the query slots of the group's queries (fp64 chains side by side)
+    if (tid < nq) {
+        qu[tid] = standardise(m.xform[F - 2], (double)iv, m.mu[F - 2], m.sd[F - 2]);
+    } else if (tid >= 32 && tid < 32 + nq) {
+        qv[tid - 32] = standardise(m.xform[F - 1], (double)ov, m.mu[F - 1], m.sd[F - 1]);
+        qo[tid - 32] = ov;
+    }
+    asm volatile("cp.async.wait_all;" ::: "memory");
+    __syncthreads();
+    // layers 1 and 2: lane = pair p, warp w = columns 2w, 2w + 1
+    if (lane < np && 2 * warp < nb) {
+        const int p = lane, ql = (p0 + p) / D - q0;
+        pair_layers(m, a, L, w2c, as + (size_t)p * L.lda, w1s, qu[ql], qv[ql], g, n0, nb,
+                    2 * warp, p);
+    }
+    __syncthreads();
+    if (tid == 0) {
+        __threadfence();
+        s_last = atomicAdd(&a.gcount[g], 1) == a.ncb - 1;
+    }
+    __syncthreads();
+    if (!s_last) return;
+    // the group's last column block: heads and cost of every pair
+    __threadfence();
+    float *h2s = sm + L.h2;     // [PAIR_G][ld2]: layer 2, a row per pair
+    float *w3s = sm + L.w3;     // [NH][H2]
+    {
+        // the group's rows, L2 to shared memory by copies that skip L1
+        const float *src = a.h2 + (size_t)g * PAIR_G * H2;
+        if ((H2 & 3) == 0) {
+            const uint32_t base = (uint32_t)__cvta_generic_to_shared(h2s);
+            const int r4 = H2 >> 2;
+            for (int e = tid; e < np * r4; e += SIMT_THREADS) {
+                const int p = e / r4, j = e - p * r4;
+                asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(
+                                 base + (uint32_t)(4 * (p * L.ld2 + 4 * j))),
+                             "l"(__cvta_generic_to_global(src + (size_t)p * H2 + 4 * j)) : "memory");
+            }
+            asm volatile("cp.async.commit_group;" ::: "memory");
+        } else {
+            for (int e = tid; e < np * H2; e += SIMT_THREADS) {
+                const int p = e / H2, j = e - p * H2;
+                h2s[p * L.ld2 + j] = __ldcg(src + (size_t)p * H2 + j);
+            }
+        }
+    }
+    for (int i = tid; i < m.NH * H2; i += SIMT_THREADS) w3s[i] = m.W3[i];
+    asm volatile("cp.async.wait_all;" ::: "memory");
+    __syncthreads();
+    __shared__ float hd[PAIR_G * 3];
+    if (warp < m.NH && lane < np) {
+        // head o = warp, pair p = lane: W3 reads are broadcasts, each lane
+        // reads its own row of layer 2, four n per vector
+        const int o = warp, p = lane;
+        const float *w3 = w3s + (size_t)o * H2, *hr = h2s + (size_t)p * L.ld2;
+        float z = m.b3[o];
+        int n = 0;
+        if ((H2 & 3) == 0) {
+            for (; n + 8 <= H2; n += 8) {
+                const float4 h0 = *reinterpret_cast<const float4 *>(hr + n);
+                const float4 h1 = *reinterpret_cast<const float4 *>(hr + n + 4);
+                const float4 v0 = *reinterpret_cast<const float4 *>(w3 + n);
+                const float4 v1 = *reinterpret_cast<const float4 *>(w3 + n + 4);
+                z = __fmaf_rn(v0.x, h0.x, z);
+                z = __fmaf_rn(v0.y, h0.y, z);
+                z = __fmaf_rn(v0.z, h0.z, z);
+                z = __fmaf_rn(v0.w, h0.w, z);
+                z = __fmaf_rn(v1.x, h1.x, z);
+                z = __fmaf_rn(v1.y, h1.y, z);
+                z = __fmaf_rn(v1.z, h1.z, z);
+                z = __fmaf_rn(v1.w, h1.w, z);
+            }
+        }
+        for (; n < H2; ++n) z = __fmaf_rn(w3[n], hr[n], z);
+        hd[p * m.NH + o] = softplus_c(z);
+    }
+    __syncthreads();
+    for (int p = tid; p < np; p += SIMT_THREADS) {
+        const int qq = (p0 + p) / D, NH = m.NH;
+        a.pairC[p0 + p] =
+            __fmaf_rn(NH == 3 ? hd[p * NH + 2] : qo[qq - q0], hd[p * NH + 1], hd[p * NH]);
+    }
+    if (tid == 0) a.gcount[g] = 0;
+    __threadfence();
+    __syncthreads();
+    pair_decide(m, q, a, p0, np, q0, nq);
+}
+
 __global__ void __launch_bounds__(SIMT_THREADS) k_route_pairs(Model m, Queries q, PairArgs a) {
-    extern __shared__ float4 sm4[];   // 16-byte aligned: W2 columns arrive as 16-byte copies
+    extern __shared__ float4 sm4[];   // 16-byte aligned: operands arrive as 16-byte copies
     float *sm = reinterpret_cast<float *>(sm4);
     __shared__ int s_last;
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const int F = m.F, H1 = m.H1, H2 = m.H2, D = m.D, M = m.M;
+    const int tid = threadIdx.x;
+    const int D = m.D, M = m.M;
     const int npair = q.Q * D, ncolb = pair_groups(npair) * a.ncb;
     if ((int)blockIdx.x < ncolb) {
-        const int g = blockIdx.x / a.ncb, cb = blockIdx.x - g * a.ncb;
-        const int p0 = g * PAIR_G, np = min(PAIR_G, npair - p0);
-        const int q0 = p0 / D, nq = (p0 + np - 1) / D - q0 + 1;   // queries touched, <= PAIR_G
-        const int n0 = cb * PAIR_COLS, nb = min(PAIR_COLS, H2 - n0);
-        float *qu = sm, *qv = sm + PAIR_G, *qo = sm + 2 * PAIR_G;
-        float *w2s = sm + 3 * PAIR_G;               // [H1][PAIR_COLS]
-        const int ld1 = H1 | 1;                     // odd: rows of 4 pairs in distinct banks
-        float *h1s = w2s + (size_t)H1 * PAIR_COLS;  // [PAIR_G][ld1]
-        // W2 columns n0 .. n0 + 31 of every k (only within the padded row)
-        {
-            const int c4n = min(PAIR_COLS, m.H2p - n0) >> 2;
-            const uint32_t base = (uint32_t)__cvta_generic_to_shared(w2s);
-            for (int e = tid; e < H1 * c4n; e += SIMT_THREADS) {
-                const int k = e / c4n, c4 = e - k * c4n;
-                asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(
-                                 base + (uint32_t)(4 * (k * PAIR_COLS + 4 * c4))),
-                             "l"(__cvta_generic_to_global(m.W2T + (size_t)k * m.H2p + n0 + 4 * c4)) : "memory");
-            }
-            asm volatile("cp.async.commit_group;" ::: "memory");
-        }
-        // the query slots of the group's queries (fp64 chains side by side)
-        if (tid < nq) {
-            qu[tid] = standardise(m.xform[F - 2], (double)q.in_len[q0 + tid], m.mu[F - 2], m.sd[F - 2]);
-        } else if (tid >= 32 && tid < 32 + nq) {
-            const float o = q.out_len[q0 + tid - 32];
-            qv[tid - 32] = standardise(m.xform[F - 1], (double)o, m.mu[F - 1], m.sd[F - 1]);
-            qo[tid - 32] = o;
-        }
-        // this thread's unit k of layer 1 for every pair of the group: the
-        // prefix loads first, all in flight together
-        const int k = tid;
-        const bool hk = k < H1;
-        float av[PAIR_G];
-        {
-            int qq = q0, d = p0 - q0 * D;
-#pragma unroll
-            for (int p = 0; p < PAIR_G; ++p) {
-                av[p] = hk && p < np ? m.A[(size_t)d * H1 + k] : 0.f;
-                if (++d == D) {
-                    d = 0;
-                    ++qq;
-                }
-            }
-        }
-        const float wi = hk ? m.W1T[(size_t)(F - 2) * H1 + k] : 0.f;
-        const float wo = hk ? m.W1T[(size_t)(F - 1) * H1 + k] : 0.f;
-        __syncthreads();
-        if (hk) {
-            int ql = 0, d = p0 - q0 * D;
-#pragma unroll
-            for (int p = 0; p < PAIR_G; ++p) {
-                if (p < np) {
-                    float x = __fmaf_rn(wi, qu[ql], av[p]);
-                    x = __fmaf_rn(wo, qv[ql], x);
-                    h1s[p * ld1 + k] = x > 0.f ? x : 0.f;
-                }
-                if (++d == D) {
-                    d = 0;
-                    ++ql;
-                }
-            }
-        }
-        asm volatile("cp.async.wait_all;" ::: "memory");
-        __syncthreads();
-        // layer 2: thread (pair p = lane, columns c .. c + 3 of warp w), serial over k
-        {
-            const int p = lane, c = 4 * warp;
-            if (p < np && c < nb) {
-                float acc[4];
-#pragma unroll
-                for (int j = 0; j < 4; ++j) acc[j] = c + j < nb ? m.b2[n0 + c + j] : 0.f;
-                const float *hr = h1s + p * ld1;
-                const float *wr = w2s + c;
-#pragma unroll 8
-                for (int kk = 0; kk < H1; ++kk) {
-                    const float4 w = *reinterpret_cast<const float4 *>(wr + kk * PAIR_COLS);
-                    const float h = hr[kk];
-                    acc[0] = __fmaf_rn(w.x, h, acc[0]);
-                    acc[1] = __fmaf_rn(w.y, h, acc[1]);
-                    acc[2] = __fmaf_rn(w.z, h, acc[2]);
-                    acc[3] = __fmaf_rn(w.w, h, acc[3]);
-                }
-                float *dst = a.h2 + ((size_t)g * H2 + n0 + c) * PAIR_G + p;
-#pragma unroll
-                for (int j = 0; j < 4; ++j)
-                    if (c + j < nb) dst[j * PAIR_G] = acc[j] > 0.f ? acc[j] : 0.f;
-                __threadfence();   // before the group's arrival below
-            }
-        }
-        __syncthreads();
-        if (tid == 0) {
-            __threadfence();
-            s_last = atomicAdd(&a.gcount[g], 1) == a.ncb - 1;
-        }
-        __syncthreads();
-        if (!s_last) return;
-        // the group's last column block: heads and cost of every pair
-        __threadfence();
-        float *h2s = w2s;                            // [H2][PAIR_G]
-        float *w3s = h2s + (size_t)H2 * PAIR_G;      // [NH][H2]
-        {
-            // the group's whole block (rows of pairs past np are not read),
-            // L2 to shared memory by 16-byte copies that skip L1
-            const uint32_t base = (uint32_t)__cvta_generic_to_shared(h2s);
-            const float *src = a.h2 + (size_t)g * H2 * PAIR_G;
-            for (int e = tid; e < H2 * PAIR_G / 4; e += SIMT_THREADS)
-                asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(base + 16u * e),
-                             "l"(__cvta_generic_to_global(src + 4 * e)) : "memory");
-            asm volatile("cp.async.commit_group;" ::: "memory");
-        }
-        for (int i = tid; i < m.NH * H2; i += SIMT_THREADS) w3s[i] = m.W3[i];
-        asm volatile("cp.async.wait_all;" ::: "memory");
-        __syncthreads();
-        __shared__ float hd[PAIR_G * 3];
-        if (warp < m.NH) {
-            // head o = warp of pair p = lane: W3 reads are broadcasts, h2
-            // reads consecutive words
-            const int o = warp, p = lane;
-            const float *w3 = w3s + (size_t)o * H2;
-            float z = m.b3[o];
-#pragma unroll 8
-            for (int n = 0; n < H2; ++n) z = __fmaf_rn(w3[n], h2s[n * PAIR_G + p], z);
-            if (p < np) hd[p * m.NH + o] = softplus_c(z);
-        }
-        __syncthreads();
-        for (int p = tid; p < np; p += SIMT_THREADS) {
-            const int qq = (p0 + p) / D, NH = m.NH;
-            a.pairC[p0 + p] =
-                __fmaf_rn(NH == 3 ? hd[p * NH + 2] : qo[qq - q0], hd[p * NH + 1], hd[p * NH]);
-        }
-        if (tid == 0) a.gcount[g] = 0;
-        __threadfence();
-        __syncthreads();
-        // each query of the group: its pairs arrive; the warp that completes
-        // the query's count decides it
-        for (int ql = warp; ql < nq; ql += SIMT_THREADS / 32) {
-            const int qq = q0 + ql;
-            const int cnt = min(p0 + np, (qq + 1) * D) - max(p0, qq * D);
-            int done = 0;
-            if (lane == 0) done = atomicAdd(&a.count[qq], cnt) + cnt == D + a.qblocks;
-            done = __shfl_sync(0xffffffffu, done, 0);
-            if (done) {
-                __threadfence();
-                pair_select(m, q, a, qq);
-            }
-        }
+        if (a.cols == PAIR_COLS) pair_cols_split(m, q, a, sm, &s_last);
+        else pair_cols_fused(m, q, a, sm, &s_last);
         return;
     }
     // quality of models [m0, m0 + PAIR_MPB) for one query
@@ -1197,13 +1493,18 @@ __global__ void __launch_bounds__(SIMT_THREADS) k_route_pairs(Model m, Queries q
         const float4 *c = reinterpret_cast<const float4 *>(mb) + tid;
         const float4 *e4 = reinterpret_cast<const float4 *>(er);
         float s = 0.f;
-#pragma unroll 4
-        for (int k4 = 0; k4 < E / 4; ++k4) {
-            const float4 x = e4[k4], y = c[(size_t)k4 * mn];
-            s = __fmaf_rn(x.x, y.x, s);
-            s = __fmaf_rn(x.y, y.y, s);
-            s = __fmaf_rn(x.z, y.z, s);
-            s = __fmaf_rn(x.w, y.w, s);
+        // E is a multiple of 8: two 4-term groups' operands, then their FMAs
+        for (int k4 = 0; k4 < E / 4; k4 += 2) {
+            const float4 x0 = e4[k4], y0 = c[(size_t)k4 * mn];
+            const float4 x1 = e4[k4 + 1], y1 = c[(size_t)(k4 + 1) * mn];
+            s = __fmaf_rn(x0.x, y0.x, s);
+            s = __fmaf_rn(x0.y, y0.y, s);
+            s = __fmaf_rn(x0.z, y0.z, s);
+            s = __fmaf_rn(x0.w, y0.w, s);
+            s = __fmaf_rn(x1.x, y1.x, s);
+            s = __fmaf_rn(x1.y, y1.y, s);
+            s = __fmaf_rn(x1.z, y1.z, s);
+            s = __fmaf_rn(x1.w, y1.w, s);
         }
         a.qualS[(size_t)qq * M + m0 + tid] = sigmoid_c(s);
         __threadfence();
@@ -1337,16 +1638,17 @@ cudaError_t launch_route_simt(const Model &m, const Queries &q, cudaStream_t s) 
 }
 
 size_t route_pairs_smem(const Model &m) {
-    const size_t cols = 3 * PAIR_G + (size_t)m.H1 * PAIR_COLS + (size_t)PAIR_G * (m.H1 | 1);
+    const size_t fused = (size_t)pair_smem(m.H1, m.H2).total;
+    const size_t split = 3 * PAIR_G + (size_t)m.H1 * PAIR_COLS + (size_t)PAIR_G * (m.H1 | 1);
     const size_t fin = 3 * PAIR_G + (size_t)m.H2 * PAIR_G + (size_t)m.NH * m.H2;
+    size_t blk = fused > split ? fused : split;
+    blk = blk > fin ? blk : fin;
     const size_t qual = (size_t)m.E * (1 + PAIR_MPB);
-    size_t f = cols > fin ? cols : fin;
-    f = f > qual ? f : qual;
-    return f * sizeof(float);
+    return (blk > qual ? blk : qual) * sizeof(float);
 }
 
 cudaError_t launch_route_pairs(const Model &m, const Queries &q, float *pairC, float *qualS,
-                               float *h2, int32_t *count, cudaStream_t s) {
+                               float *h2, int32_t *count, int nsm, cudaStream_t s) {
     if (q.Q <= 0) return cudaSuccess;
     if ((long)q.Q * m.D > PAIRS_MAX_PAIRS) return cudaErrorInvalidValue;
     PairArgs a;
@@ -1356,7 +1658,17 @@ cudaError_t launch_route_pairs(const Model &m, const Queries &q, float *pairC, f
     a.count = count;
     a.gcount = count + PAIRS_MAX_PAIRS;
     a.qblocks = (m.M + PAIR_MPB - 1) / PAIR_MPB;
-    a.ncb = (m.H2 + PAIR_COLS - 1) / PAIR_COLS;
+    // The fused shape, 8 columns per block, when the whole grid still has an
+    // SM per block: a layer-2 chain step there waits mostly on its shared
+    // loads, so narrower blocks (fewer chains sharing an SM's shared memory)
+    // finish sooner; with more groups the split shape's 32 columns per block
+    // keep the grid to one wave.
+    const int groups = pair_groups(q.Q * m.D);
+    a.cols = (long)groups * ((m.H2 + PAIR_FUSED_COLS - 1) / PAIR_FUSED_COLS) +
+                         (long)q.Q * a.qblocks <= nsm
+                 ? PAIR_FUSED_COLS
+                 : PAIR_COLS;
+    a.ncb = (m.H2 + a.cols - 1) / a.cols;
     const int blocks = pair_groups(q.Q * m.D) * a.ncb + q.Q * a.qblocks;
     k_route_pairs<<<blocks, SIMT_THREADS, route_pairs_smem(m), s>>>(m, q, a);
     return cudaGetLastError();
@@ -1452,3 +1764,4 @@ cudaError_t launch_seq_chain_tc(const Model &m, const Queries &q, int Qs, const 
 }
 
 }  // namespace hwr
+
