@@ -297,6 +297,34 @@ def test_pairs_kernel_group_shapes_exact(monkeypatch, shape, Q):
     assert np.array_equal(C, Cw.astype(np.float32))
 
 
+# the small-batch kernel's fused column blocks (8 columns, taken when every
+# block of the grid has an SM of its own): H1 with a 4-wide tail (92), H1 not
+# a multiple of 4 (37), H2 with a ragged last block and an odd head row (30,
+# 45), a query straddling two groups (D = 15), every query spanning two groups
+# (D = 64), and the sweep's cluster (D = 32, H = 256) at one and four queries
+@pytest.mark.parametrize("shape,Q", [
+    (dict(M=5, G=3, F=24, H1=92, H2=30, E=40), 3),
+    (dict(M=3, G=2, F=20, H1=37, H2=45, E=16), 9),
+    (dict(M=16, G=4, F=48, H1=64, H2=64, E=32), 2),
+    ("cfg4", 1),
+    ("cfg4", 4),
+])
+def test_pairs_kernel_fused_shapes_exact(monkeypatch, shape, Q):
+    monkeypatch.setenv("HWR_PAIRS_MAX_PAIRS", "2048")
+    if shape == "cfg4":
+        p = W.make_config(4, Q=Q)
+    else:
+        p = W.make_problem(Q=Q, dtype="f32", lam=0.3, slo=3.0, seed=47, bias_std=0.2, **shape)
+    r = H.Router(p)
+    got = r.route()
+    C, qual = r.score()
+    r.close()
+    orc = O.Problem(p)
+    assert_exact(got, orc.route(mode=O.F32, nthreads=8), str(shape))
+    Cw, _ = orc.score_all(mode=O.F32, nthreads=8)
+    assert np.array_equal(C, Cw.astype(np.float32))
+
+
 # ---------------------------------------------------------------------------
 # sequential mode on more shapes: D > 32 (two deployments per lane of the
 # chain's warp), odd D, D = 1, a bf16 context, several chunks each
