@@ -15,6 +15,8 @@
 #include <string>
 #include <vector>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "hwr_internal.cuh"
 
 using namespace hwr;
@@ -22,6 +24,16 @@ using namespace hwr;
 namespace {
 
 thread_local std::string g_create_error;
+
+// An NVTX range over one API call: a profiler that records NVTX (Nsight
+// Systems, for one) shows each call on the calling thread's timeline; with
+// none attached a push / pop costs a few nanoseconds.
+struct ApiRange {
+    explicit ApiRange(const char *name) { nvtxRangePushA(name); }
+    ~ApiRange() { nvtxRangePop(); }
+    ApiRange(const ApiRange &) = delete;
+    ApiRange &operator=(const ApiRange &) = delete;
+};
 
 // Host-side fault hooks for tests, read at hwr_create: HWR_TEST_FAIL_ALLOC=n
 // makes the n-th allocation of the context (counting from 1) report failure;
@@ -579,6 +591,7 @@ static void free_ctx(hwr_ctx *c) {
 extern "C" hwr_status hwr_create(const hwr_deployment_table *table, const hwr_predictor *pred,
                                  const void *model_emb, int32_t E, hwr_dtype emb_dtype,
                                  void *cuda_stream, hwr_ctx **out) {
+    ApiRange range_("hwr_create");
     if (!out) return fail(nullptr, HWR_ERR_INVALID_ARG, "out is NULL");
     *out = nullptr;
     g_create_error.clear();
@@ -625,6 +638,7 @@ extern "C" hwr_status hwr_create(const hwr_deployment_table *table, const hwr_pr
 }
 
 extern "C" hwr_status hwr_destroy(hwr_ctx *c) {
+    ApiRange range_("hwr_destroy");
     if (c) free_ctx(c);
     return HWR_OK;
 }
@@ -633,6 +647,7 @@ extern "C" hwr_status hwr_destroy(hwr_ctx *c) {
 // snapshot
 
 extern "C" hwr_status hwr_update_snapshot(hwr_ctx *c, const hwr_snapshot *s) {
+    ApiRange range_("hwr_update_snapshot");
     if (!c) return fail(nullptr, HWR_ERR_INVALID_ARG, "ctx is NULL");
     if (c->broken) return HWR_ERR_STATE;
     if (!s || !s->running || !s->waiting || !s->kv_util || !s->gpu_util || !s->ttft_avg ||
@@ -677,6 +692,7 @@ extern "C" hwr_status hwr_update_snapshot(hwr_ctx *c, const hwr_snapshot *s) {
 }
 
 extern "C" hwr_status hwr_get_snapshot(hwr_ctx *c, int32_t *running_out) {
+    ApiRange range_("hwr_get_snapshot");
     if (!c) return fail(nullptr, HWR_ERR_INVALID_ARG, "ctx is NULL");
     if (c->broken) return HWR_ERR_STATE;
     if (!running_out) return fail(c, HWR_ERR_INVALID_ARG, "running_out is NULL");
@@ -1166,6 +1182,7 @@ extern "C" hwr_status hwr_route_batch(hwr_ctx *c, int32_t Q, const float *in_len
                                       const float *out_len, const void *q_emb, float slo,
                                       float lambda, uint32_t flags, int32_t *chosen,
                                       float *pred_latency, float *utility) {
+    ApiRange range_("hwr_route_batch");
     return route_impl(c, Q, in_len, out_len, q_emb, slo, nullptr, lambda, flags, chosen,
                       pred_latency, utility);
 }
@@ -1173,6 +1190,7 @@ extern "C" hwr_status hwr_route_batch(hwr_ctx *c, int32_t Q, const float *in_len
 extern "C" hwr_status hwr_score_batch(hwr_ctx *c, int32_t Q, const float *in_len,
                                       const float *out_len, const void *q_emb, uint32_t flags,
                                       float *cost, float *quality) {
+    ApiRange range_("hwr_score_batch");
     if (!c) return fail(nullptr, HWR_ERR_INVALID_ARG, "ctx is NULL");
     if (!cost && !quality) return fail(c, HWR_ERR_INVALID_ARG, "cost and quality both NULL");
     ScoreOut so{cost, quality};
@@ -1185,6 +1203,7 @@ extern "C" hwr_status hwr_route_batch_multi(hwr_ctx *c, int32_t Q, const float *
                                             const float *lambdas, int32_t K, uint32_t flags,
                                             int32_t *chosen, float *pred_latency,
                                             float *utility) {
+    ApiRange range_("hwr_route_batch_multi");
     if (!c) return fail(nullptr, HWR_ERR_INVALID_ARG, "ctx is NULL");
     if (!lambdas) return fail(c, HWR_ERR_INVALID_ARG, "lambdas is NULL");
     if (K < 1 || K > MAX_LAMBDAS)
@@ -1204,6 +1223,7 @@ extern "C" hwr_status hwr_route_batch_slo(hwr_ctx *c, int32_t Q, const float *in
                                           const float *out_len, const void *q_emb,
                                           const hwr_slo_spec *slo, float lambda, uint32_t flags,
                                           int32_t *chosen, float *pred_latency, float *utility) {
+    ApiRange range_("hwr_route_batch_slo");
     if (!c) return fail(nullptr, HWR_ERR_INVALID_ARG, "ctx is NULL");
     if (!slo) return fail(c, HWR_ERR_INVALID_ARG, "slo specification is NULL");
     return route_impl(c, Q, in_len, out_len, q_emb, 0.0f, slo, lambda, flags, chosen,
@@ -1211,6 +1231,7 @@ extern "C" hwr_status hwr_route_batch_slo(hwr_ctx *c, int32_t Q, const float *in
 }
 
 extern "C" hwr_status hwr_synchronize(hwr_ctx *c) {
+    ApiRange range_("hwr_synchronize");
     if (!c) return fail(nullptr, HWR_ERR_INVALID_ARG, "ctx is NULL");
     if (c->broken) return HWR_ERR_STATE;
     CK(c, cudaStreamSynchronize(c->stream), "synchronize");
