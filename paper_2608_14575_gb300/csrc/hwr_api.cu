@@ -1078,18 +1078,26 @@ static hwr_status route_impl(hwr_ctx *c, int32_t Q, const float *in_len, const f
         if (small && SQ)
             CK(c, cudaMemcpyAsync(SQ + (size_t)lo * c->M, c->pairQ, n * rowQ,
                                   cudaMemcpyDeviceToDevice, c->stream), "copy quality");
-        if (tensor && SQ)
+        // the selection over several lambdas reads the tensor path's quality
+        // buffer itself (rows of Mpad); only scoring copies it out
+        const float *selQ = SQ ? SQ + (size_t)lo * c->M : nullptr;
+        int qstride = c->M;
+        if (tensor && SQ && so)
             CK(c, cudaMemcpy2DAsync(SQ + (size_t)lo * c->M, rowQ, c->qual_last, (size_t)c->Mpad * 4,
                                     rowQ, n, cudaMemcpyDeviceToDevice, c->stream),
                "copy quality");
+        if (tensor && SQ && !so) {
+            selQ = c->qual_last;
+            qstride = c->Mpad;
+        }
         if (!ml) return HWR_OK;
         Queries qs = qc;
         qs.chosen = q.chosen + lo;
         qs.lat = q.lat + lo;
         qs.util = q.util + lo;
         LaunchScope ls(c, HWR_K_ROUTE_SIMT, flags & HWR_PROFILE);
-        CK(c, launch_select_multi(mv, qs, SC + (size_t)lo * c->D, SQ + (size_t)lo * c->M, c->M,
-                                  *ml, Q, c->stream), "select kernel");
+        CK(c, launch_select_multi(mv, qs, SC + (size_t)lo * c->D, selQ, qstride, *ml, Q,
+                                  c->stream), "select kernel");
         ls.done();
         return HWR_OK;
     };
