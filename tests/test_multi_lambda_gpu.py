@@ -148,3 +148,43 @@ def test_pair_kernel_rows_equal_oracle(monkeypatch, c, Q):
         _exact_row(got, k, orc.route(lam=float(lam), mode=O.F32, nthreads=8), f"cfg{c} lambda={lam}")
     Cw, _ = orc.score_all(mode=O.F32, nthreads=8)
     assert np.array_equal(C, Cw.astype(np.float32))
+
+
+# the selection kernel's lane map (lane l: deployments l and l + 32) on
+# clusters of 1, 15, 33 and 64 deployments, and exact ties (every model's
+# quality 0.5 and only the GPU one-hot and the query lengths feeding layer 1:
+# deployments of one GPU type tie exactly and the lowest index must win)
+@pytest.mark.parametrize("shape", [
+    dict(M=1, G=1, F=12, H1=8, H2=8, E=8),
+    dict(M=5, G=3, F=24, H1=40, H2=24, E=16),
+    dict(M=11, G=3, F=24, H1=32, H2=36, E=24),
+    dict(M=16, G=4, F=48, H1=32, H2=32, E=16),
+])
+def test_selection_lane_map_rows_exact(shape):
+    p = W.make_problem(Q=150, dtype="f32", lam=0.3, slo=3.0, seed=53, bias_std=0.2, **shape)
+    r = H.Router(p)
+    got = r.route_multi(LAMS)
+    r.close()
+    orc = O.Problem(p)
+    for k, lam in enumerate(LAMS):
+        _exact_row(got, k, orc.route(lam=float(lam), mode=O.F32, nthreads=8), f"{shape} lambda={lam}")
+
+
+@pytest.mark.parametrize("slo", [float("inf"), float("-inf")])
+def test_selection_exact_ties_rows(slo):
+    M, G, F = 16, 4, 48
+    p = W.make_problem(Q=60, dtype="f32", M=M, G=G, F=F, H1=32, H2=32, E=16, seed=9,
+                       lam=0.4, slo=2.0, bias_std=0.3)
+    keep = np.zeros(F, bool)
+    keep[M:M + G] = True
+    keep[F - 2:] = True
+    p["W1"] = np.where(keep[None, :], p["W1"], 0.0).astype(p["W1"].dtype)
+    p["memb"] = np.zeros_like(p["memb"])
+    r = H.Router(p)
+    got = r.route_multi(LAMS, slo=slo)
+    r.close()
+    orc = O.Problem(p)
+    for k, lam in enumerate(LAMS):
+        _exact_row(got, k, orc.route(slo=slo, lam=float(lam), mode=O.F32, nthreads=8),
+                   f"ties slo={slo} lambda={lam}")
+        assert np.all((got[0][k] >= 0) & (got[0][k] < G))
