@@ -241,15 +241,22 @@ __device__ __forceinline__ void tile_sync() {
     asm volatile("bar.sync 1, %0;" ::"n"(SIMT_THREADS) : "memory");
 }
 
+// n rounded up to a multiple of 4, then to an odd multiple of 4: rows of
+// this stride, read by a warp as 16-byte vectors (one row per lane), fall in
+// distinct banks across each wavefront's 8 lanes.
+__host__ __device__ constexpr int odd_units(int n) {
+    return (((n + 3) & ~3) >> 2) & 1 ? (n + 3) & ~3 : ((n + 3) & ~3) + 4;
+}
+
 __host__ __device__ constexpr int tile_width(int H2) {
     return H2 <= 32 ? 32 : H2 <= 64 ? 64 : H2 <= 128 ? 128 : 256;
 }
 
 __host__ __device__ constexpr size_t tile_floats_for(int H2) {
     return (size_t)SIMT_KC * TILE_ROWS + 2 * (size_t)SIMT_KC * tile_width(H2) >
-                   (size_t)TILE_ROWS * (H2 + 1)
+                   (size_t)TILE_ROWS * odd_units(H2)
                ? (size_t)SIMT_KC * TILE_ROWS + 2 * (size_t)SIMT_KC * tile_width(H2)
-               : (size_t)TILE_ROWS * (H2 + 1);
+               : (size_t)TILE_ROWS * odd_units(H2);
 }
 
 // Rows k0 .. k0 + kc - 1 of W2 transposed into dst [kc][W] by 16-byte
@@ -386,7 +393,7 @@ __device__ void pair_mlp(const Model &m, int R, const Rows &rows, const float *u
     }
 
     float *h2s = tile;
-    const int ld = H2 + 1;
+    const int ld = odd_units(H2);
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
         const int r = 8 * warp + i;
@@ -401,10 +408,30 @@ __device__ void pair_mlp(const Model &m, int R, const Rows &rows, const float *u
     }
     tile_sync();
     for (int e = tid; e < m.NH * R; e += SIMT_THREADS) {
+        // head chain o of row r, n ascending: eight n of operands as 16-byte
+        // vectors before their FMAs (a chain step waiting on its own shared
+        // loads costs several times its FMA)
         const int r = e / m.NH, o = e - r * m.NH;
-        const float *w3 = w3s + (size_t)o * H2;
+        const float *w3 = w3s + (size_t)o * H2, *hr = h2s + (size_t)r * ld;
         float z = m.b3[o];
-        for (int n = 0; n < H2; ++n) z = __fmaf_rn(w3[n], h2s[r * ld + n], z);
+        int n = 0;
+        if ((H2 & 3) == 0) {
+            for (; n + 8 <= H2; n += 8) {
+                const float4 h0 = *reinterpret_cast<const float4 *>(hr + n);
+                const float4 h1 = *reinterpret_cast<const float4 *>(hr + n + 4);
+                const float4 v0 = *reinterpret_cast<const float4 *>(w3 + n);
+                const float4 v1 = *reinterpret_cast<const float4 *>(w3 + n + 4);
+                z = __fmaf_rn(v0.x, h0.x, z);
+                z = __fmaf_rn(v0.y, h0.y, z);
+                z = __fmaf_rn(v0.z, h0.z, z);
+                z = __fmaf_rn(v0.w, h0.w, z);
+                z = __fmaf_rn(v1.x, h1.x, z);
+                z = __fmaf_rn(v1.y, h1.y, z);
+                z = __fmaf_rn(v1.z, h1.z, z);
+                z = __fmaf_rn(v1.w, h1.w, z);
+            }
+        }
+        for (; n < H2; ++n) z = __fmaf_rn(w3[n], hr[n], z);
         sp[e] = softplus_c(z);
     }
     tile_sync();
@@ -441,6 +468,7 @@ __host__ __device__ inline RouteLayout route_layout(int D, int M, int H2) {
     L.sp = o; o += 3 * 64;
     L.C = o; o += 64;
     L.U = o; o += 64;
+    o = (o + 3) & ~(size_t)3;   // W3 rows read as 16-byte vectors
     L.w3 = o; o += 3 * (size_t)H2;
     L.w1q = o; o += 2 * (size_t)MAX_H;
     o = (o + 3) & ~(size_t)3;
@@ -665,6 +693,7 @@ __host__ __device__ inline SeqLayout seq_layout(int H2) {
     L.gi = o; o += TILE_ROWS;
     L.qi = o; o += TILE_ROWS;
     L.sp = o; o += 3 * TILE_ROWS;
+    o = (o + 3) & ~(size_t)3;   // W3 rows read as 16-byte vectors
     L.w3 = o; o += 3 * (size_t)H2;
     L.w1q = o; o += 2 * (size_t)MAX_H;
     o = (o + 3) & ~(size_t)3;
@@ -1030,11 +1059,6 @@ struct PairSmem {
     int h2, w3;                 // last block: layer-2 rows, W3
     int total;
 };
-
-__host__ __device__ inline int odd_units(int n) {   // n rounded up to 4, then to an odd multiple of 4
-    const int r = (n + 3) & ~3;
-    return ((r >> 2) & 1) ? r : r + 4;
-}
 
 __host__ __device__ inline PairSmem pair_smem(int H1, int H2) {
     PairSmem L;
